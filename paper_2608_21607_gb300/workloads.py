@@ -1,0 +1,251 @@
+"""Seeded synthetic inputs for the SALSA block sweep.
+
+This module only *generates* inputs: the sparse nonnegative matrix S (CSR) and
+the initial factors W (m x r) and H (r x n).  It contains none of the solver's
+arithmetic, so the fp64 oracle and the CUDA path can both consume it without
+sharing any part of the method.
+
+The paper's datasets (MNIST similarities, the FlyWire connectome, Wikipedia
+bigrams; Sec. 2.5, Table 1) are not available, so every workload is a seeded
+stand-in with the structure the paper describes:
+
+* ``planted``     -- S = max(0, U V^T - tau), a thresholded low-rank matrix
+                     (Def. 2 / Prop. 1 of Sec. 2.1: it admits an exact
+                     completion of rank d+1).
+* ``identity``    -- S = I_n (Corollary "ident", Sec. 2.2: rank-3 completion).
+* ``connectome``  -- a directed graph with power-law out-degree (exponent 2.2,
+                     mean 20) and integer log-normal synapse counts, shaped
+                     like the connectome of Table 1 (139k x 139k, sparse).
+
+All random draws come from numpy's PCG64 with explicit seeds, so both sides of
+every parity test see bit-identical inputs.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Optional
+
+import numpy as np
+
+__all__ = [
+    "CSR", "Workload", "csr_from_dense", "planted", "identity", "connectome",
+    "init_factors", "workload", "WORKLOADS",
+]
+
+
+@dataclasses.dataclass
+class CSR:
+    """Compressed sparse rows: ``row_ptr`` (int64, m+1), ``col_idx`` (int32,
+    strictly increasing within a row), ``vals`` (float32 or float64, > 0)."""
+    m: int
+    n: int
+    row_ptr: np.ndarray
+    col_idx: np.ndarray
+    vals: np.ndarray
+
+    @property
+    def nnz(self) -> int:
+        return int(self.row_ptr[-1])
+
+    def todense(self, dtype=np.float64) -> np.ndarray:
+        d = np.zeros((self.m, self.n), dtype=dtype)
+        rows = np.repeat(np.arange(self.m), np.diff(self.row_ptr))
+        d[rows, self.col_idx] = self.vals
+        return d
+
+
+@dataclasses.dataclass
+class Workload:
+    name: str
+    S: CSR
+    r: int
+    W0: np.ndarray            # m x r, float32
+    H0: np.ndarray            # r x n, float32
+    block_rows: int
+    block_cols: int
+    schedule: str             # "exact" | "stoch"
+    sweeps: int
+    eta: float
+    gamma: float
+    seed: int
+    info: dict
+
+    @property
+    def m(self) -> int:
+        return self.S.m
+
+    @property
+    def n(self) -> int:
+        return self.S.n
+
+
+def csr_from_dense(D: np.ndarray, dtype=np.float32) -> CSR:
+    """CSR of the strictly positive entries of a dense array."""
+    m, n = D.shape
+    mask = D > 0
+    counts = mask.sum(axis=1)
+    row_ptr = np.zeros(m + 1, dtype=np.int64)
+    np.cumsum(counts, out=row_ptr[1:])
+    rows, cols = np.nonzero(mask)
+    return CSR(m, n, row_ptr, cols.astype(np.int32), D[rows, cols].astype(dtype))
+
+
+def init_factors(m: int, n: int, r: int, seed: int, sigma: float = 0.1):
+    """W (m x r) and H (r x n) iid N(0, sigma^2), float32."""
+    rng = np.random.default_rng([seed, 0xF0C7])
+    W = (sigma * rng.standard_normal((m, r))).astype(np.float32)
+    H = (sigma * rng.standard_normal((r, n))).astype(np.float32)
+    return W, H
+
+
+def _csr_from_rows(m, n, row_cols, row_vals, dtype) -> CSR:
+    counts = np.fromiter((len(c) for c in row_cols), dtype=np.int64, count=m)
+    row_ptr = np.zeros(m + 1, dtype=np.int64)
+    np.cumsum(counts, out=row_ptr[1:])
+    col_idx = np.concatenate(row_cols).astype(np.int32) if m else np.zeros(0, np.int32)
+    vals = np.concatenate(row_vals).astype(dtype) if m else np.zeros(0, dtype)
+    return CSR(m, n, row_ptr, col_idx, vals)
+
+
+def planted(m: int = 600, n: int = 400, d: int = 4, tau: Optional[float] = 0.5,
+            density: Optional[float] = None, noise: float = 0.0, seed: int = 0,
+            dtype=np.float32, chunk: int = 2048):
+    """S = max(0, U V^T - tau) with U (m x d), V (n x d) iid N(0,1).
+
+    If ``density`` is given, tau is the empirical (1-density) quantile of
+    U_i . V_j over 10^6 seeded (i, j) pairs.  If ``noise`` > 0 every positive
+    entry is multiplied by (1 + noise * N(0,1)).  Returns (S, U, V, tau).
+    The product is formed in fp64 so that the support does not depend on the
+    host's BLAS.
+    """
+    rng = np.random.default_rng([seed, 0x5EED])
+    U = rng.standard_normal((m, d))
+    V = rng.standard_normal((n, d))
+    if density is not None:
+        k = 1_000_000
+        ii = rng.integers(0, m, size=k)
+        jj = rng.integers(0, n, size=k)
+        samp = np.einsum("kd,kd->k", U[ii], V[jj])
+        tau = float(np.quantile(samp, 1.0 - density))
+    rows_cols, rows_vals = [], []
+    for r0 in range(0, m, chunk):
+        L = U[r0:r0 + chunk] @ V.T - tau
+        for row in L:
+            c = np.nonzero(row > 0)[0]
+            rows_cols.append(c)
+            rows_vals.append(row[c])
+    S = _csr_from_rows(m, n, rows_cols, rows_vals, np.float64)
+    if noise > 0:
+        nrng = np.random.default_rng([seed, 0x0015E])
+        S.vals = S.vals * (1.0 + noise * nrng.standard_normal(S.nnz))
+        S.vals = np.maximum(S.vals, np.finfo(np.float32).tiny)
+    S.vals = S.vals.astype(dtype)
+    return S, U, V, tau
+
+
+def identity(n: int = 4096, dtype=np.float32) -> CSR:
+    """S = I_n in CSR (n nonzeros of value 1)."""
+    return CSR(n, n, np.arange(n + 1, dtype=np.int64), np.arange(n, dtype=np.int32),
+               np.ones(n, dtype=dtype))
+
+
+def connectome(n: int = 139255, mean_degree: float = 20.0, exponent: float = 2.2,
+               seed: int = 0, dtype=np.float32) -> CSR:
+    """Directed graph shaped like the fly connectome of Table 1.
+
+    Out-degree d_i = min(n-1, floor(x_min * u^(-1/(exponent-1)))), u ~ U(0,1],
+    a discrete power law with tail exponent ``exponent``; x_min is tuned by
+    bisection on the realised degrees so that their mean is ``mean_degree``.
+    Targets are uniform without replacement over the other n-1 nodes (no
+    self-loops); values are synapse counts ceil(exp(1 + N(0,1))).
+    """
+    rng = np.random.default_rng([seed, 0xC0EC7])
+    u = 1.0 - rng.random(n)                       # (0, 1]
+    base = u ** (-1.0 / (exponent - 1.0))
+    cap = n - 1
+
+    def mean_for(xm):
+        return np.minimum(cap, np.floor(xm * base)).mean()
+
+    lo, hi = 0.0, 2.0 * mean_degree
+    for _ in range(100):
+        mid = 0.5 * (lo + hi)
+        if mean_for(mid) >= mean_degree:
+            hi = mid
+        else:
+            lo = mid
+    x_min = hi
+    deg = np.minimum(cap, np.floor(x_min * base)).astype(np.int64)
+
+    rows_cols, rows_vals = [], []
+    for i in range(n):
+        d = int(deg[i])
+        if d == 0:
+            rows_cols.append(np.zeros(0, np.int64))
+            rows_vals.append(np.zeros(0, np.float64))
+            continue
+        if 2 * d > cap:
+            c = rng.permutation(cap)[:d]
+        else:
+            got = np.zeros(0, np.int64)
+            while got.size < d:
+                k = d - got.size
+                cand = np.concatenate([got, rng.integers(0, cap, size=k + k // 8 + 8)])
+                _, first = np.unique(cand, return_index=True)
+                first.sort()
+                got = cand[first[:d]]
+            c = got
+        c = np.where(c >= i, c + 1, c)
+        v = np.ceil(np.exp(1.0 + rng.standard_normal(d)))
+        o = np.argsort(c, kind="stable")
+        rows_cols.append(c[o])
+        rows_vals.append(v[o])
+    S = _csr_from_rows(n, n, rows_cols, rows_vals, dtype)
+    return S
+
+
+# ---------------------------------------------------------------------------
+# Named workloads.  ``scale`` shrinks the large ones (same generator and
+# structure) for parity tests the oracle finishes in seconds.
+# ---------------------------------------------------------------------------
+
+def _planted_tiny(seed=0, r=4, **kw):
+    S, U, V, tau = planted(600, 400, 4, tau=0.5, seed=seed)
+    W, H = init_factors(S.m, S.n, r, seed)
+    return Workload("planted-600x400-r%d" % r, S, r, W, H, 128, 128, "exact", 20, 1.0, 0.0,
+                    seed, {"tau": tau, "d": 4})
+
+
+def _identity(seed=0, n=4096, r=3, block=512, **kw):
+    S = identity(n)
+    W, H = init_factors(n, n, r, seed)
+    return Workload("identity-%d-r%d" % (n, r), S, r, W, H, block, block, "stoch", 200,
+                    1.0, 0.9, seed, {})
+
+
+def _planted_medium(seed=0, n=20000, r=32, block=2048, **kw):
+    S, U, V, tau = planted(n, n, 32, tau=None, density=0.05, noise=0.01, seed=seed)
+    W, H = init_factors(n, n, r, seed)
+    return Workload("planted-%dx%d-r%d" % (n, n, r), S, r, W, H, block, block, "stoch", 50,
+                    1.0, 0.9, seed, {"tau": tau, "d": 32})
+
+
+def _connectome(seed=0, n=139255, r=64, block=4096, sweeps=10, **kw):
+    S = connectome(n, seed=seed)
+    W, H = init_factors(n, n, r, seed)
+    return Workload("connectome-%d-r%d" % (n, r), S, r, W, H, block, block, "stoch", sweeps,
+                    1.0, 0.9, seed, {})
+
+
+WORKLOADS = {
+    "planted_tiny": _planted_tiny,
+    "identity": _identity,
+    "planted_medium": _planted_medium,
+    "connectome_r64": lambda seed=0, **kw: _connectome(seed, r=64, block=4096, sweeps=10, **kw),
+    "connectome_r256": lambda seed=0, **kw: _connectome(seed, r=256, block=8192, sweeps=5, **kw),
+}
+
+
+def workload(name: str, seed: int = 0, **kw) -> Workload:
+    return WORKLOADS[name](seed=seed, **kw)

@@ -1,0 +1,324 @@
+"""Pins of the fp64 oracle against what the paper and mathematics fix.
+
+Each test checks the oracle through a route other than its own code: a
+published test vector, a textbook factorisation, a library least-squares
+solve on a dense brute-force problem, a closed-form zero-loss point from the
+paper, or an invariant the paper proves.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+
+import oracle as O
+from paper_2608_21607_gb300 import workloads as WL
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _read_numbers(name):
+    rows = []
+    for line in open(os.path.join(GOLDEN, name)):
+        line = line.strip()
+        if line and not line.startswith("#"):
+            rows.append([float(x) if "." in x or "e" in x else int(x) for x in line.split()])
+    return rows
+
+
+def _rand_sparse(m, n, density, seed):
+    rng = np.random.default_rng(seed)
+    D = np.where(rng.random((m, n)) < density, rng.random((m, n)) + 0.1, 0.0)
+    return WL.csr_from_dense(D, dtype=np.float64), D
+
+
+# --------------------------------------------------------------------------
+# block order
+# --------------------------------------------------------------------------
+
+def test_splitmix64_reference_vector():
+    expect = [row[0] for row in _read_numbers("splitmix64_seed1234567.txt")]
+    g = O.SplitMix64(1234567)
+    assert [g.next() for _ in range(5)] == expect
+
+
+def test_block_permutation_is_a_seeded_permutation():
+    for K in (1, 2, 8, 34, 157):
+        p = O.block_permutation(0, 0, 0, K)
+        assert sorted(p) == list(range(K))
+        assert p == O.block_permutation(0, 0, 0, K)
+    a = O.block_permutation(0, 0, O.ROW, 34)
+    assert a != O.block_permutation(0, 1, O.ROW, 34)
+    assert a != O.block_permutation(0, 0, O.COL, 34)
+    assert a != O.block_permutation(1, 0, O.ROW, 34)
+
+
+def test_block_permutation_golden():
+    """Regression against permutations written by tests/golden/make_golden.py."""
+    for row in _read_numbers("block_order.txt"):
+        seed, sweep, side, K = row[:4]
+        assert O.block_permutation(seed, sweep, side, K) == row[4:]
+
+
+def test_fisher_yates_uniform_small():
+    """All 3! orders of 3 blocks appear with roughly equal frequency."""
+    counts = {}
+    for s in range(6000):
+        p = tuple(O.block_permutation(7, s, 0, 3))
+        counts[p] = counts.get(p, 0) + 1
+    assert len(counts) == 6
+    assert min(counts.values()) > 850 and max(counts.values()) < 1150
+
+
+# --------------------------------------------------------------------------
+# Z update (eq. updateZ) and the Delta identity (eq. updateD)
+# --------------------------------------------------------------------------
+
+def test_update_z_constraints_and_delta_identity():
+    rng = np.random.default_rng(1)
+    S = np.where(rng.random((30, 20)) < 0.2, rng.random((30, 20)) + 0.05, 0.0)
+    L = rng.standard_normal((30, 20))
+    Z = O.update_z(S, L)
+    sup = S > 0
+    assert np.array_equal(Z[sup], S[sup])            # S = max(0, Z) on the support
+    assert np.all(Z[~sup] <= 0)                        # and Z <= 0 off it
+    assert np.array_equal(np.maximum(0, Z), S)
+    Shat = np.maximum(0, L)
+    delta = sup * (S + Shat - L) - Shat                # eq. updateD
+    np.testing.assert_allclose(Z - L, delta, rtol=0, atol=1e-15)
+    # Z minimises ||Z - L|| subject to max(0, Z) = S, entry by entry:
+    for z, l, s in zip(Z.ravel(), L.ravel(), S.ravel()):
+        cands = [s] if s > 0 else [min(0.0, l), 0.0, -abs(l) - 1.0]
+        assert abs(z - l) <= min(abs(c - l) for c in cands) + 1e-15
+
+
+# --------------------------------------------------------------------------
+# dense linear algebra
+# --------------------------------------------------------------------------
+
+def test_cholesky_textbook_example():
+    rows = _read_numbers("cholesky_textbook.txt")
+    G = np.array(rows[:3], dtype=float)
+    C = np.array(rows[3:], dtype=float)
+    np.testing.assert_allclose(O.cholesky(G), C, atol=1e-14)
+
+
+def test_cholesky_and_solve_against_library():
+    rng = np.random.default_rng(2)
+    for r in (1, 3, 16, 64):
+        Q = rng.standard_normal((3 * r + 5, r))
+        G = Q.T @ Q
+        C = O.cholesky(G)
+        np.testing.assert_allclose(C, np.linalg.cholesky(G), rtol=1e-10, atol=1e-12)
+        R = rng.standard_normal((40, r))
+        X = O.solve_normal(C, R)
+        np.testing.assert_allclose(X, np.linalg.solve(G, R.T).T, rtol=1e-9, atol=1e-10)
+
+
+def test_cholesky_rejects_non_spd():
+    with pytest.raises(O.NotSPD):
+        O.cholesky(np.array([[1.0, 2.0], [2.0, 1.0]]))
+    with pytest.raises(O.NotSPD):
+        O.cholesky(np.zeros((3, 3)))
+
+
+# --------------------------------------------------------------------------
+# block updates against dense brute force (lstsq on the explicit Z)
+# --------------------------------------------------------------------------
+
+def _bruteforce_update(D, A, B, side, block, kind, opts, EA, EB):
+    """Dense restatement: pick the sub-problem, build Z, solve with lstsq."""
+    m, n = D.shape
+    A, B, EA, EB = A.copy(), B.copy(), EA.copy(), EB.copy()
+    if side == O.ROW:
+        i0, i1 = O.block_range(block, opts.block_rows, m)
+        if kind == O.EXACT:
+            Z = O.update_z(D[i0:i1], A[i0:i1] @ B.T)
+            X = np.linalg.lstsq(B, Z.T, rcond=None)[0].T       # argmin ||Z - X B^T||
+            A[i0:i1] += opts.eta * (X - A[i0:i1])
+        else:
+            Z = O.update_z(D[i0:i1].T, B @ A[i0:i1].T)         # n x |I|
+            X = np.linalg.lstsq(A[i0:i1], Z.T, rcond=None)[0].T
+            EB[:] = opts.eta * (X - B) + opts.gamma * EB
+            B += EB
+    else:
+        j0, j1 = O.block_range(block, opts.block_cols, n)
+        if kind == O.EXACT:
+            Z = O.update_z(D[:, j0:j1].T, B[j0:j1] @ A.T)
+            X = np.linalg.lstsq(A, Z.T, rcond=None)[0].T
+            B[j0:j1] += opts.eta * (X - B[j0:j1])
+        else:
+            Z = O.update_z(D[:, j0:j1], A @ B[j0:j1].T)
+            X = np.linalg.lstsq(B[j0:j1], Z.T, rcond=None)[0].T
+            EA[:] = opts.eta * (X - A) + opts.gamma * EA
+            A += EA
+    return A, B, EA, EB
+
+
+@pytest.mark.parametrize("side", [O.ROW, O.COL])
+@pytest.mark.parametrize("kind", [O.EXACT, O.STOCH])
+def test_block_update_matches_dense_bruteforce(side, kind):
+    S, D = _rand_sparse(13, 11, 0.3, 3)
+    rng = np.random.default_rng(4)
+    r = 3
+    W = rng.standard_normal((13, r))
+    H = rng.standard_normal((r, 11))
+    opts = O.Options(block_rows=5, block_cols=4, eta=0.7, gamma=0.5)
+    st = O.State(S, W, H, opts)
+    st.EA[:] = 0.01 * rng.standard_normal(st.EA.shape)
+    st.EB[:] = 0.01 * rng.standard_normal(st.EB.shape)
+    nb = O.num_blocks(13 if side == O.ROW else 11, 5 if side == O.ROW else 4)
+    for block in range(nb):                            # includes the ragged last block
+        A, B, EA, EB = _bruteforce_update(D, st.A, st.B, side, block, kind, opts, st.EA, st.EB)
+        st.block_update(side, block, kind)
+        np.testing.assert_allclose(st.A, A, rtol=1e-10, atol=1e-11)
+        np.testing.assert_allclose(st.B, B, rtol=1e-10, atol=1e-11)
+        np.testing.assert_allclose(st.EA, EA, rtol=1e-10, atol=1e-11)
+        np.testing.assert_allclose(st.EB, EB, rtol=1e-10, atol=1e-11)
+
+
+def test_stochastic_full_batch_equals_parallel():
+    """A mini-batch covering every column with eta=1, gamma=0 is plain ALS (eq. lsqA)."""
+    S, _ = _rand_sparse(20, 15, 0.25, 5)
+    W, H = WL.init_factors(20, 15, 4, 0)
+    a = O.State(S, W, H, O.Options(block_rows=20, block_cols=15, eta=1.0, gamma=0.0))
+    b = O.State(S, W, H, O.Options(block_rows=20, block_cols=15, eta=1.0, gamma=0.0))
+    a.block_update(O.COL, 0, O.STOCH)
+    b.block_update(O.ROW, 0, O.EXACT)
+    np.testing.assert_allclose(a.A, b.A, rtol=1e-12, atol=1e-13)
+
+
+# --------------------------------------------------------------------------
+# properties the paper proves
+# --------------------------------------------------------------------------
+
+def test_exact_halfsteps_never_increase_objective():
+    """Sec. 3.2: each alternating minimisation step lowers ||Z - L||."""
+    S, _, _, _ = WL.planted(60, 50, 4, tau=0.5, seed=1)
+    W, H = WL.init_factors(60, 50, 4, 1)
+    st = O.State(S, W, H, O.Options(block_rows=16, block_cols=16, schedule=O.EXACT))
+    prev = st.loss()["obj"]
+    for _ in range(3):
+        for side, block, kind in st.sweep_steps():
+            st.block_update(side, block, kind)
+            cur = st.loss()["obj"]
+            assert cur <= prev * (1 + 1e-12) + 1e-15
+            prev = cur
+        st.sweep_index += 1
+
+
+def test_exact_row_blocks_are_order_independent():
+    """Sec. 4.1: row blocks of A are independent given B."""
+    S, _, _, _ = WL.planted(50, 40, 3, tau=0.3, seed=2)
+    W, H = WL.init_factors(50, 40, 3, 2)
+    a = O.State(S, W, H, O.Options(block_rows=8, block_cols=8, schedule=O.EXACT))
+    b = O.State(S, W, H, O.Options(block_rows=8, block_cols=8, schedule=O.EXACT))
+    K = O.num_blocks(50, 8)
+    for blk in range(K):
+        a.block_update(O.ROW, blk, O.EXACT)
+    for blk in O.block_permutation(9, 3, 0, K):
+        b.block_update(O.ROW, blk, O.EXACT)
+    assert np.array_equal(a.A, b.A)
+
+
+def _planted_exact(m, n, d, tau, seed):
+    """S = max(0, U V^T - tau) in fp64 and its rank-(d+1) completion [U, 1][V, -tau]^T."""
+    S, U, V, _ = WL.planted(m, n, d, tau=tau, seed=seed, dtype=np.float64)
+    W0 = np.hstack([U, np.ones((m, 1))])
+    H0 = np.hstack([V, -tau * np.ones((n, 1))]).T
+    return S, W0, H0
+
+
+@pytest.mark.parametrize("schedule", [O.EXACT, O.STOCH])
+def test_planted_completion_is_zero_loss_fixed_point(schedule):
+    """Prop. 1 (Sec. 2.1): a thresholded rank-d matrix has a rank-(d+1) completion."""
+    S, W0, H0 = _planted_exact(70, 50, 4, 0.5, 3)
+    # blocks of 16 rows and 10 columns: every block (the ragged last one too)
+    # has at least r = 5 rows, so each block Gram matrix is nonsingular
+    st = O.State(S, W0, H0, O.Options(block_rows=16, block_cols=10, schedule=schedule,
+                                      eta=1.0, gamma=0.9))
+    l0 = st.loss()
+    assert l0["obj"] < 1e-14 and l0["rmse"] < 1e-14 and l0["wjd"] < 1e-14
+    st.sweep()
+    np.testing.assert_allclose(st.A, W0, atol=1e-11)
+    np.testing.assert_allclose(st.B, H0.T, atol=1e-11)
+    assert st.loss()["obj"] < 1e-12
+
+
+def _omega_factors(n):
+    th = 2 * np.pi * np.arange(n) / n
+    c = np.cos(2 * np.pi / n)
+    W = np.stack([np.cos(th), np.sin(th), -c * np.ones(n)], 1) / (1 - c)
+    H = np.stack([np.cos(th), np.sin(th), np.ones(n)], 1).T
+    return W, H
+
+
+def test_identity_has_rank3_completion_omega():
+    """Corollary 'ident' (eq. Omega): I_n = max(0, Omega), rank(Omega) <= 3."""
+    n = 64
+    W, H = _omega_factors(n)
+    Om = W @ H
+    i, j = np.meshgrid(np.arange(n), np.arange(n), indexing="ij")
+    c = np.cos(2 * np.pi / n)
+    np.testing.assert_allclose(Om, (np.cos(2 * np.pi * (i - j) / n) - c) / (1 - c), atol=1e-10)
+    np.testing.assert_allclose(np.maximum(0, Om), np.eye(n), atol=1e-9)
+    # Corollary 'nuclear': ||Omega||_* = n (1 + |cos phi|) / (1 - cos phi)
+    nuc = np.linalg.svd(Om, compute_uv=False).sum()
+    assert nuc == pytest.approx(n * (1 + abs(c)) / (1 - c), rel=1e-10)
+    S = WL.identity(n, dtype=np.float64)
+    st = O.State(S, W, H, O.Options(block_rows=16, block_cols=16, eta=1.0, gamma=0.9))
+    assert st.loss()["obj"] < 1e-9
+    st.sweep()
+    assert st.loss()["obj"] < 1e-8
+    np.testing.assert_allclose(st.A @ st.B.T, Om, atol=1e-7)
+
+
+def test_loss_of_all_zero_model_is_one():
+    """Sec. 3.1: RMSE(S, 0) = WJD(S, 0) = 1; with L = 0, Z = S so the objective is 1 too."""
+    S, _ = _rand_sparse(20, 30, 0.2, 6)
+    l = O.loss(O.Sparse.from_csr(S), np.zeros((20, 3)), np.zeros((30, 3)))
+    assert l["obj"] == pytest.approx(1.0) and l["rmse"] == pytest.approx(1.0)
+    assert l["wjd"] == pytest.approx(1.0)
+
+
+def test_loss_definitions_bruteforce_and_lipschitz():
+    """eq. SLloss equals ||Z - L||^2; eq. RMSE / WJD written densely; obj >= RMSE (Prop. 'Lipschitz')."""
+    S, D = _rand_sparse(17, 23, 0.3, 7)
+    rng = np.random.default_rng(8)
+    A = rng.standard_normal((17, 4))
+    B = rng.standard_normal((23, 4))
+    L = A @ B.T
+    sl = np.sum(np.where(D == 0, np.maximum(0, L) ** 2, 0)) + np.sum(np.where(D > 0, (D - L) ** 2, 0))
+    Shat = np.maximum(0, L)
+    sf = np.sqrt(np.sum(D ** 2))
+    l = O.loss(O.Sparse.from_csr(S), A, B)
+    assert l["obj"] == pytest.approx(math.sqrt(sl) / sf, rel=1e-12)
+    assert l["rmse"] == pytest.approx(np.sqrt(np.sum((D - Shat) ** 2)) / sf, rel=1e-12)
+    assert l["wjd"] == pytest.approx(1 - np.minimum(D, Shat).sum() / np.maximum(D, Shat).sum(), rel=1e-12)
+    assert l["obj"] >= l["rmse"]
+
+
+def test_momentum_is_heavy_ball():
+    """Momentum reading: M_{t+1} - M_t = U_t + gamma (M_t - M_{t-1})."""
+    S, _ = _rand_sparse(30, 24, 0.2, 9)
+    W, H = WL.init_factors(30, 24, 3, 3)
+    opts = O.Options(block_rows=8, block_cols=8, eta=0.8, gamma=0.6)
+    st = O.State(S, W, H, opts)
+    prev = st.A.copy()
+    for t, blk in enumerate([0, 2, 1]):
+        M = st.A.copy()
+        R, G = st.block_terms(O.COL, blk, O.STOCH)
+        U = opts.eta * (np.linalg.solve(G, R.T).T - M)
+        st.block_update(O.COL, blk, O.STOCH)
+        np.testing.assert_allclose(st.A - M, U + opts.gamma * (M - prev), rtol=1e-9, atol=1e-12)
+        prev = M
+
+
+def test_stochastic_sweep_decreases_loss_on_planted():
+    S, _, _, _ = WL.planted(200, 160, 4, tau=0.5, seed=4)
+    W, H = WL.init_factors(200, 160, 5, 4)
+    st = O.State(S, W, H, O.Options(block_rows=40, block_cols=40, eta=1.0, gamma=0.5))
+    l0 = st.loss()["obj"]
+    for _ in range(10):
+        st.sweep()
+    assert st.loss()["obj"] < 0.5 * l0
