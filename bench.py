@@ -1,0 +1,310 @@
+#!/usr/bin/env python3
+"""Throughput of the SALSA block sweep on GB300.
+
+One step = one full stochastic sweep of the connectome-shaped workload
+(139,255 x 139,255, power-law out-degree with mean 20, ~2.8M nonzeros,
+r = 64, blocks of 4096; seeded synthetic data): for every block step the
+Gram matrix and its inverse, the fused Z-panel tensor-core kernel, the sparse
+support correction and the least-squares/momentum update.  Metric: Z entries
+per second = 2 m n / sweep time (a sweep touches every entry of Z twice).
+
+Default (``--impl ours``): the CUDA library through its C ABI, inputs resident
+in HBM, device time with CUDA events over exactly K sweeps after W warm-up
+sweeps.  ``e2e`` repeats the measurement through the public API with host
+buffers: per step the factors are copied in from pinned host memory, one
+sweep runs, and the factors are copied back.  ``--impl reference`` times the
+fp64 CPU oracle on the host cores on a bounded sample of the same workload.
+
+Under torchrun (N > 1 GPUs) every rank runs an independent replica of the
+workload (the sweep has no data-path collective); rank 0 prints the
+whole-job rate over the slowest rank's time.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+WORKLOADS = {
+    # name: (generator key, r, block, precision default)
+    "connectome_r64": ("connectome_r64", 64, 4096),
+    "connectome_r256": ("connectome_r256", 256, 8192),
+    "planted_medium": ("planted_medium", 32, 2048),
+    "identity": ("identity", 3, 512),
+}
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + q,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, smax, reasons = [], [], set()
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, v in zip(["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                                "sw_power_cap"], f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def oracle_sample(wl, budget_s=20.0):
+    """Time the fp64 oracle on block steps of the workload until the budget
+    (at least one COL/STOCH and one ROW/STOCH step); Z entries per second."""
+    import numpy as np
+    import oracle as O
+    st = O.State(wl.S, wl.W0, wl.H0, O.Options(block_rows=wl.block_rows, block_cols=wl.block_cols,
+                                                 eta=wl.eta, gamma=wl.gamma))
+    steps = st.sweep_steps(0)
+    entries, t_used, done = 0, 0.0, []
+    for side, block, kind in steps:
+        M, _, (m0, m1), _, _, (c0, c1) = st._roles(side, block, kind)
+        t0 = time.perf_counter()
+        st.block_update(side, block, kind)
+        dt = time.perf_counter() - t0
+        entries += (m1 - m0) * (c1 - c0)
+        t_used += dt
+        done.append((side, block))
+        if t_used >= budget_s and len(done) >= 2:
+            break
+    return entries / t_used, len(done), t_used
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="connectome_r64")
+    ap.add_argument("--precision", choices=["bf16", "fp32"], default="bf16")
+    ap.add_argument("--epilogue", choices=["z", "delta"], default="z")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+
+    ws, rank, local = dist_setup()
+    metric = "Z entries/s per full ALS sweep (2*m*n / sweep time)"
+    from paper_2608_21607_gb300 import workloads as WLm
+    gen, r, block = WORKLOADS[args.workload]
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        wl = WLm.workload(gen, seed=0)
+        cores = os.cpu_count()
+        vals = []
+        for i in range(args.warmup + args.steps):
+            v, nsteps, t = oracle_sample(wl, budget_s=max(1.0, 60.0 / (args.warmup + args.steps)))
+            if i >= args.warmup:
+                vals.append((v, nsteps, t))
+        value = statistics.median(v for v, _, _ in vals)
+        tsum = sum(t for _, _, t in vals)
+        sample = ("%d block steps of the sweep per timed step (first COL/STOCH and ROW/STOCH blocks of "
+                  "sweep 0), fp64 oracle, numpy on %d host cores" % (vals[0][1], cores))
+        line = {"impl": "reference", "metric": metric, "value": value, "unit": "Z entries/s",
+                "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+                "ms_per_step": 1e3 * tsum / len(vals), "higher_is_better": True, "scaling": "weak",
+                "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+                "config": {"workload": wl.name, "m": wl.m, "n": wl.n, "nnz": wl.S.nnz, "r": r,
+                           "block": block, "schedule": "stochastic", "parallelism": "host cores"},
+                "cpu_baseline": {"value": value, "unit": "Z entries/s", "cores": cores, "kind": "oracle",
+                                 "sample": sample},
+                "e2e": {"value": value, "unit": "Z entries/s", "h2d_bytes_per_step": 0,
+                        "d2h_bytes_per_step": 0}}
+        print(json.dumps(line))
+        return 0
+
+    import numpy as np
+    import torch
+    from paper_2608_21607_gb300 import build as B
+    from paper_2608_21607_gb300 import nmd as N
+
+    torch.cuda.set_device(local)
+    dist = None
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    B.build()
+    wl = WLm.workload(gen, seed=0)
+    prec = {"bf16": N.NMD_BF16, "fp32": N.NMD_FP32}[args.precision]
+    epi = {"z": N.NMD_EPI_Z, "delta": N.NMD_EPI_DELTA}[args.epilogue]
+    sol = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols, schedule=N.NMD_STOCH,
+                   eta=wl.eta, gamma=wl.gamma, precision=prec, epilogue=epi, seed=0)
+    sol.set_factors(wl.W0, wl.H0)
+    stream = sol.stream
+
+    def barrier():
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    # ---------------- device-resident timing ----------------
+    for _ in range(args.warmup):
+        sol.sweep()
+    sol.sync()
+    barrier()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    l0 = sol.launches
+    sol.profile(True)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        sol.sweep()
+    e1.record(stream)
+    sol.sync()
+    ms_total = e0.elapsed_time(e1)
+    launches = sol.launches - l0
+    dense_ms, dense_n = sol.profile_read(N.NMD_K_DENSE)
+    other = {name: sol.profile_read(k) for name, k in
+             [("sparse", N.NMD_K_SPARSE), ("gram_inverse", N.NMD_K_GRAM), ("update", N.NMD_K_UPDATE)]}
+    sol.profile(False)
+    clk = clocks.stop()
+    barrier()
+    t_max = ms_total
+    if dist is not None:
+        t = torch.tensor([ms_total], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        t_max = float(t.item())
+    entries = 2.0 * wl.m * wl.n
+    value = ws * entries * args.steps / (t_max / 1e3)
+
+    # dense kernel roofline: 4 M K r algorithmic flops per launch (2 M K r for
+    # L = M Q^T and 2 M K r for R = P Q), summed over the launches of a sweep
+    Kr = -(-wl.m // wl.block_rows)
+    Kc = -(-wl.n // wl.block_cols)
+    flops_sweep = 4.0 * wl.r * (wl.m * wl.n + wl.n * wl.m)   # COL steps: M=m, sum K = n; ROW steps: M=n, sum K=m
+    launches_per_sweep = Kr + Kc
+    flops_per_launch = flops_sweep / launches_per_sweep
+    pk, pk_kind = peaks()
+    peak = pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    achieved = flops_sweep * args.steps / (dense_ms / 1e3) / 1e12 if dense_ms > 0 else None
+    roofline = {"bound": "tensor", "kernel": "panel_tc_kernel (fused Z-panel, tcgen05)",
+                "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+                "frac": (achieved / peak) if achieved else None, "traffic": None,
+                "peak_kind": "%s bf16 dense, sustained" % pk_kind,
+                "flops_per_launch": flops_per_launch, "launches": dense_n,
+                "avg_launch_us": 1e3 * dense_ms / max(dense_n, 1),
+                "share_of_step": dense_ms / ms_total if ms_total > 0 else None,
+                "other_kernels_ms": {k: v[0] for k, v in other.items()}}
+    if prec == N.NMD_FP32:
+        roofline["note"] = "fp32-accurate mode issues 3 bf16 MMAs per product; flops counted once"
+
+    # ---------------- end to end through the public API, host buffers -------
+    Wh = torch.from_numpy(np.ascontiguousarray(wl.W0, np.float32)).pin_memory()
+    Hh = torch.from_numpy(np.ascontiguousarray(wl.H0, np.float32)).pin_memory()
+    Wo = torch.empty_like(Wh).pin_memory()
+    Ho = torch.empty_like(Hh).pin_memory()
+    h2d = (Wh.numel() + Hh.numel()) * 4
+    d2h = (Wo.numel() + Ho.numel()) * 4
+
+    def e2e_step():
+        N.nmd_set_factors(sol.h, Wh, Hh, False)
+        N.nmd_sweep(sol.h)
+        N.nmd_get_factors(sol.h, Wo, Ho, False)
+
+    for _ in range(args.warmup):
+        e2e_step()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        e2e_step()
+    torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - t0
+    if dist is not None:
+        t = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    e2e = {"value": ws * entries * args.steps / e2e_s, "unit": "Z entries/s", "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * e2e_s / args.steps}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        v, nsteps, t = oracle_sample(wl, budget_s=15.0)
+        cpu = {"value": v, "unit": "Z entries/s", "cores": os.cpu_count(), "kind": "oracle",
+               "sample": "%d block steps (%.1f s) of sweep 0 of the same workload, fp64 oracle (numpy)"
+                         % (nsteps, t)}
+
+    if rank == 0:
+        line = {"metric": metric, "value": value, "unit": "Z entries/s", "n_gpus": ws, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": t_max / args.steps, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": args.precision if prec == N.NMD_BF16 else "f32",
+                "data": "synthetic",
+                "config": {"workload": wl.name, "m": wl.m, "n": wl.n, "nnz": wl.S.nnz, "r": wl.r,
+                           "block": wl.block_rows, "schedule": "stochastic, alternating", "eta": wl.eta,
+                           "gamma": wl.gamma, "precision": args.precision,
+                           "epilogue": args.epilogue, "parallelism": "replicas" if ws > 1 else "single GPU",
+                           "l2": "inputs larger than L2 (factors, momentum and operand copies ~260 MB)"},
+                "e2e": e2e, "roofline": roofline, "cpu_baseline": cpu, "clocks": clk,
+                "gpu_launches": launches}
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,234 @@
+/*
+ * nmd.h -- C ABI of libnmd, a single-GPU (sm_103a) implementation of the
+ * stochastic alternating least-squares sweep (SALSA) for subzero matrix
+ * completion S ~ max(0, W H) of a sparse nonnegative m x n matrix S.
+ *
+ * The method (paper "Subzero matrix completion for sparse data analysis"):
+ *   - auxiliary matrix, Sec. 3.2 eq. (updateZ): Z_ij = S_ij where S_ij > 0,
+ *     otherwise min(0, L_ij), with L = W H = A B^T (eq. ABt; A = W, B = H^T);
+ *   - factor updates, eqs. (lsqA)/(lsqB) in the Delta form of eqs.
+ *     (spLsqA)/(spLsqB), restricted to a contiguous block of rows (parallel
+ *     least squares, eq. lsqA_par) or to a mini-batch of columns with step
+ *     size eta (stochastic least squares, eq. lsqA_sto) plus momentum
+ *     (Sec. 4.1, after eq. lsqA_sto);
+ *   - losses, Sec. 3.1: objective ||Z - L||_F/||S||_F (eq. auxCost, evaluated
+ *     as eq. SLloss), RMSE (eq. RMSE), weighted Jaccard distance (eq. WJD).
+ * Z is never stored: every kernel forms its tiles of L on chip.
+ *
+ * Conventions shared by every call:
+ *   - Matrices are row-major, float32.  W is m x r, H is r x n.
+ *   - Ownership: the caller owns every pointer it passes.  The library copies
+ *     the CSR at nmd_create, keeps only the device workspace pointer it is
+ *     given (and never frees it), and frees only its own host objects in
+ *     nmd_destroy.  The library itself allocates no device memory.
+ *   - Asynchrony: calls that take a handle enqueue their work on the CUDA
+ *     stream given to nmd_create and return without waiting, except
+ *     nmd_create (waits for its copies), nmd_get_factors, nmd_get_state,
+ *     nmd_loss, nmd_sync and nmd_block_terms, which synchronise that stream.
+ *   - Errors: every call returns an nmd_status.  A non-OK return leaves the
+ *     handle usable; nmd_last_error() gives a one-line description.  Errors
+ *     found on the device (a non-positive Cholesky pivot, a non-finite
+ *     factor, a wait that ran out) are sticky: they are recorded in device
+ *     memory, every later update becomes a no-op, and the next synchronising
+ *     call returns the status and clears it.
+ *   - Thread safety: none per handle; distinct handles are independent.
+ */
+#ifndef NMD_H
+#define NMD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct nmd_handle nmd_handle;
+
+typedef enum {
+  NMD_OK = 0,
+  NMD_ERR_INVALID = 1,     /* bad argument (size, index, option, null pointer) */
+  NMD_ERR_CSR = 2,         /* malformed CSR: see nmd_create */
+  NMD_ERR_NOT_SPD = 3,     /* a block Gram matrix had a non-positive pivot */
+  NMD_ERR_DIVERGED = 4,    /* an update produced a non-finite factor entry */
+  NMD_ERR_TIMEOUT = 5,     /* a bounded device-side wait ran out */
+  NMD_ERR_CUDA = 6,        /* a CUDA runtime call failed */
+  NMD_ERR_WORKSPACE = 7,   /* workspace too small or misaligned */
+  NMD_ERR_UNSUPPORTED = 8  /* no kernel for this device / rank / precision */
+} nmd_status;
+
+typedef enum { NMD_ROW = 0, NMD_COL = 1 } nmd_side;
+typedef enum { NMD_EXACT = 0, NMD_STOCH = 1 } nmd_kind;
+typedef enum { NMD_ALTERNATE = 0, NMD_PHASED = 1 } nmd_order;
+
+/* Arithmetic of the dense Z-panel contraction and of the loss:
+ *   NMD_BF16 -- operands rounded to bf16 (round to nearest even), products on
+ *               the tcgen05 tensor cores with fp32 accumulation;
+ *   NMD_FP32 -- fp32-accurate: every operand x is split as x = hi + lo with
+ *               hi = bf16(x), lo = bf16(x - hi) and each product is formed as
+ *               hi*hi + hi*lo + lo*hi on the tensor cores (3 MMAs, fp32 accumulate);
+ *   NMD_SIMT -- plain fp32 FMA on the CUDA cores (slow; reference path).
+ * Gram matrices, Cholesky, solves and updates are fp32 in every mode;
+ * loss reductions are fp64. */
+typedef enum { NMD_BF16 = 0, NMD_FP32 = 1, NMD_SIMT = 2 } nmd_precision;
+
+/* Form of the dense contraction (both give the same update, Sec. 3.2):
+ *   NMD_EPI_Z     -- R = Z Q with the min(0, L) tile epilogue (eq. updateZ),
+ *                    update M <- M + eta (R G^{-1} - M)         (eqs. lsqA/lsqB);
+ *   NMD_EPI_DELTA -- R = Delta Q with the -max(0, L) tile epilogue (eq. updateD),
+ *                    update M <- M + eta R G^{-1}                (eqs. spLsqA/spLsqB). */
+typedef enum { NMD_EPI_Z = 0, NMD_EPI_DELTA = 1 } nmd_epilogue;
+
+typedef struct {
+  int64_t block_rows;   /* rows of S per row block  (>= 1) */
+  int64_t block_cols;   /* columns of S per column block (>= 1) */
+  int32_t schedule;     /* nmd_kind used by nmd_sweep */
+  int32_t order;        /* nmd_order used by nmd_sweep for NMD_STOCH */
+  double eta;           /* step size (> 0); Sec. 4.1 eq. lsqA_sto */
+  double gamma;         /* momentum in [0, 1); used by NMD_STOCH updates only */
+  double ridge;         /* lambda added to the Gram diagonal (>= 0; default 0) */
+  int32_t precision;    /* nmd_precision */
+  int32_t epilogue;     /* nmd_epilogue */
+  uint64_t seed;        /* block-order seed */
+} nmd_options;
+
+typedef struct {
+  double obj;        /* ||Z - L||_F / ||S||_F  (eq. auxCost) */
+  double rmse;       /* ||S - max(0, L)||_F / ||S||_F  (eq. RMSE) */
+  double wjd;        /* 1 - sum min(S, Shat) / sum max(S, Shat)  (eq. WJD) */
+  double s_fro;      /* ||S||_F */
+  double sum_relu2;  /* sum over all (i, j) of max(0, L_ij)^2 */
+  double sum_relu;   /* sum over all (i, j) of max(0, L_ij) */
+} nmd_loss_out;
+
+/* Library version string (static storage). */
+const char* nmd_version(void);
+
+/* Defaults: blocks of 4096, NMD_STOCH, NMD_ALTERNATE, eta = 1, gamma = 0.9
+ * (the paper's defaults, Sec. 5.2 and Table "hyper"), ridge = 0, NMD_BF16,
+ * NMD_EPI_Z, seed = 0. */
+void nmd_default_options(nmd_options* opts);
+
+/* Device workspace (bytes) nmd_create needs for this problem.  Validates the
+ * CSR exactly as nmd_create does.  The workspace must be 256-byte aligned. */
+nmd_status nmd_workspace_bytes(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
+                               const int32_t* col_idx, const float* vals,
+                               const nmd_options* opts, size_t* bytes);
+
+/* Create a solver for the m x n matrix S given as host CSR (row_ptr[m+1],
+ * col_idx[nnz], vals[nnz]; the support of S is the set of stored entries
+ * with value > 0, eq. updateZ -- stored zeros are dropped).
+ * Rejected with NMD_ERR_CSR: row_ptr[0] != 0, decreasing row_ptr, column
+ * index outside [0, n), columns not strictly increasing within a row,
+ * negative or non-finite values.  Rejected with NMD_ERR_INVALID: m or n < 1
+ * or >= 2^31, r < 1 or r > 256, block sizes < 1, eta <= 0, gamma outside
+ * [0, 1), ridge < 0, unknown enum values.
+ * d_workspace: device memory of at least nmd_workspace_bytes() bytes, owned
+ * by the caller and kept until nmd_destroy.  stream: a cudaStream_t (NULL =
+ * the legacy default stream).  The factors start at zero: call
+ * nmd_set_factors before updating. */
+nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
+                      const int32_t* col_idx, const float* vals, const nmd_options* opts,
+                      void* d_workspace, size_t ws_bytes, void* stream, nmd_handle** out);
+
+/* Set W (m x r, row-major) and H (r x n, row-major); host pointers if
+ * on_device == 0, device pointers otherwise.  Resets both momentum buffers
+ * to zero.  Asynchronous; host buffers must stay valid until the stream
+ * reaches this point (the call waits for the host-to-device copies). */
+nmd_status nmd_set_factors(nmd_handle* h, const float* W, const float* H, int on_device);
+
+/* Copy W (m x r) and H (r x n) out, to host (on_device == 0) or device memory.
+ * Synchronises the stream and reports any sticky device error. */
+nmd_status nmd_get_factors(nmd_handle* h, float* W, float* H, int on_device);
+
+/* One block update of one of four kinds (the M-side is the
+ * factor updated, Q-side the rows contracted against):
+ *   (NMD_ROW, NMD_EXACT, I): W_I <- least squares against all of H on S[I, :]
+ *                            (eq. lsqA_par), W_I += eta (W_ls - W_I);
+ *   (NMD_COL, NMD_EXACT, J): H_:J likewise on S[:, J];
+ *   (NMD_COL, NMD_STOCH, J): all of W from the mini-batch H_:J on S[:, J]
+ *                            (eq. lsqA_sto), with momentum;
+ *   (NMD_ROW, NMD_STOCH, I): all of H from the mini-batch W_I on S[I, :].
+ * Blocks are contiguous ranges [k b, min((k+1) b, N)) with b = block_rows
+ * (row blocks, N = m) or block_cols (column blocks, N = n).  The block's Gram
+ * matrix must be nonsingular (a block needs at least r rows with linearly
+ * independent factor rows), else NMD_ERR_NOT_SPD is reported by the next
+ * synchronising call and the update is skipped.  Asynchronous. */
+nmd_status nmd_block_update(nmd_handle* h, int32_t side, int64_t block, int32_t kind);
+
+/* One sweep: block orders are SplitMix64 + Fisher-Yates permutations of the
+ * row blocks and column blocks for (seed, sweep index, side).  NMD_EXACT:
+ * all row blocks, then all column blocks.  NMD_STOCH + NMD_ALTERNATE: for
+ * t = 0 .. max(Kc, Kr)-1, column block perm_c[t] (if t < Kc) then row block
+ * perm_r[t] (if t < Kr); NMD_PHASED: all column blocks, then all row blocks.
+ * Every sweep visits each entry of Z twice.  Advances the sweep counter.
+ * Asynchronous. */
+nmd_status nmd_sweep(nmd_handle* h);
+
+/* Block order of one sweep and side (perm must hold K = number of blocks of
+ * that side; K is checked).  Pure host computation. */
+nmd_status nmd_block_order(const nmd_handle* h, int64_t sweep, int32_t side, int64_t* perm,
+                           int64_t K);
+
+/* Losses of the current factors (eqs. auxCost/SLloss, RMSE, WJD): a dense
+ * pass over all m x n entries of L plus a correction over the support of S,
+ * reduced in a fixed order in fp64.  Synchronises the stream. */
+nmd_status nmd_loss(nmd_handle* h, nmd_loss_out* out);
+
+/* Waits for the stream and returns (then clears) any sticky device error. */
+nmd_status nmd_sync(nmd_handle* h);
+
+/* Verification hook: the right-hand side R = Z Q (NMD_EPI_Z) or Delta Q
+ * (NMD_EPI_DELTA) for the M-side rows of one block update (rows x r,
+ * row-major) and the Gram matrix G = Q^T Q (r x r), without updating
+ * anything.  Host pointers; either may be NULL.  Synchronises. */
+nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* R,
+                           float* G, int64_t* rows);
+
+/* Verification hook: L = M Q^T, the first product of the tensor-core panel
+ * kernel (eq. ABt restricted to one block), for the M-side rows and Q-side
+ * rows of one block update, before any epilogue.  d_L: device memory of
+ * rows x K floats (row-major), owned by the caller; rows and K are returned
+ * in *rows and *cols when those are not NULL.  NMD_ERR_UNSUPPORTED for
+ * NMD_SIMT.  Synchronises. */
+nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* d_L,
+                              int64_t* rows, int64_t* cols);
+
+/* Verification hook: the sparse traversal of one block update -- for every
+ * M-side row with support in the block's panel, ascending, its entries in
+ * ascending Q-side order.  Writes up to cap (row, q) index pairs to
+ * rows_out/q_out (q relative to the block's first Q-side row) and the total
+ * count to *count.  Pure host computation over the panel index. */
+nmd_status nmd_panel_traversal(const nmd_handle* h, int32_t side, int64_t block, int32_t kind,
+                               int64_t* rows_out, int64_t* q_out, int64_t cap, int64_t* count);
+
+/* Checkpoint: factors W (m x r), H (r x n), momentum EW (m x r), EH (r x n)
+ * and the sweep counter.  Host pointers.  nmd_get_state synchronises;
+ * nmd_set_state is asynchronous (waits for its host copies). */
+nmd_status nmd_get_state(nmd_handle* h, float* W, float* H, float* EW, float* EH,
+                         int64_t* sweep_index);
+nmd_status nmd_set_state(nmd_handle* h, const float* W, const float* H, const float* EW,
+                         const float* EH, int64_t sweep_index);
+
+/* Kernel timing with CUDA events recorded on the handle's stream around each
+ * launch.  nmd_profile(h, 1) clears the totals and starts recording,
+ * nmd_profile(h, 0) stops.  nmd_profile_read synchronises and returns the
+ * device time (ms) and launch count accumulated for one kernel class:
+ * NMD_K_DENSE (the fused Z-panel kernel), NMD_K_SPARSE (support
+ * correction), NMD_K_GRAM (Gram matrix + inverse), NMD_K_UPDATE (least
+ * squares / momentum update), NMD_K_LOSS (dense loss pass). */
+typedef enum { NMD_K_DENSE = 0, NMD_K_SPARSE = 1, NMD_K_GRAM = 2, NMD_K_UPDATE = 3, NMD_K_LOSS = 4 } nmd_kernel_class;
+nmd_status nmd_profile(nmd_handle* h, int on);
+nmd_status nmd_profile_read(nmd_handle* h, int32_t kernel_class, double* ms, int64_t* launches);
+
+/* Number of kernel launches this handle has issued (for launch accounting). */
+int64_t nmd_launch_count(const nmd_handle* h);
+
+const char* nmd_status_string(nmd_status s);
+const char* nmd_last_error(const nmd_handle* h);
+void nmd_destroy(nmd_handle* h);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* NMD_H */

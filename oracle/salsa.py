@@ -269,10 +269,24 @@ class State:
             return self.B, self.EB, (j0, j1), self.A, self.St, (0, self.m)
         return self.A, self.EA, (0, self.m), self.B[j0:j1], self.S, (j0, j1)
 
-    def block_terms(self, side: int, block: int, kind: int, chunk_elems: int = 1 << 24):
-        """R = Z Q for the M-side rows, G = Q^T Q, and the Q rows used."""
+    def block_terms(self, side: int, block: int, kind: int, chunk_elems: int = 1 << 24,
+                    rows=None):
+        """R = Z Q for the M-side rows and G = Q^T Q.
+
+        With ``rows`` (indices relative to the first M-side row) only those
+        rows of R are formed -- each row of R depends on its own row of Z only.
+        """
         M, _, (m0, m1), Q, src, (c0, c1) = self._roles(side, block, kind)
         K = c1 - c0
+        G = Q.T @ Q
+        if rows is not None:
+            R = np.zeros((len(rows), self.r))
+            for t, i in enumerate(rows):
+                a = m0 + int(i)
+                L = M[a:a + 1] @ Q.T
+                Z = update_z(src.dense_panel(a, a + 1, c0, c1), L)
+                R[t] = (Z @ Q)[0]
+            return R, G
         R = np.zeros((m1 - m0, self.r))
         step = max(1, chunk_elems // max(K, 1))
         for a in range(m0, m1, step):
@@ -280,8 +294,18 @@ class State:
             L = M[a:b] @ Q.T
             Z = update_z(src.dense_panel(a, b, c0, c1), L)
             R[a - m0:b - m0] = Z @ Q
-        G = Q.T @ Q
         return R, G
+
+    def traversal(self, side: int, block: int, kind: int):
+        """(M-side row, Q-side index) pairs of the block's support: rows
+        ascending, Q-side index ascending within a row (both relative to the
+        block's first M-side / Q-side row)."""
+        _, _, (m0, m1), _, src, (c0, c1) = self._roles(side, block, kind)
+        a, b = src.row_ptr[m0], src.row_ptr[m1]
+        rows = np.repeat(np.arange(m0, m1), np.diff(src.row_ptr[m0:m1 + 1]))
+        cols = src.col_idx[a:b]
+        keep = (cols >= c0) & (cols < c1)
+        return rows[keep] - m0, cols[keep] - c0
 
     def block_update(self, side: int, block: int, kind: int):
         o = self.opts

@@ -1,0 +1,827 @@
+// Host side of libnmd: argument checks, CSR/CSC and panel-index construction,
+// workspace layout, the block schedule of a sweep and the C ABI of nmd.h.
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <algorithm>
+#include <string>
+#include <vector>
+
+#include "nmd_internal.cuh"
+
+using namespace nmd;
+
+#define NMD_VERSION_STRING "libnmd 0.1 (sm_103a)"
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// Block order: SplitMix64 (S. Vigna's published generator) driving a
+// Fisher-Yates shuffle.  State for (seed, sweep, side) is
+// mix(seed) ^ mix((sweep << 1) | side); for i = K-1 down to 1 the block at i
+// is swapped with the one at next() % (i + 1).
+// ---------------------------------------------------------------------------
+inline uint64_t sm64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+std::vector<int64_t> permutation(uint64_t seed, int64_t sweep, int side, int64_t K) {
+  uint64_t state = sm64_mix(seed) ^ sm64_mix((((uint64_t)sweep) << 1) | (uint64_t)side);
+  std::vector<int64_t> p(K);
+  for (int64_t i = 0; i < K; ++i) p[i] = i;
+  for (int64_t i = K - 1; i >= 1; --i) {
+    state += 0x9E3779B97F4A7C15ull;
+    uint64_t j = sm64_mix(state) % (uint64_t)(i + 1);
+    std::swap(p[i], p[(int64_t)j]);
+  }
+  return p;
+}
+
+inline int64_t nblocks(int64_t N, int64_t b) { return (N + b - 1) / b; }
+
+int pad_rank(int r) {
+  if (r <= 16) return 16;
+  if (r <= 32) return 32;
+  if (r <= 64) return 64;
+  if (r <= 128) return 128;
+  return 256;
+}
+
+// ---------------------------------------------------------------------------
+// Host copy of S: validated CSR of the positive entries and its transpose.
+// ---------------------------------------------------------------------------
+struct HostSparse {
+  int64_t m = 0, n = 0;
+  std::vector<int64_t> rowptr, colptr;
+  std::vector<int32_t> col, row;
+  std::vector<float> val, valT;
+  double s_fro = 0.0;
+};
+
+nmd_status check_options(const nmd_options* o, std::string* why) {
+  if (!o) { *why = "options pointer is NULL"; return NMD_ERR_INVALID; }
+  if (o->block_rows < 1 || o->block_cols < 1) { *why = "block sizes must be >= 1"; return NMD_ERR_INVALID; }
+  if (o->schedule != NMD_EXACT && o->schedule != NMD_STOCH) { *why = "unknown schedule"; return NMD_ERR_INVALID; }
+  if (o->order != NMD_ALTERNATE && o->order != NMD_PHASED) { *why = "unknown order"; return NMD_ERR_INVALID; }
+  if (!(o->eta > 0.0) || !isfinite(o->eta)) { *why = "eta must be a finite positive number"; return NMD_ERR_INVALID; }
+  if (!(o->gamma >= 0.0 && o->gamma < 1.0)) { *why = "gamma must lie in [0, 1)"; return NMD_ERR_INVALID; }
+  if (!(o->ridge >= 0.0) || !isfinite(o->ridge)) { *why = "ridge must be finite and >= 0"; return NMD_ERR_INVALID; }
+  if (o->precision != NMD_BF16 && o->precision != NMD_FP32 && o->precision != NMD_SIMT) {
+    *why = "unknown precision"; return NMD_ERR_INVALID;
+  }
+  if (o->epilogue != NMD_EPI_Z && o->epilogue != NMD_EPI_DELTA) { *why = "unknown epilogue"; return NMD_ERR_INVALID; }
+  return NMD_OK;
+}
+
+nmd_status build_sparse(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
+                        const int32_t* col_idx, const float* vals, HostSparse* S,
+                        std::string* why) {
+  if (m < 1 || n < 1 || m >= (int64_t(1) << 31) || n >= (int64_t(1) << 31)) {
+    *why = "m and n must lie in [1, 2^31)"; return NMD_ERR_INVALID;
+  }
+  if (r < 1 || r > 256) { *why = "rank r must lie in [1, 256]"; return NMD_ERR_INVALID; }
+  if (!row_ptr) { *why = "row_ptr is NULL"; return NMD_ERR_INVALID; }
+  if (row_ptr[0] != 0) { *why = "row_ptr[0] must be 0"; return NMD_ERR_CSR; }
+  for (int64_t i = 0; i < m; ++i)
+    if (row_ptr[i + 1] < row_ptr[i]) {
+      char b[96]; snprintf(b, sizeof b, "row_ptr decreases at row %lld", (long long)i);
+      *why = b; return NMD_ERR_CSR;
+    }
+  int64_t nnz_in = row_ptr[m];
+  if (nnz_in > 0 && (!col_idx || !vals)) { *why = "col_idx or vals is NULL"; return NMD_ERR_INVALID; }
+  S->m = m; S->n = n;
+  S->rowptr.assign(m + 1, 0);
+  S->col.clear(); S->val.clear();
+  S->col.reserve(nnz_in); S->val.reserve(nnz_in);
+  double fro = 0.0;
+  for (int64_t i = 0; i < m; ++i) {
+    int64_t prev = -1;
+    for (int64_t e = row_ptr[i]; e < row_ptr[i + 1]; ++e) {
+      int64_t c = col_idx[e];
+      float v = vals[e];
+      if (c < 0 || c >= n) {
+        char b[128]; snprintf(b, sizeof b, "column index %lld out of range at row %lld", (long long)c, (long long)i);
+        *why = b; return NMD_ERR_CSR;
+      }
+      if (c <= prev) {
+        char b[128]; snprintf(b, sizeof b, "columns not strictly increasing in row %lld", (long long)i);
+        *why = b; return NMD_ERR_CSR;
+      }
+      if (!isfinite(v) || v < 0.0f) {
+        char b[128]; snprintf(b, sizeof b, "negative or non-finite value in row %lld", (long long)i);
+        *why = b; return NMD_ERR_CSR;
+      }
+      prev = c;
+      if (v > 0.0f) {
+        S->col.push_back((int32_t)c);
+        S->val.push_back(v);
+        fro += (double)v * (double)v;
+      }
+    }
+    S->rowptr[i + 1] = (int64_t)S->col.size();
+  }
+  if (S->col.empty()) { *why = "S has no positive entry (||S||_F = 0)"; return NMD_ERR_CSR; }
+  S->s_fro = sqrt(fro);
+  // transpose (counting sort by column; rows stay ascending within a column)
+  int64_t nnz = (int64_t)S->col.size();
+  S->colptr.assign(n + 1, 0);
+  for (int64_t e = 0; e < nnz; ++e) S->colptr[S->col[e] + 1]++;
+  for (int64_t j = 0; j < n; ++j) S->colptr[j + 1] += S->colptr[j];
+  S->row.resize(nnz); S->valT.resize(nnz);
+  std::vector<int64_t> cur(S->colptr.begin(), S->colptr.end() - 1);
+  for (int64_t i = 0; i < m; ++i)
+    for (int64_t e = S->rowptr[i]; e < S->rowptr[i + 1]; ++e) {
+      int64_t p = cur[S->col[e]]++;
+      S->row[p] = (int32_t)i;
+      S->valT[p] = S->val[e];
+    }
+  return NMD_OK;
+}
+
+// Panel lists.  Over a CSR-like (ptr, idx) with N rows: for each block of the
+// *index* range (block size b over Nidx), the rows with entries in the block.
+void build_stoch_panels(const std::vector<int64_t>& ptr, const std::vector<int32_t>& idx,
+                        int64_t N, int64_t Nidx, int64_t b, PanelSet* P) {
+  int64_t K = nblocks(Nidx, b);
+  std::vector<std::vector<PanelRow>> per(K);
+  for (int64_t i = 0; i < N; ++i) {
+    int64_t e = ptr[i], end = ptr[i + 1];
+    while (e < end) {
+      int64_t blk = idx[e] / b;
+      int64_t s = e;
+      while (e < end && idx[e] / b == blk) ++e;
+      per[blk].push_back(PanelRow{(int32_t)i, (int32_t)(e - s), s});
+    }
+  }
+  P->host.clear();
+  P->light_ptr.assign(K + 1, 0);
+  P->heavy_ptr.assign(K, 0);
+  for (int64_t k = 0; k < K; ++k) {
+    P->light_ptr[k] = (int64_t)P->host.size();
+    for (auto& pr : per[k]) if (pr.len <= kHeavyRow) P->host.push_back(pr);
+    P->heavy_ptr[k] = (int64_t)P->host.size();
+    for (auto& pr : per[k]) if (pr.len > kHeavyRow) P->host.push_back(pr);
+  }
+  P->light_ptr[K] = (int64_t)P->host.size();
+}
+
+// Exact panels: block k of rows [k b, (k+1) b) with their complete rows.
+void build_exact_panels(const std::vector<int64_t>& ptr, int64_t N, int64_t b, PanelSet* P) {
+  int64_t K = nblocks(N, b);
+  P->host.clear();
+  P->light_ptr.assign(K + 1, 0);
+  P->heavy_ptr.assign(K, 0);
+  for (int64_t k = 0; k < K; ++k) {
+    int64_t i0 = k * b, i1 = std::min(N, (k + 1) * b);
+    P->light_ptr[k] = (int64_t)P->host.size();
+    for (int64_t i = i0; i < i1; ++i) {
+      int64_t len = ptr[i + 1] - ptr[i];
+      if (len > 0 && len <= kHeavyRow) P->host.push_back(PanelRow{(int32_t)i, (int32_t)len, ptr[i]});
+    }
+    P->heavy_ptr[k] = (int64_t)P->host.size();
+    for (int64_t i = i0; i < i1; ++i) {
+      int64_t len = ptr[i + 1] - ptr[i];
+      if (len > kHeavyRow) {
+        // rows longer than 2^31 - 1 entries are split (n < 2^31 bounds len anyway)
+        P->host.push_back(PanelRow{(int32_t)i, (int32_t)len, ptr[i]});
+      }
+    }
+  }
+  P->light_ptr[K] = (int64_t)P->host.size();
+}
+
+void build_panels(const HostSparse& S, const nmd_options& o, PanelSet P[2][2]) {
+  build_exact_panels(S.rowptr, S.m, o.block_rows, &P[NMD_ROW][NMD_EXACT]);
+  build_exact_panels(S.colptr, S.n, o.block_cols, &P[NMD_COL][NMD_EXACT]);
+  // COL/STOCH block J: all rows of S (M = W), entries with column in J
+  build_stoch_panels(S.rowptr, S.col, S.m, S.n, o.block_cols, &P[NMD_COL][NMD_STOCH]);
+  // ROW/STOCH block I: all columns of S (M = B), entries with row in I
+  build_stoch_panels(S.colptr, S.row, S.n, S.m, o.block_rows, &P[NMD_ROW][NMD_STOCH]);
+}
+
+// ---------------------------------------------------------------------------
+// Workspace layout
+// ---------------------------------------------------------------------------
+struct Carver {
+  char* base;
+  size_t off = 0;
+  explicit Carver(void* b) : base((char*)b) {}
+  template <class T>
+  T* take(size_t count) {
+    off = (off + 255) & ~size_t(255);
+    T* p = base ? (T*)(base + off) : nullptr;
+    off += count * sizeof(T);
+    return p;
+  }
+};
+
+void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanels, Workspace* w,
+            Factor* W, Factor* B) {
+  w->rowptr = c.take<int64_t>(m + 1);
+  w->col = c.take<int32_t>(nnz);
+  w->val = c.take<float>(nnz);
+  w->colptr = c.take<int64_t>(n + 1);
+  w->row = c.take<int32_t>(nnz);
+  w->valT = c.take<float>(nnz);
+  w->panels = c.take<PanelRow>(std::max<int64_t>(npanels, 1));
+  for (Factor* f : {W, B}) {
+    int64_t N = f == W ? m : n;
+    f->rows = N;
+    f->master = c.take<float>(N * rp);
+    f->hi = c.take<bf16>(N * rp);
+    f->lo = c.take<bf16>(N * rp);
+    f->E = c.take<float>(N * rp);
+  }
+  w->R = c.take<float>(std::max(m, n) * rp);
+  w->gram_part = c.take<float>((size_t)kGramParts * rp * rp);
+  w->G = c.take<float>((size_t)rp * rp);
+  w->Ginv = c.take<float>((size_t)rp * rp);
+  w->chol_scratch = c.take<float>((size_t)2 * rp * rp);
+  w->loss_part = c.take<double>((size_t)kLossParts * 8);
+  w->loss_out = c.take<double>(8);
+  w->status = c.take<int>(kStatusWords);
+  w->counters = c.take<int>(64);
+  c.off = (c.off + 255) & ~size_t(255);
+  w->bytes = c.off;
+}
+
+int64_t panel_total(PanelSet P[2][2]) {
+  int64_t t = 0;
+  for (int s = 0; s < 2; ++s)
+    for (int k = 0; k < 2; ++k) t += (int64_t)P[s][k].host.size();
+  return t;
+}
+
+// ---------------------------------------------------------------------------
+// Error plumbing
+// ---------------------------------------------------------------------------
+nmd_status fail(nmd_handle* h, nmd_status s, const std::string& why) {
+  if (h) h->last_error = why;
+  return s;
+}
+
+nmd_status cuda_check(nmd_handle* h, cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return NMD_OK;
+  std::string w = std::string(what) + ": " + cudaGetErrorString(e);
+  return fail(h, NMD_ERR_CUDA, w);
+}
+
+#define CK(h, call)                                          \
+  do {                                                       \
+    nmd_status _s = cuda_check((h), (call), #call);          \
+    if (_s != NMD_OK) return _s;                             \
+  } while (0)
+
+nmd_status after_launch(nmd_handle* h, const char* what) {
+  return cuda_check(h, cudaGetLastError(), what);
+}
+
+const char* status_name(int s) {
+  switch (s) {
+    case NMD_OK: return "ok";
+    case NMD_ERR_INVALID: return "invalid argument";
+    case NMD_ERR_CSR: return "malformed CSR";
+    case NMD_ERR_NOT_SPD: return "block Gram matrix is not positive definite";
+    case NMD_ERR_DIVERGED: return "non-finite factor entry (diverged)";
+    case NMD_ERR_TIMEOUT: return "device-side wait timed out";
+    case NMD_ERR_CUDA: return "CUDA error";
+    case NMD_ERR_WORKSPACE: return "workspace too small or misaligned";
+    case NMD_ERR_UNSUPPORTED: return "unsupported configuration";
+  }
+  return "unknown status";
+}
+
+// Synchronise, then read and clear the sticky device status.
+nmd_status sync_and_check(nmd_handle* h) {
+  CK(h, cudaStreamSynchronize(h->stream));
+  int st[kStatusWords];
+  CK(h, cudaMemcpy(st, h->ws.status, sizeof st, cudaMemcpyDeviceToHost));
+  if (st[0] != 0) {
+    CK(h, cudaMemset(h->ws.status, 0, sizeof st));
+    char b[192];
+    snprintf(b, sizeof b, "%s (device detail %d, at block step %d)", status_name(st[0]), st[1], st[2]);
+    return fail(h, (nmd_status)st[0], b);
+  }
+  return NMD_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Kernel timing: an event pair around a launch when profiling is on
+// ---------------------------------------------------------------------------
+cudaEvent_t pool_event(nmd_handle* h) {
+  if (!h->event_pool.empty()) {
+    cudaEvent_t e = h->event_pool.back();
+    h->event_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+struct TimedScope {
+  nmd_handle* h;
+  int cls;
+  cudaEvent_t a = nullptr, b = nullptr;
+  TimedScope(nmd_handle* h_, int c) : h(h_), cls(c) {
+    if (h->profiling) {
+      a = pool_event(h);
+      b = pool_event(h);
+      cudaEventRecord(a, h->stream);
+    }
+  }
+  ~TimedScope() {
+    if (a) {
+      cudaEventRecord(b, h->stream);
+      h->timed.push_back({cls, a, b});
+    }
+  }
+};
+
+void collect_timing(nmd_handle* h) {
+  for (auto& t : h->timed) {
+    float ms = 0.f;
+    if (cudaEventElapsedTime(&ms, t.a, t.b) == cudaSuccess) {
+      h->prof_ms[t.cls] += ms;
+      h->prof_launches[t.cls] += 1;
+    }
+    h->event_pool.push_back(t.a);
+    h->event_pool.push_back(t.b);
+  }
+  h->timed.clear();
+}
+
+// ---------------------------------------------------------------------------
+// One block step
+// ---------------------------------------------------------------------------
+struct Roles {
+  Factor* fm;
+  Factor* fq;
+  int64_t m0, M, q0, K;
+  const PanelSet* P;
+  const int32_t* qidx;   // absolute Q-side index of each sparse entry
+  const float* vals;
+};
+
+nmd_status roles(nmd_handle* h, int side, int64_t block, int kind, Roles* R) {
+  if (side != NMD_ROW && side != NMD_COL) return fail(h, NMD_ERR_INVALID, "side must be NMD_ROW or NMD_COL");
+  if (kind != NMD_EXACT && kind != NMD_STOCH) return fail(h, NMD_ERR_INVALID, "kind must be NMD_EXACT or NMD_STOCH");
+  int64_t b = side == NMD_ROW ? h->opt.block_rows : h->opt.block_cols;
+  int64_t N = side == NMD_ROW ? h->m : h->n;
+  int64_t K = nblocks(N, b);
+  if (block < 0 || block >= K) {
+    char s[128]; snprintf(s, sizeof s, "block %lld out of range [0, %lld)", (long long)block, (long long)K);
+    return fail(h, NMD_ERR_INVALID, s);
+  }
+  int64_t i0 = block * b, i1 = std::min(N, (block + 1) * b);
+  const PanelSet* P = &h->panels[side][kind];
+  if (side == NMD_ROW && kind == NMD_EXACT) {        // W_I from all of B on S[I, :]
+    *R = Roles{&h->W, &h->B, i0, i1 - i0, 0, h->n, P, h->ws.col, h->ws.val};
+  } else if (side == NMD_COL && kind == NMD_EXACT) { // B_J from all of W on S[:, J]^T
+    *R = Roles{&h->B, &h->W, i0, i1 - i0, 0, h->m, P, h->ws.row, h->ws.valT};
+  } else if (side == NMD_COL) {                      // all of W from B_J on S[:, J]
+    *R = Roles{&h->W, &h->B, 0, h->m, i0, i1 - i0, P, h->ws.col, h->ws.val};
+  } else {                                           // all of B from W_I on S[I, :]^T
+    *R = Roles{&h->B, &h->W, 0, h->n, i0, i1 - i0, P, h->ws.row, h->ws.valT};
+  }
+  return NMD_OK;
+}
+
+nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_update) {
+  Roles ro;
+  nmd_status st = roles(h, side, block, kind, &ro);
+  if (st != NMD_OK) return st;
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue};
+  cudaStream_t s = h->stream;
+  // Gram G = Q^T Q of the Q-side rows, then Cholesky and G^{-1}
+  int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 255) / 256));
+  {
+    TimedScope ts(h, NMD_K_GRAM);
+    launch_gram(*ro.fq, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, s);
+    launch_chol_inv(h->ws.gram_part, nparts, h->r, h->rp, (float)h->opt.ridge, h->ws.G, h->ws.Ginv,
+                    h->ws.chol_scratch, h->ws.status, s);
+    h->launches += 2;
+  }
+  if ((st = after_launch(h, "gram/cholesky")) != NMD_OK) return st;
+  // dense Z-panel contraction R = P(L) Q over every (M-side, Q-side) pair
+  {
+    TimedScope ts(h, NMD_K_DENSE);
+    if (h->opt.precision == NMD_SIMT) {
+      launch_panel_simt(a, h->ws.R, s);
+      h->launches++;
+    } else {
+      st = launch_panel_tc(a, h->ws.R, h->ws.status, h->ws.counters, h->num_sms, s, &h->launches);
+    }
+  }
+  if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
+  if ((st = after_launch(h, "dense panel")) != NMD_OK) return st;
+  // sparse correction over the block's support
+  const PanelSet& P = *ro.P;
+  int64_t lb = P.light_ptr[block], hb = P.heavy_ptr[block], he = P.light_ptr[block + 1];
+  {
+    TimedScope ts(h, NMD_K_SPARSE);
+    launch_sparse(a, P.d + lb, hb - lb, P.d + hb, he - hb, ro.qidx, ro.vals, h->ws.R, s);
+    h->launches += (hb > lb) + (he > hb);
+  }
+  if ((st = after_launch(h, "sparse correction")) != NMD_OK) return st;
+  if (do_update) {
+    bool momentum = kind == NMD_STOCH;
+    {
+      TimedScope ts(h, NMD_K_UPDATE);
+      launch_update(a, h->ws.R, h->ws.Ginv, (float)h->opt.eta, momentum ? (float)h->opt.gamma : 0.f,
+                    momentum, h->ws.status, s);
+      h->launches++;
+    }
+    if ((st = after_launch(h, "update")) != NMD_OK) return st;
+  }
+  h->step_index++;
+  return NMD_OK;
+}
+
+}  // namespace
+
+nmd_handle::~nmd_handle() {
+  if (!timed.empty()) cudaStreamSynchronize(stream);
+  for (auto& t : timed) {
+    cudaEventDestroy(t.a);
+    cudaEventDestroy(t.b);
+  }
+  for (cudaEvent_t e : event_pool) cudaEventDestroy(e);
+}
+
+// ===========================================================================
+// C ABI
+// ===========================================================================
+extern "C" {
+
+const char* nmd_version(void) { return NMD_VERSION_STRING; }
+
+void nmd_default_options(nmd_options* o) {
+  if (!o) return;
+  memset(o, 0, sizeof *o);
+  o->block_rows = 4096;
+  o->block_cols = 4096;
+  o->schedule = NMD_STOCH;
+  o->order = NMD_ALTERNATE;
+  o->eta = 1.0;
+  o->gamma = 0.9;
+  o->ridge = 0.0;
+  o->precision = NMD_BF16;
+  o->epilogue = NMD_EPI_Z;
+  o->seed = 0;
+}
+
+const char* nmd_status_string(nmd_status s) { return status_name((int)s); }
+
+const char* nmd_last_error(const nmd_handle* h) { return h ? h->last_error.c_str() : ""; }
+
+int64_t nmd_launch_count(const nmd_handle* h) { return h ? h->launches : 0; }
+
+nmd_status nmd_workspace_bytes(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
+                               const int32_t* col_idx, const float* vals, const nmd_options* opts,
+                               size_t* bytes) {
+  std::string why;
+  nmd_status st = check_options(opts, &why);
+  if (st != NMD_OK) return st;
+  if (!bytes) return NMD_ERR_INVALID;
+  HostSparse S;
+  if ((st = build_sparse(m, n, r, row_ptr, col_idx, vals, &S, &why)) != NMD_OK) return st;
+  PanelSet P[2][2];
+  build_panels(S, *opts, P);
+  Carver c(nullptr);
+  Workspace w;
+  Factor W, B;
+  layout(c, m, n, (int64_t)S.col.size(), pad_rank(r), panel_total(P), &w, &W, &B);
+  *bytes = w.bytes;
+  return NMD_OK;
+}
+
+nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
+                      const int32_t* col_idx, const float* vals, const nmd_options* opts,
+                      void* d_workspace, size_t ws_bytes, void* stream, nmd_handle** out) {
+  if (!out) return NMD_ERR_INVALID;
+  *out = nullptr;
+  nmd_handle* h = new nmd_handle();
+  std::string why;
+  nmd_status st = check_options(opts, &why);
+  HostSparse S;
+  if (st == NMD_OK) st = build_sparse(m, n, r, row_ptr, col_idx, vals, &S, &why);
+  if (st != NMD_OK) {
+    fprintf(stderr, "nmd_create: %s\n", why.c_str());
+    delete h;
+    return st;
+  }
+  h->m = m; h->n = n; h->r = r; h->rp = pad_rank(r);
+  h->nnz = (int64_t)S.col.size();
+  h->opt = *opts;
+  h->stream = (cudaStream_t)stream;
+  h->s_fro = S.s_fro;
+  build_panels(S, h->opt, h->panels);
+  Carver c(d_workspace);
+  layout(c, m, n, h->nnz, h->rp, panel_total(h->panels), &h->ws, &h->W, &h->B);
+  auto bail = [&](nmd_status s, const std::string& w) {
+    fprintf(stderr, "nmd_create: %s\n", w.c_str());
+    delete h;
+    return s;
+  };
+  if (!d_workspace || ((uintptr_t)d_workspace & 255) != 0)
+    return bail(NMD_ERR_WORKSPACE, "workspace pointer is NULL or not 256-byte aligned");
+  if (ws_bytes < h->ws.bytes) {
+    char b[160]; snprintf(b, sizeof b, "workspace has %zu bytes, needs %zu", ws_bytes, h->ws.bytes);
+    return bail(NMD_ERR_WORKSPACE, b);
+  }
+  cudaError_t e = cudaGetDevice(&h->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, h->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->cc_major, cudaDevAttrComputeCapabilityMajor, h->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->cc_minor, cudaDevAttrComputeCapabilityMinor, h->device);
+  if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("device query: ") + cudaGetErrorString(e));
+  if (h->cc_major != 10) {
+    char b[128]; snprintf(b, sizeof b, "device has compute capability %d.%d; libnmd is built for sm_103a",
+                          h->cc_major, h->cc_minor);
+    return bail(NMD_ERR_UNSUPPORTED, b);
+  }
+  // panel lists, concatenated [ROW][EXACT], [ROW][STOCH], [COL][EXACT], [COL][STOCH]
+  std::vector<PanelRow> all;
+  for (int s2 = 0; s2 < 2; ++s2)
+    for (int k = 0; k < 2; ++k) {
+      h->panels[s2][k].d = h->ws.panels + all.size();
+      all.insert(all.end(), h->panels[s2][k].host.begin(), h->panels[s2][k].host.end());
+    }
+  cudaStream_t s = h->stream;
+  struct Cp { void* d; const void* src; size_t n; } cps[] = {
+      {h->ws.rowptr, S.rowptr.data(), S.rowptr.size() * 8},
+      {h->ws.col, S.col.data(), S.col.size() * 4},
+      {h->ws.val, S.val.data(), S.val.size() * 4},
+      {h->ws.colptr, S.colptr.data(), S.colptr.size() * 8},
+      {h->ws.row, S.row.data(), S.row.size() * 4},
+      {h->ws.valT, S.valT.data(), S.valT.size() * 4},
+      {h->ws.panels, all.data(), all.size() * sizeof(PanelRow)},
+  };
+  for (auto& cp : cps)
+    if (cp.n && (e = cudaMemcpyAsync(cp.d, cp.src, cp.n, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+      return bail(NMD_ERR_CUDA, std::string("copy-in: ") + cudaGetErrorString(e));
+  // zero factors, momentum and the status words
+  for (Factor* f : {&h->W, &h->B}) {
+    e = cudaMemsetAsync(f->master, 0, f->rows * h->rp * 4, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(f->hi, 0, f->rows * h->rp * 2, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(f->lo, 0, f->rows * h->rp * 2, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(f->E, 0, f->rows * h->rp * 4, s);
+    if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("memset: ") + cudaGetErrorString(e));
+  }
+  e = cudaMemsetAsync(h->ws.status, 0, kStatusWords * sizeof(int), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->ws.counters, 0, 64 * sizeof(int), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("create: ") + cudaGetErrorString(e));
+  // the host copies of the panel lists are kept for nmd_panel_traversal
+  *out = h;
+  return NMD_OK;
+}
+
+nmd_status nmd_set_factors(nmd_handle* h, const float* W, const float* H, int on_device) {
+  if (!h || !W || !H) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_set_factors");
+  cudaStream_t s = h->stream;
+  cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+  // stage through R (max(m, n) x rp floats >= m x r and r x n)
+  CK(h, cudaMemcpyAsync(h->ws.R, W, (size_t)h->m * h->r * 4, kind, s));
+  launch_pack(h->ws.R, false, h->m, h->r, h->rp, h->W, s);
+  h->launches++;
+  CK(h, cudaMemcpyAsync(h->ws.R, H, (size_t)h->n * h->r * 4, kind, s));
+  launch_pack(h->ws.R, true, h->n, h->r, h->rp, h->B, s);
+  h->launches++;
+  CK(h, cudaMemsetAsync(h->W.E, 0, (size_t)h->m * h->rp * 4, s));
+  CK(h, cudaMemsetAsync(h->B.E, 0, (size_t)h->n * h->rp * 4, s));
+  nmd_status st = after_launch(h, "pack factors");
+  if (st != NMD_OK) return st;
+  if (!on_device) CK(h, cudaStreamSynchronize(s));   // host buffers may be released after return
+  return NMD_OK;
+}
+
+nmd_status nmd_get_factors(nmd_handle* h, float* W, float* H, int on_device) {
+  if (!h) return NMD_ERR_INVALID;
+  nmd_status st = sync_and_check(h);
+  cudaStream_t s = h->stream;
+  cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
+  if (W) {
+    launch_unpack(h->W.master, false, h->m, h->r, h->rp, h->ws.R, s);
+    h->launches++;
+    CK(h, cudaMemcpyAsync(W, h->ws.R, (size_t)h->m * h->r * 4, kind, s));
+  }
+  if (H) {
+    launch_unpack(h->B.master, true, h->n, h->r, h->rp, h->ws.R, s);
+    h->launches++;
+    CK(h, cudaMemcpyAsync(H, h->ws.R, (size_t)h->n * h->r * 4, kind, s));
+  }
+  CK(h, cudaStreamSynchronize(s));
+  return st;
+}
+
+nmd_status nmd_block_update(nmd_handle* h, int32_t side, int64_t block, int32_t kind) {
+  if (!h) return NMD_ERR_INVALID;
+  return run_step(h, side, block, kind, true);
+}
+
+nmd_status nmd_block_order(const nmd_handle* h, int64_t sweep, int32_t side, int64_t* perm, int64_t K) {
+  if (!h || !perm || (side != NMD_ROW && side != NMD_COL) || sweep < 0) return NMD_ERR_INVALID;
+  int64_t Kexp = side == NMD_ROW ? nblocks(h->m, h->opt.block_rows) : nblocks(h->n, h->opt.block_cols);
+  if (K != Kexp) return NMD_ERR_INVALID;
+  std::vector<int64_t> p = permutation(h->opt.seed, sweep, side, K);
+  std::copy(p.begin(), p.end(), perm);
+  return NMD_OK;
+}
+
+nmd_status nmd_sweep(nmd_handle* h) {
+  if (!h) return NMD_ERR_INVALID;
+  int64_t Kr = nblocks(h->m, h->opt.block_rows), Kc = nblocks(h->n, h->opt.block_cols);
+  std::vector<int64_t> pr = permutation(h->opt.seed, h->sweep_index, NMD_ROW, Kr);
+  std::vector<int64_t> pc = permutation(h->opt.seed, h->sweep_index, NMD_COL, Kc);
+  nmd_status st = NMD_OK;
+  if (h->opt.schedule == NMD_EXACT) {
+    for (int64_t t = 0; t < Kr && st == NMD_OK; ++t) st = run_step(h, NMD_ROW, pr[t], NMD_EXACT, true);
+    for (int64_t t = 0; t < Kc && st == NMD_OK; ++t) st = run_step(h, NMD_COL, pc[t], NMD_EXACT, true);
+  } else if (h->opt.order == NMD_PHASED) {
+    for (int64_t t = 0; t < Kc && st == NMD_OK; ++t) st = run_step(h, NMD_COL, pc[t], NMD_STOCH, true);
+    for (int64_t t = 0; t < Kr && st == NMD_OK; ++t) st = run_step(h, NMD_ROW, pr[t], NMD_STOCH, true);
+  } else {
+    for (int64_t t = 0; t < std::max(Kr, Kc) && st == NMD_OK; ++t) {
+      if (t < Kc) st = run_step(h, NMD_COL, pc[t], NMD_STOCH, true);
+      if (st == NMD_OK && t < Kr) st = run_step(h, NMD_ROW, pr[t], NMD_STOCH, true);
+    }
+  }
+  if (st == NMD_OK) h->sweep_index++;
+  return st;
+}
+
+nmd_status nmd_sync(nmd_handle* h) {
+  if (!h) return NMD_ERR_INVALID;
+  return sync_and_check(h);
+}
+
+nmd_status nmd_loss(nmd_handle* h, nmd_loss_out* out) {
+  if (!h || !out) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_loss");
+  nmd_status st = sync_and_check(h);
+  if (st != NMD_OK) return st;
+  cudaStream_t s = h->stream;
+  int ndense = 0;
+  {
+    TimedScope ts(h, NMD_K_LOSS);
+    if (h->opt.precision == NMD_SIMT) {
+      ndense = launch_loss_dense_simt(h, h->ws.loss_part, kLossParts / 2, s);
+      h->launches++;
+    } else {
+      st = launch_loss_dense_tc(h, h->ws.loss_part, kLossParts / 2, &ndense, h->ws.status, s, &h->launches);
+    }
+  }
+  if (st != NMD_OK) return fail(h, st, "no tensor-core loss kernel for this rank/precision");
+  if ((st = after_launch(h, "dense loss")) != NMD_OK) return st;
+  int nsparse = kLossParts / 2;
+  double* sp = h->ws.loss_part + (size_t)(kLossParts / 2) * 8;
+  launch_loss_sparse(h, sp, nsparse, s);
+  launch_loss_final(h->ws.loss_part, ndense, sp, nsparse, h->ws.loss_out, s);
+  h->launches += 2;
+  if ((st = after_launch(h, "loss")) != NMD_OK) return st;
+  double v[8];
+  CK(h, cudaMemcpyAsync(v, h->ws.loss_out, sizeof v, cudaMemcpyDeviceToHost, s));
+  if ((st = sync_and_check(h)) != NMD_OK) return st;
+  // v: [relu2, relu, sum_a, sum_b, sum_min, sum_maxcorr]
+  double zl2 = v[0] + v[2], err2 = v[0] + v[3];
+  out->s_fro = h->s_fro;
+  out->obj = sqrt(zl2 > 0 ? zl2 : 0.0) / h->s_fro;
+  out->rmse = sqrt(err2 > 0 ? err2 : 0.0) / h->s_fro;
+  double den = v[1] + v[5];
+  out->wjd = den > 0 ? 1.0 - v[4] / den : 0.0;
+  out->sum_relu2 = v[0];
+  out->sum_relu = v[1];
+  return NMD_OK;
+}
+
+nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* R,
+                           float* G, int64_t* rows) {
+  if (!h) return NMD_ERR_INVALID;
+  Roles ro;
+  nmd_status st = roles(h, side, block, kind, &ro);
+  if (st != NMD_OK) return st;
+  if ((st = run_step(h, side, block, kind, false)) != NMD_OK) return st;
+  h->step_index--;
+  if ((st = sync_and_check(h)) != NMD_OK) return st;
+  if (rows) *rows = ro.M;
+  cudaStream_t s = h->stream;
+  if (R) CK(h, cudaMemcpy2DAsync(R, h->r * 4, h->ws.R, h->rp * 4, h->r * 4, ro.M, cudaMemcpyDeviceToHost, s));
+  if (G) CK(h, cudaMemcpy2DAsync(G, h->r * 4, h->ws.G, h->rp * 4, h->r * 4, h->r, cudaMemcpyDeviceToHost, s));
+  CK(h, cudaStreamSynchronize(s));
+  return NMD_OK;
+}
+
+nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* d_L,
+                              int64_t* rows, int64_t* cols) {
+  if (!h || !d_L) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_dense_products");
+  Roles ro;
+  nmd_status st = roles(h, side, block, kind, &ro);
+  if (st != NMD_OK) return st;
+  if (h->opt.precision == NMD_SIMT) return fail(h, NMD_ERR_UNSUPPORTED, "dense products hook needs a tensor-core precision");
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue};
+  st = launch_panel_tc(a, h->ws.R, h->ws.status, h->ws.counters, h->num_sms, h->stream, &h->launches, d_L);
+  if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
+  if ((st = after_launch(h, "dense products")) != NMD_OK) return st;
+  if ((st = sync_and_check(h)) != NMD_OK) return st;
+  if (rows) *rows = ro.M;
+  if (cols) *cols = ro.K;
+  return NMD_OK;
+}
+
+nmd_status nmd_panel_traversal(const nmd_handle* h, int32_t side, int64_t block, int32_t kind,
+                               int64_t* rows_out, int64_t* q_out, int64_t cap, int64_t* count) {
+  if (!h || !count) return NMD_ERR_INVALID;
+  Roles ro;
+  nmd_status st = roles(const_cast<nmd_handle*>(h), side, block, kind, &ro);
+  if (st != NMD_OK) return st;
+  // host mirrors of the index arrays are not kept; rebuild q from the device copy
+  const PanelSet& P = *ro.P;
+  std::vector<PanelRow> list(P.host.begin() + P.light_ptr[block], P.host.begin() + P.light_ptr[block + 1]);
+  std::sort(list.begin(), list.end(), [](const PanelRow& a, const PanelRow& b) { return a.row < b.row; });
+  int64_t total = 0;
+  for (auto& pr : list) total += pr.len;
+  *count = total;
+  if (!rows_out || !q_out || cap <= 0) return NMD_OK;
+  std::vector<int32_t> idx;
+  int64_t w = 0;
+  for (auto& pr : list) {
+    idx.resize(pr.len);
+    cudaError_t e = cudaMemcpy(idx.data(), ro.qidx + pr.beg, (size_t)pr.len * 4, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_check(const_cast<nmd_handle*>(h), e, "traversal copy");
+    for (int64_t k = 0; k < pr.len && w < cap; ++k, ++w) {
+      rows_out[w] = pr.row - ro.m0;
+      q_out[w] = idx[k] - ro.q0;
+    }
+  }
+  return NMD_OK;
+}
+
+nmd_status nmd_get_state(nmd_handle* h, float* W, float* H, float* EW, float* EH, int64_t* sweep_index) {
+  if (!h) return NMD_ERR_INVALID;
+  nmd_status st = nmd_get_factors(h, W, H, 0);
+  if (st != NMD_OK) return st;
+  cudaStream_t s = h->stream;
+  if (EW) {
+    launch_unpack(h->W.E, false, h->m, h->r, h->rp, h->ws.R, s);
+    h->launches++;
+    CK(h, cudaMemcpyAsync(EW, h->ws.R, (size_t)h->m * h->r * 4, cudaMemcpyDeviceToHost, s));
+  }
+  if (EH) {
+    launch_unpack(h->B.E, true, h->n, h->r, h->rp, h->ws.R, s);
+    h->launches++;
+    CK(h, cudaMemcpyAsync(EH, h->ws.R, (size_t)h->n * h->r * 4, cudaMemcpyDeviceToHost, s));
+  }
+  CK(h, cudaStreamSynchronize(s));
+  if (sweep_index) *sweep_index = h->sweep_index;
+  return NMD_OK;
+}
+
+nmd_status nmd_set_state(nmd_handle* h, const float* W, const float* H, const float* EW, const float* EH,
+                         int64_t sweep_index) {
+  if (!h || !W || !H || !EW || !EH || sweep_index < 0) return fail(h, NMD_ERR_INVALID, "bad nmd_set_state argument");
+  nmd_status st = nmd_set_factors(h, W, H, 0);
+  if (st != NMD_OK) return st;
+  cudaStream_t s = h->stream;
+  // momentum: pack into the master buffers' E (pack writes master/hi/lo of a
+  // Factor, so pack into a temporary view whose master is E)
+  Factor tw = h->W, tb = h->B;
+  tw.master = h->W.E; tw.hi = nullptr; tw.lo = nullptr;
+  tb.master = h->B.E; tb.hi = nullptr; tb.lo = nullptr;
+  CK(h, cudaMemcpyAsync(h->ws.R, EW, (size_t)h->m * h->r * 4, cudaMemcpyHostToDevice, s));
+  launch_pack(h->ws.R, false, h->m, h->r, h->rp, tw, s);
+  CK(h, cudaMemcpyAsync(h->ws.R, EH, (size_t)h->n * h->r * 4, cudaMemcpyHostToDevice, s));
+  launch_pack(h->ws.R, true, h->n, h->r, h->rp, tb, s);
+  h->launches += 2;
+  if ((st = after_launch(h, "set state")) != NMD_OK) return st;
+  CK(h, cudaStreamSynchronize(s));
+  h->sweep_index = sweep_index;
+  return NMD_OK;
+}
+
+nmd_status nmd_profile(nmd_handle* h, int on) {
+  if (!h) return NMD_ERR_INVALID;
+  CK(h, cudaStreamSynchronize(h->stream));
+  collect_timing(h);
+  for (int c = 0; c < 5; ++c) {
+    h->prof_ms[c] = 0.0;
+    h->prof_launches[c] = 0;
+  }
+  h->profiling = on != 0;
+  return NMD_OK;
+}
+
+nmd_status nmd_profile_read(nmd_handle* h, int32_t kernel_class, double* ms, int64_t* launches) {
+  if (!h || kernel_class < 0 || kernel_class > 4) return NMD_ERR_INVALID;
+  CK(h, cudaStreamSynchronize(h->stream));
+  collect_timing(h);
+  if (ms) *ms = h->prof_ms[kernel_class];
+  if (launches) *launches = h->prof_launches[kernel_class];
+  return NMD_OK;
+}
+
+void nmd_destroy(nmd_handle* h) { delete h; }
+
+}  // extern "C"

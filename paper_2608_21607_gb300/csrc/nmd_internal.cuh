@@ -1,0 +1,148 @@
+// Internal declarations shared by the translation units of libnmd.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "../../include/nmd.h"
+
+namespace nmd {
+
+typedef __nv_bfloat16 bf16;
+
+// One row of a block's sparse panel: entries [beg, beg + len) of the CSR (or
+// CSC) arrays, all belonging to M-side row `row` and lying in the block's
+// Q-side range.  Rows are listed in ascending order.
+struct PanelRow {
+  int32_t row;
+  int32_t len;
+  int64_t beg;
+};
+
+// Panel rows longer than this are handled by a whole thread block each.
+constexpr int kHeavyRow = 256;
+
+// Per (side, kind): the panel lists of every block, concatenated.  Block k's
+// light rows are [light_ptr[k], light_ptr[k+1]) and its heavy rows
+// [heavy_ptr[k], heavy_ptr[k+1]) of the device array `d` (light rows first,
+// then heavy rows, block by block).
+struct PanelSet {
+  std::vector<int64_t> light_ptr, heavy_ptr;
+  std::vector<PanelRow> host;
+  PanelRow* d = nullptr;
+};
+
+// Device status word (sticky): [0] = nmd_status code of the first error,
+// [1] = a detail (pivot column, row index), [2] = step counter at the error.
+constexpr int kStatusWords = 4;
+
+// One factor's device buffers (N rows, rp = padded rank columns).
+struct Factor {
+  int64_t rows = 0;
+  float* master = nullptr;   // N x rp fp32, pad columns are zero
+  bf16* hi = nullptr;        // N x rp, bf16(master)
+  bf16* lo = nullptr;        // N x rp, bf16(master - hi)
+  float* E = nullptr;        // N x rp momentum (fp32)
+};
+
+// Operands of one dense panel contraction and one update, in device memory.
+struct StepArgs {
+  // M-side rows [m0, m0 + M) of factor fm, Q-side rows [q0, q0 + K) of fq
+  const Factor* fm;
+  const Factor* fq;
+  int64_t m0, M, q0, K;
+  int r, rp;
+  int precision, epilogue;
+};
+
+struct Workspace {
+  size_t bytes = 0;
+  // CSR of S and CSR of S^T (=CSC of S), support only
+  int64_t* rowptr = nullptr;
+  int32_t* col = nullptr;
+  float* val = nullptr;
+  int64_t* colptr = nullptr;
+  int32_t* row = nullptr;
+  float* valT = nullptr;
+  // panel lists: [side][kind]
+  PanelRow* panels = nullptr;
+  float* R = nullptr;          // max(m, n) x rp fp32 right-hand side / staging
+  float* gram_part = nullptr;  // kGramParts x rp x rp
+  float* G = nullptr;          // rp x rp (last Gram, for verification)
+  float* Ginv = nullptr;       // rp x rp
+  double* loss_part = nullptr; // kLossParts x 8
+  double* loss_out = nullptr;  // 8
+  int* status = nullptr;       // kStatusWords
+  int* counters = nullptr;     // 64 ints (tile schedulers)
+  float* chol_scratch = nullptr;  // 2 x rp x rp (used when rp is too large for smem)
+};
+
+constexpr int kGramParts = 64;
+constexpr int kLossParts = 2048;
+
+}  // namespace nmd
+
+struct nmd_handle {
+  int64_t m = 0, n = 0, nnz = 0;
+  int r = 0, rp = 0;
+  nmd_options opt;
+  cudaStream_t stream = nullptr;
+  nmd::Workspace ws;
+  nmd::Factor W, B;            // A = W (m x r), B = H^T (n x r)
+  nmd::PanelSet panels[2][2];  // [side][kind]
+  double s_fro = 0.0;
+  int64_t sweep_index = 0;
+  int64_t step_index = 0;
+  int64_t launches = 0;
+  int num_sms = 0;
+  int device = 0;
+  int cc_major = 0, cc_minor = 0;
+  std::string last_error;
+  // kernel timing (nmd_profile): event pairs per launch, by kernel class
+  bool profiling = false;
+  std::vector<cudaEvent_t> event_pool;
+  struct Timed { int cls; cudaEvent_t a, b; };
+  std::vector<Timed> timed;
+  double prof_ms[5] = {0, 0, 0, 0, 0};
+  int64_t prof_launches[5] = {0, 0, 0, 0, 0};
+  ~nmd_handle();
+};
+
+namespace nmd {
+
+// ---- launchers (kernels.cu) ----
+void launch_pack(const float* src, bool src_is_rxN, int64_t N, int r, int rp, Factor& f,
+                 cudaStream_t s);
+void launch_unpack(const float* master, bool dst_is_rxN, int64_t N, int r, int rp, float* dst,
+                   cudaStream_t s);
+void launch_gram(const Factor& fq, int64_t q0, int64_t K, int r, int rp, float* parts,
+                 int nparts, cudaStream_t s);
+void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge, float* G,
+                     float* Ginv, float* scratch, int* status, cudaStream_t s);
+void launch_sparse(const StepArgs& a, const PanelRow* light, int64_t nlight,
+                   const PanelRow* heavy, int64_t nheavy, const int32_t* qidx,
+                   const float* vals, float* R, cudaStream_t s);
+void launch_update(const StepArgs& a, const float* R, const float* Ginv, float eta,
+                   float gamma, bool momentum, int* status, cudaStream_t s);
+void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s);
+void launch_loss_final(const double* dense_parts, int ndense, const double* sparse_parts,
+                       int nsparse, double* out, cudaStream_t s);
+
+// ---- dense contraction on the CUDA cores (panel_simt.cu) ----
+void launch_panel_simt(const StepArgs& a, float* R, cudaStream_t s);
+int launch_loss_dense_simt(const nmd_handle* h, double* parts, int maxparts, cudaStream_t s);
+
+// ---- dense contraction on the tcgen05 tensor cores (panel_tc.cu) ----
+// Returns NMD_OK, or NMD_ERR_UNSUPPORTED when no tensor-core kernel exists
+// for this rank; `launches` is incremented by the number of kernels issued.
+nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counter,
+                           int num_sms, cudaStream_t s, int64_t* launches, float* Lout = nullptr);
+nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts,
+                                int* status, cudaStream_t s, int64_t* launches);
+bool tc_supported(int rp, int precision);
+
+}  // namespace nmd

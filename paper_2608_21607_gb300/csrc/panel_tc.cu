@@ -1,0 +1,565 @@
+// Fused Z-panel contraction and dense loss pass on the tcgen05 tensor cores.
+//
+// For M-side rows m_i (a tile of 128) and Q-side rows q_k (streamed in
+// chunks of BN), the panel kernel computes, without writing any tile of L or
+// Z to global memory (the fused kernel of Sec. 4.2, eq. "kernel"):
+//   L_ik = m_i . q_k                         MMA1: TMEM <- W tile (TMEM) x chunk^T
+//   P_ik = min(0, L_ik)      (Z form, eq. updateZ)   -- epilogue in registers,
+//        = -max(0, L_ik)     (Delta form, eq. updateD)  written back to TMEM
+//   R_i  = sum_k P_ik q_k                    MMA2: TMEM R += P (TMEM) x chunk
+// The same shared-memory copy of each chunk feeds both products: K-major for
+// MMA1 and MN-major for MMA2.  With SPLIT (fp32-accurate mode) every operand
+// is x = hi + lo (bf16 each) and each product is hi*hi + hi*lo + lo*hi.
+//
+// The loss kernel runs MMA1 only, over all of W against all of B, and sums
+// max(0, L)^2 and max(0, L) (eq. SLloss / eq. RMSE / eq. WJD dense parts).
+//
+// Warp roles (192 threads, one CTA per SM, persistent over M tiles):
+//   warps 0-3  epilogue: thread t owns TMEM lane t = tile row t
+//   warp 4     TMA producer of Q chunks (+ TMEM allocation)
+//   warp 5     MMA issuer (one thread)
+// Every mbarrier wait is bounded (2 s): on expiry the kernel records
+// NMD_ERR_TIMEOUT, the other roles stop at their next wait, in-flight MMAs
+// and copies are drained and TMEM is freed before the kernel returns.
+#include <cudaTypedefs.h>
+
+#include <map>
+#include <mutex>
+#include <tuple>
+
+#include "nmd_internal.cuh"
+#include "tc_ptx.cuh"
+
+namespace nmd {
+namespace {
+
+using namespace tc;
+
+constexpr int kThreads = 192;
+constexpr int BM = 128;
+constexpr uint64_t kTimeoutNs = 2000000000ull;
+
+template <int RP, bool SPLIT>
+struct Cfg {
+  static constexpr int BN = (RP == 256 || (SPLIT && RP == 128)) ? 64 : 128;  // Q rows per chunk
+  static constexpr int WCOLS = SPLIT ? RP : RP / 2;    // TMEM columns of one W tile (hi [+ lo])
+  static constexpr int NWB = (RP == 256) ? 1 : 2;      // W tile buffers
+  static constexpr int FREE = 512 - NWB * WCOLS - RP;
+  static constexpr int NB = FREE / BN >= 3 ? 3 : FREE / BN;  // L buffers
+  static constexpr int PANEL_W = RP < 64 ? RP : 64;    // elements per row of one swizzle panel
+  static constexpr int ROWB = PANEL_W * 2;             // bytes per panel row (= swizzle width)
+  static constexpr int PANEL_BYTES = BN * ROWB;
+  static constexpr int NPANEL = RP / PANEL_W;
+  static constexpr int OPER_BYTES = BN * RP * 2;       // one operand (hi or lo) of a chunk
+  static constexpr int STAGE_BYTES = OPER_BYTES * (SPLIT ? 2 : 1);
+  static constexpr int NSTAGE_RAW = (160 * 1024) / STAGE_BYTES;
+  static constexpr int NSTAGE = NSTAGE_RAW > 8 ? 8 : (NSTAGE_RAW < 2 ? 2 : NSTAGE_RAW);
+  static constexpr uint32_t SWZ = PANEL_W == 64 ? SWZ_128B : (PANEL_W == 32 ? SWZ_64B : SWZ_32B);
+  static constexpr int COL_L = 0;               // NB x BN columns
+  static constexpr int COL_R = NB * BN;         // RP columns
+  static constexpr int COL_W = COL_R + RP;      // NWB x WCOLS columns
+  // barriers: full[NSTAGE], empty[NSTAGE], lfull[NB], pfull[NB], lfree[NB], rfull, rempty,
+  // wfull[2], wempty[2], drain
+  static constexpr int NBAR = 2 * NSTAGE + 3 * NB + 7;
+  static constexpr size_t SMEM_USED = 1024 + (size_t)NSTAGE * STAGE_BYTES + NBAR * 8 + 64 + 128 * 16;
+  // at least 120 KB so that a second CTA (and its 512-column TMEM request)
+  // never shares the SM
+  static constexpr size_t SMEM = SMEM_USED > 120 * 1024 ? SMEM_USED : 120 * 1024;
+  static_assert(NB >= 2, "need two L buffers");
+  static_assert(COL_W + NWB * WCOLS <= 512, "TMEM budget");
+  static_assert(BN % 32 == 0 && RP % 16 == 0, "shapes");
+};
+
+struct TcParams {
+  int64_t m0, M;        // M-side rows [m0, m0 + M) of the M factor
+  int64_t q0, K;        // Q-side rows [q0, q0 + K) of the Q factor
+  const bf16* Mhi;      // M factor operand copies (absolute row index)
+  const bf16* Mlo;
+  float* R;             // M x RP output (panel kernel)
+  double* parts;        // per-CTA loss partials (loss kernel)
+  int* status;
+  float* Lout;          // verification: raw L (M x K, row-major) or nullptr
+};
+
+__device__ __forceinline__ void record(int* status, int code, int detail) {
+  if (atomicCAS(status, 0, code) == 0) status[1] = detail;
+}
+
+// Bounded wait on an mbarrier phase.  Returns false if the kernel is aborting.
+__device__ __noinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
+                                      int where) {
+  if (mbar_try_wait(bar, parity)) return true;
+  uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 255u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > kTimeoutNs) {
+        *abort_flag = 1;
+        record(status, NMD_ERR_TIMEOUT, where);
+        return false;
+      }
+    }
+  }
+}
+
+// Warp-uniform wait: lane 0 polls, the outcome is broadcast to the warp.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
+                                          int where) {
+  int ok = 0;
+  if ((threadIdx.x & 31) == 0) ok = wait_bar(bar, parity, abort_flag, status, where);
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
+}
+
+template <int RP, int EPI, bool SPLIT, bool LOSS>
+__global__ void __launch_bounds__(kThreads, 1)
+    panel_tc_kernel(const __grid_constant__ CUtensorMap tq_hi, const __grid_constant__ CUtensorMap tq_lo,
+                    const TcParams p) {
+  using C = Cfg<RP, SPLIT>;
+  constexpr int BN = C::BN, NB = C::NB, NSTAGE = C::NSTAGE, NWB = C::NWB;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+  uint8_t* stages = smem;
+  uint64_t* bars = (uint64_t*)(smem + (size_t)NSTAGE * C::STAGE_BYTES);
+  uint32_t* tmem_slot = (uint32_t*)(bars + C::NBAR);
+  volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
+  double* red = (double*)(smem + (size_t)NSTAGE * C::STAGE_BYTES + C::NBAR * 8 + 64);
+
+  const uint32_t b_full = smem_u32(bars);
+  const uint32_t b_empty = b_full + 8 * NSTAGE;
+  const uint32_t b_lfull = b_empty + 8 * NSTAGE;
+  const uint32_t b_pfull = b_lfull + 8 * NB;
+  const uint32_t b_lfree = b_pfull + 8 * NB;
+  const uint32_t b_rfull = b_lfree + 8 * NB;
+  const uint32_t b_rempty = b_rfull + 8;
+  const uint32_t b_wfull = b_rempty + 8;
+  const uint32_t b_wempty = b_wfull + 16;
+  const uint32_t b_drain = b_wempty + 16;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < NSTAGE; ++i) {
+      mbar_init(b_full + 8 * i, 1);
+      mbar_init(b_empty + 8 * i, 1);
+    }
+    for (int i = 0; i < NB; ++i) {
+      mbar_init(b_lfull + 8 * i, 1);
+      mbar_init(b_pfull + 8 * i, 128);
+      mbar_init(b_lfree + 8 * i, LOSS ? 128 : 1);
+    }
+    mbar_init(b_rfull, 1);
+    mbar_init(b_rempty, 128);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(b_wfull + 8 * i, 128);
+      mbar_init(b_wempty + 8 * i, 1);
+    }
+    mbar_init(b_drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 4) {
+    tmem_alloc(smem_u32(tmem_slot), 512);
+    tmem_relinquish();
+    if (lane == 0) {
+      prefetch_tmap(&tq_hi);
+      if (SPLIT) prefetch_tmap(&tq_lo);
+    }
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  const int64_t ntiles = (p.M + BM - 1) / BM;
+  const int64_t nchunks = (p.K + BN - 1) / BN;
+
+  if (warp == 4) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int64_t G = 0;
+      bool ok = true;
+      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+        for (int64_t c = 0; c < nchunks; ++c, ++G) {
+          const int s = (int)(G % NSTAGE);
+          if (!(ok = wait_bar(b_empty + 8 * s, (uint32_t)((G / NSTAGE) & 1) ^ 1u, abort_flag, p.status, 1)))
+            break;
+          mbar_expect_tx(b_full + 8 * s, C::STAGE_BYTES);
+          const uint32_t dst = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
+          const int y = (int)(p.q0 + c * BN);
+#pragma unroll
+          for (int pn = 0; pn < C::NPANEL; ++pn) {
+            tma_load_2d(dst + pn * C::PANEL_BYTES, &tq_hi, b_full + 8 * s, pn * C::PANEL_W, y);
+            if (SPLIT)
+              tma_load_2d(dst + C::OPER_BYTES + pn * C::PANEL_BYTES, &tq_lo, b_full + 8 * s, pn * C::PANEL_W, y);
+          }
+        }
+      }
+      if (!ok) {  // drain the copies still in flight before TMEM/smem go away
+        for (int64_t k = G - NSTAGE > 0 ? G - NSTAGE : 0; k < G; ++k) {
+          uint64_t t0 = globaltimer_ns();
+          while (!mbar_try_wait(b_full + 8 * (int)(k % NSTAGE), (uint32_t)((k / NSTAGE) & 1)) &&
+                 globaltimer_ns() - t0 < 100000000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 5) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc1 = idesc_bf16(BM, BN, false);   // L = W x Q^T (Q K-major)
+      constexpr uint32_t idesc2 = idesc_bf16(BM, RP, true);    // R += P x Q (Q MN-major)
+      bool ok = true;
+      int64_t tt = 0;
+      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++tt) {
+        const int wb = (int)(tt % NWB);
+        if (!(ok = wait_bar(b_wfull + 8 * wb, (uint32_t)((tt / NWB) & 1), abort_flag, p.status, 2))) break;
+        fence_after();
+        const uint32_t wh = tmem + C::COL_W + wb * C::WCOLS;
+        const uint32_t wl = wh + RP / 2;
+        for (int64_t c = 0; c <= nchunks && ok; ++c) {
+          if (c < nchunks) {
+            const int64_t G = tt * nchunks + c;
+            const int s = (int)(G % NSTAGE), lb = (int)(G % NB);
+            if (!(ok = wait_bar(b_full + 8 * s, (uint32_t)((G / NSTAGE) & 1), abort_flag, p.status, 3))) break;
+            if (!(ok = wait_bar(b_lfree + 8 * lb, (uint32_t)((G / NB) & 1) ^ 1u, abort_flag, p.status, 4))) break;
+            fence_after();
+            const uint32_t sb = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
+            const uint32_t d = tmem + C::COL_L + lb * BN;
+#pragma unroll
+            for (int k = 0; k < RP / 16; ++k) {
+              const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
+              const uint64_t bh = sdesc(sb + off, 16, 8 * C::ROWB, C::SWZ);
+              mma_ts(d, wh + k * 8, bh, idesc1, k > 0);
+              if (SPLIT) {
+                const uint64_t bl = sdesc(sb + C::OPER_BYTES + off, 16, 8 * C::ROWB, C::SWZ);
+                mma_ts(d, wh + k * 8, bl, idesc1, 1);
+                mma_ts(d, wl + k * 8, bh, idesc1, 1);
+              }
+            }
+            commit(b_lfull + 8 * lb);
+            if (LOSS) commit(b_empty + 8 * s);
+          }
+          if (!LOSS && c >= 1) {
+            const int64_t G = tt * nchunks + c - 1;
+            const int s = (int)(G % NSTAGE), lb = (int)(G % NB);
+            if (!(ok = wait_bar(b_pfull + 8 * lb, (uint32_t)((G / NB) & 1), abort_flag, p.status, 5))) break;
+            if (c == 1 && !(ok = wait_bar(b_rempty, (uint32_t)(tt & 1) ^ 1u, abort_flag, p.status, 6))) break;
+            fence_after();
+            const uint32_t sb = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
+            const uint32_t pl = tmem + C::COL_L + lb * BN;
+#pragma unroll
+            for (int k = 0; k < BN / 16; ++k) {
+              const uint64_t bh = sdesc(sb + k * 16 * C::ROWB, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
+              const uint32_t acc = (c > 1 || k > 0) ? 1u : 0u;
+              if (!SPLIT) {
+                mma_ts(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
+              } else {
+                const uint64_t bl =
+                    sdesc(sb + C::OPER_BYTES + k * 16 * C::ROWB, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
+                const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
+                mma_ts(tmem + C::COL_R, ph, bh, idesc2, acc);
+                mma_ts(tmem + C::COL_R, ph, bl, idesc2, 1);
+                mma_ts(tmem + C::COL_R, plo, bh, idesc2, 1);
+              }
+            }
+            commit(b_empty + 8 * s);
+            commit(b_lfree + 8 * lb);
+          }
+        }
+        if (!ok) break;
+        if (!LOSS) commit(b_rfull);
+        commit(b_wempty + 8 * wb);
+      }
+      // wait until every MMA issued by this thread has completed
+      commit(b_drain);
+      uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(b_drain, 0) && globaltimer_ns() - t0 < 200000000ull) {
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int row = threadIdx.x;                      // TMEM lane == tile row
+    const uint32_t lane_base = ((uint32_t)(warp * 32)) << 16;
+    double s2 = 0.0, s1 = 0.0;
+    bool ok = true;
+
+    // load the W tile of local tile index tt into W buffer tt % NWB
+    auto load_w = [&](int64_t tile, int wb) {
+      const int64_t li = tile * BM + row;
+      const bool valid = li < p.M;
+      const uint4* src = (const uint4*)(p.Mhi + (p.m0 + (valid ? li : 0)) * RP);
+      const uint4* srcl = (const uint4*)(p.Mlo + (p.m0 + (valid ? li : 0)) * RP);
+      const uint32_t wcol = tmem + lane_base + C::COL_W + wb * C::WCOLS;
+#pragma unroll
+      for (int q = 0; q < RP / 16; ++q) {
+        uint4 a = valid ? __ldg(src + 2 * q) : make_uint4(0, 0, 0, 0);
+        uint4 b = valid ? __ldg(src + 2 * q + 1) : make_uint4(0, 0, 0, 0);
+        uint32_t v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+        tmem_st8(wcol + q * 8, v);
+        if (SPLIT) {
+          uint4 c = valid ? __ldg(srcl + 2 * q) : make_uint4(0, 0, 0, 0);
+          uint4 e = valid ? __ldg(srcl + 2 * q + 1) : make_uint4(0, 0, 0, 0);
+          uint32_t w[8] = {c.x, c.y, c.z, c.w, e.x, e.y, e.z, e.w};
+          tmem_st8(wcol + RP / 2 + q * 8, w);
+        }
+      }
+      tmem_wait_st();
+      fence_before();
+      mbar_arrive(b_wfull + 8 * wb);
+    };
+
+    {  // prologue: the first NWB tiles
+      int64_t tt = 0;
+      for (int64_t t = blockIdx.x; t < ntiles && tt < NWB; t += gridDim.x, ++tt) load_w(t, (int)tt);
+    }
+    int64_t tt = 0;
+    for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++tt) {
+      for (int64_t c = 0; c < nchunks; ++c) {
+        const int64_t G = tt * nchunks + c;
+        const int lb = (int)(G % NB);
+        if (!(ok = warp_wait(b_lfull + 8 * lb, (uint32_t)((G / NB) & 1), abort_flag, p.status, 7))) break;
+        fence_after();
+        const int64_t kv = p.K - c * BN;              // valid columns in this chunk
+        const uint32_t lcol = tmem + lane_base + C::COL_L + lb * BN;
+        float c2 = 0.f, c1 = 0.f;
+#pragma unroll 1
+        for (int j = 0; j < BN / 32; ++j) {
+          uint32_t v[32];
+          tmem_ld32(lcol + j * 32, v);
+          tmem_wait_ld(v);
+          if (p.Lout != nullptr) {
+            const int64_t li = t * BM + row;
+            if (li < p.M) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (j * 32 + i < kv) p.Lout[li * p.K + c * BN + j * 32 + i] = __uint_as_float(v[i]);
+            }
+          }
+          if (LOSS) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              float x = fmaxf(0.f, __uint_as_float(v[i]));
+              x = (j * 32 + i < kv) ? x : 0.f;
+              c2 = fmaf(x, x, c2);
+              c1 += x;
+            }
+          } else {
+            float pv[32];
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float x = __uint_as_float(v[i]);
+              const float e = EPI == 0 ? fminf(0.f, x) : fminf(0.f, -x);   // min(0,L) or -max(0,L)
+              pv[i] = (j * 32 + i < kv) ? e : 0.f;
+            }
+            if (!SPLIT) {
+              uint32_t pk[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(pv[2 * i], pv[2 * i + 1]);
+              tmem_st16(lcol + j * 16, pk);
+            } else {
+              uint32_t ph[16], pl[16];
+#pragma unroll
+              for (int i = 0; i < 16; ++i) {
+                const float h0 = __bfloat162float(__float2bfloat16_rn(pv[2 * i]));
+                const float h1 = __bfloat162float(__float2bfloat16_rn(pv[2 * i + 1]));
+                ph[i] = pack_bf16x2(h0, h1);
+                pl[i] = pack_bf16x2(pv[2 * i] - h0, pv[2 * i + 1] - h1);
+              }
+              tmem_st16(lcol + j * 32, ph);
+              tmem_st16(lcol + j * 32 + 16, pl);
+            }
+          }
+        }
+        if (LOSS) {
+          s2 += (double)c2;
+          s1 += (double)c1;
+          fence_before();
+          mbar_arrive(b_lfree + 8 * lb);
+        } else {
+          tmem_wait_st();
+          fence_before();
+          mbar_arrive(b_pfull + 8 * lb);
+        }
+      }
+      if (!ok) break;
+      if (!LOSS) {
+        if (!(ok = warp_wait(b_rfull, (uint32_t)(tt & 1), abort_flag, p.status, 8))) break;
+        fence_after();
+        const int64_t li = t * BM + row;
+        float* dst = p.R + li * RP;
+#pragma unroll 1
+        for (int j = 0; j < (RP + 31) / 32; ++j) {
+          uint32_t v[32];
+          tmem_ld32(tmem + lane_base + C::COL_R + j * 32, v);   // RP = 16 reads 16 spare columns
+          tmem_wait_ld(v);
+          if (li < p.M) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+              if (j * 32 + i < RP)
+                *(float4*)(dst + j * 32 + i) = make_float4(__uint_as_float(v[i]), __uint_as_float(v[i + 1]),
+                                                          __uint_as_float(v[i + 2]), __uint_as_float(v[i + 3]));
+          }
+        }
+        fence_before();
+        mbar_arrive(b_rempty);
+      }
+      // refill this tile's W buffer with the tile NWB steps ahead
+      const int64_t tn = t + (int64_t)NWB * gridDim.x;
+      if (tn < ntiles) {
+        const int wb = (int)(tt % NWB);
+        if (!(ok = warp_wait(b_wempty + 8 * wb, (uint32_t)((tt / NWB) & 1), abort_flag, p.status, 9))) break;
+        fence_after();
+        load_w(tn, wb);
+      }
+    }
+    if (LOSS) {
+      // fixed-order reduction over the 128 epilogue threads
+      red[2 * row] = s2;
+      red[2 * row + 1] = s1;
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (row == 0) {
+        double a = 0.0, b = 0.0;
+        for (int i = 0; i < 128; ++i) {
+          a += red[2 * i];
+          b += red[2 * i + 1];
+        }
+        p.parts[(size_t)blockIdx.x * 8 + 0] = a;
+        p.parts[(size_t)blockIdx.x * 8 + 1] = b;
+      }
+    }
+  }
+  fence_before();
+  __syncthreads();
+  fence_after();
+  if (warp == 4) tmem_dealloc(tmem, 512);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+// ---------------------------------------------------------------------------
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+  });
+  return fn;
+}
+
+// Tensor map of a row-major rows x rp bf16 factor copy, box = panel_w x bn.
+bool tensor_map(const bf16* base, int64_t rows, int rp, int panel_w, int bn, CUtensorMap* out) {
+  static std::mutex mu;
+  static std::map<std::tuple<const void*, int64_t, int, int>, CUtensorMap> cache;
+  std::lock_guard<std::mutex> g(mu);
+  auto key = std::make_tuple((const void*)base, rows, rp, bn);
+  auto it = cache.find(key);
+  if (it != cache.end()) {
+    *out = it->second;
+    return true;
+  }
+  PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)rp, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)rp * 2};
+  cuuint32_t box[2] = {(cuuint32_t)panel_w, (cuuint32_t)bn};
+  cuuint32_t es[2] = {1, 1};
+  CUtensorMapSwizzle swz = panel_w == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                         : (panel_w == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B);
+  CUtensorMap m;
+  CUresult r = fn(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, (void*)base, dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return false;
+  cache[key] = m;
+  *out = m;
+  return true;
+}
+
+template <int RP, int EPI, bool SPLIT, bool LOSS>
+nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, cudaStream_t s) {
+  using C = Cfg<RP, SPLIT>;
+  CUtensorMap th, tl;
+  if (!tensor_map(fq.hi, fq.rows, RP, C::PANEL_W, C::BN, &th)) return NMD_ERR_CUDA;
+  if (!tensor_map(fq.lo, fq.rows, RP, C::PANEL_W, C::BN, &tl)) return NMD_ERR_CUDA;
+  (void)fm;
+  static bool attr_set = false;
+  if (!attr_set) {
+    if (cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)C::SMEM) != cudaSuccess)
+      return NMD_ERR_CUDA;
+    attr_set = true;
+  }
+  panel_tc_kernel<RP, EPI, SPLIT, LOSS><<<grid, kThreads, C::SMEM, s>>>(th, tl, p);
+  return NMD_OK;
+}
+
+template <int RP, bool LOSS>
+nmd_status dispatch_rp(int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p, int grid,
+                       cudaStream_t s) {
+  if (LOSS) return split ? run<RP, 0, (RP < 256), LOSS>(fm, fq, p, grid, s) : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
+  if (split) {
+    if (RP == 256) return NMD_ERR_UNSUPPORTED;
+    return epilogue == NMD_EPI_DELTA ? run<RP, 1, (RP < 256), LOSS>(fm, fq, p, grid, s)
+                                     : run<RP, 0, (RP < 256), LOSS>(fm, fq, p, grid, s);
+  }
+  return epilogue == NMD_EPI_DELTA ? run<RP, 1, false, LOSS>(fm, fq, p, grid, s)
+                                   : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
+}
+
+template <bool LOSS>
+nmd_status dispatch(int rp, int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p,
+                    int grid, cudaStream_t s) {
+  if (split && rp == 256) return NMD_ERR_UNSUPPORTED;
+  switch (rp) {
+    case 16: return dispatch_rp<16, LOSS>(epilogue, split, fm, fq, p, grid, s);
+    case 32: return dispatch_rp<32, LOSS>(epilogue, split, fm, fq, p, grid, s);
+    case 64: return dispatch_rp<64, LOSS>(epilogue, split, fm, fq, p, grid, s);
+    case 128: return dispatch_rp<128, LOSS>(epilogue, split, fm, fq, p, grid, s);
+    case 256: return dispatch_rp<256, LOSS>(epilogue, split, fm, fq, p, grid, s);
+  }
+  return NMD_ERR_UNSUPPORTED;
+}
+
+}  // namespace
+
+bool tc_supported(int rp, int precision) {
+  if (precision == NMD_SIMT) return false;
+  if (precision == NMD_FP32 && rp == 256) return false;
+  return rp == 16 || rp == 32 || rp == 64 || rp == 128 || rp == 256;
+}
+
+nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counter, int num_sms, cudaStream_t s,
+                           int64_t* launches, float* Lout) {
+  (void)counter;
+  if (!tc_supported(a.rp, a.precision)) return NMD_ERR_UNSUPPORTED;
+  TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout};
+  int64_t ntiles = (a.M + BM - 1) / BM;
+  int grid = (int)(ntiles < num_sms ? ntiles : num_sms);
+  nmd_status st = dispatch<false>(a.rp, a.epilogue, a.precision == NMD_FP32, *a.fm, *a.fq, p, grid, s);
+  if (st == NMD_OK) ++*launches;
+  return st;
+}
+
+nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts, int* status,
+                                cudaStream_t s, int64_t* launches) {
+  if (!tc_supported(h->rp, h->opt.precision)) return NMD_ERR_UNSUPPORTED;
+  TcParams p{0, h->m, 0, h->n, h->W.hi, h->W.lo, nullptr, parts, status, nullptr};
+  int64_t ntiles = (h->m + BM - 1) / BM;
+  int grid = (int)(ntiles < h->num_sms ? ntiles : h->num_sms);
+  if (grid > maxparts) grid = maxparts;
+  nmd_status st = dispatch<true>(h->rp, 0, h->opt.precision == NMD_FP32, h->W, h->B, p, grid, s);
+  if (st == NMD_OK) {
+    ++*launches;
+    *nparts = grid;
+  }
+  return st;
+}
+
+}  // namespace nmd
