@@ -141,6 +141,37 @@ nmd_status build_sparse(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   return NMD_OK;
 }
 
+// Split every block's rows (ascending) into single rows (len <= kSeg) and
+// segments of kSeg entries for the longer rows.
+void finalize_panels(const std::vector<std::vector<PanelRow>>& per, PanelSet* P) {
+  int64_t K = (int64_t)per.size();
+  P->host.clear(); P->seg.clear(); P->multi.clear();
+  P->row_ptr.assign(K + 1, 0);
+  P->seg_ptr.assign(K + 1, 0);
+  P->multi_ptr.assign(K + 1, 0);
+  P->max_segments = 0;
+  for (int64_t k = 0; k < K; ++k) {
+    P->row_ptr[k] = (int64_t)P->host.size();
+    P->seg_ptr[k] = (int64_t)P->seg.size();
+    P->multi_ptr[k] = (int64_t)P->multi.size();
+    for (const PanelRow& pr : per[k]) {
+      if (pr.len <= kSeg) {
+        P->host.push_back(pr);
+        continue;
+      }
+      int64_t first = (int64_t)P->seg.size() - P->seg_ptr[k];   // slot within the block
+      int32_t nseg = 0;
+      for (int64_t off = 0; off < pr.len; off += kSeg, ++nseg)
+        P->seg.push_back(PanelRow{pr.row, (int32_t)std::min<int64_t>(kSeg, pr.len - off), pr.beg + off});
+      P->multi.push_back(PanelRow{pr.row, nseg, first});
+    }
+    P->max_segments = std::max<int64_t>(P->max_segments, (int64_t)P->seg.size() - P->seg_ptr[k]);
+  }
+  P->row_ptr[K] = (int64_t)P->host.size();
+  P->seg_ptr[K] = (int64_t)P->seg.size();
+  P->multi_ptr[K] = (int64_t)P->multi.size();
+}
+
 // Panel lists.  Over a CSR-like (ptr, idx) with N rows: for each block of the
 // *index* range (block size b over Nidx), the rows with entries in the block.
 void build_stoch_panels(const std::vector<int64_t>& ptr, const std::vector<int32_t>& idx,
@@ -156,41 +187,21 @@ void build_stoch_panels(const std::vector<int64_t>& ptr, const std::vector<int32
       per[blk].push_back(PanelRow{(int32_t)i, (int32_t)(e - s), s});
     }
   }
-  P->host.clear();
-  P->light_ptr.assign(K + 1, 0);
-  P->heavy_ptr.assign(K, 0);
-  for (int64_t k = 0; k < K; ++k) {
-    P->light_ptr[k] = (int64_t)P->host.size();
-    for (auto& pr : per[k]) if (pr.len <= kHeavyRow) P->host.push_back(pr);
-    P->heavy_ptr[k] = (int64_t)P->host.size();
-    for (auto& pr : per[k]) if (pr.len > kHeavyRow) P->host.push_back(pr);
-  }
-  P->light_ptr[K] = (int64_t)P->host.size();
+  finalize_panels(per, P);
 }
 
 // Exact panels: block k of rows [k b, (k+1) b) with their complete rows.
 void build_exact_panels(const std::vector<int64_t>& ptr, int64_t N, int64_t b, PanelSet* P) {
   int64_t K = nblocks(N, b);
-  P->host.clear();
-  P->light_ptr.assign(K + 1, 0);
-  P->heavy_ptr.assign(K, 0);
+  std::vector<std::vector<PanelRow>> per(K);
   for (int64_t k = 0; k < K; ++k) {
     int64_t i0 = k * b, i1 = std::min(N, (k + 1) * b);
-    P->light_ptr[k] = (int64_t)P->host.size();
     for (int64_t i = i0; i < i1; ++i) {
       int64_t len = ptr[i + 1] - ptr[i];
-      if (len > 0 && len <= kHeavyRow) P->host.push_back(PanelRow{(int32_t)i, (int32_t)len, ptr[i]});
-    }
-    P->heavy_ptr[k] = (int64_t)P->host.size();
-    for (int64_t i = i0; i < i1; ++i) {
-      int64_t len = ptr[i + 1] - ptr[i];
-      if (len > kHeavyRow) {
-        // rows longer than 2^31 - 1 entries are split (n < 2^31 bounds len anyway)
-        P->host.push_back(PanelRow{(int32_t)i, (int32_t)len, ptr[i]});
-      }
+      if (len > 0) per[k].push_back(PanelRow{(int32_t)i, (int32_t)len, ptr[i]});
     }
   }
-  P->light_ptr[K] = (int64_t)P->host.size();
+  finalize_panels(per, P);
 }
 
 void build_panels(const HostSparse& S, const nmd_options& o, PanelSet P[2][2]) {
@@ -218,8 +229,8 @@ struct Carver {
   }
 };
 
-void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanels, Workspace* w,
-            Factor* W, Factor* B) {
+void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanels, int64_t maxseg,
+            Workspace* w, Factor* W, Factor* B) {
   w->rowptr = c.take<int64_t>(m + 1);
   w->col = c.take<int32_t>(nnz);
   w->val = c.take<float>(nnz);
@@ -233,6 +244,7 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
     f->master = c.take<float>(N * rp);
     f->hi = c.take<bf16>(N * rp);
     f->lo = c.take<bf16>(N * rp);
+    f->lo2 = c.take<bf16>(N * rp);
     f->E = c.take<float>(N * rp);
   }
   w->R = c.take<float>(std::max(m, n) * rp);
@@ -240,6 +252,7 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->G = c.take<float>((size_t)rp * rp);
   w->Ginv = c.take<float>((size_t)rp * rp);
   w->chol_scratch = c.take<float>((size_t)2 * rp * rp);
+  w->seg_partials = c.take<float>((size_t)std::max<int64_t>(maxseg, 1) * rp);
   w->loss_part = c.take<double>((size_t)kLossParts * 8);
   w->loss_out = c.take<double>(8);
   w->status = c.take<int>(kStatusWords);
@@ -251,7 +264,14 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
 int64_t panel_total(PanelSet P[2][2]) {
   int64_t t = 0;
   for (int s = 0; s < 2; ++s)
-    for (int k = 0; k < 2; ++k) t += (int64_t)P[s][k].host.size();
+    for (int k = 0; k < 2; ++k) t += (int64_t)(P[s][k].host.size() + P[s][k].seg.size() + P[s][k].multi.size());
+  return t;
+}
+
+int64_t max_segments(PanelSet P[2][2]) {
+  int64_t t = 0;
+  for (int s = 0; s < 2; ++s)
+    for (int k = 0; k < 2; ++k) t = std::max(t, P[s][k].max_segments);
   return t;
 }
 
@@ -297,6 +317,7 @@ const char* status_name(int s) {
 // Synchronise, then read and clear the sticky device status.
 nmd_status sync_and_check(nmd_handle* h) {
   CK(h, cudaStreamSynchronize(h->stream));
+  if (h->side) CK(h, cudaStreamSynchronize(h->side));
   int st[kStatusWords];
   CK(h, cudaMemcpy(st, h->ws.status, sizeof st, cudaMemcpyDeviceToHost));
   if (st[0] != 0) {
@@ -325,17 +346,18 @@ cudaEvent_t pool_event(nmd_handle* h) {
 struct TimedScope {
   nmd_handle* h;
   int cls;
+  cudaStream_t st;
   cudaEvent_t a = nullptr, b = nullptr;
-  TimedScope(nmd_handle* h_, int c) : h(h_), cls(c) {
+  TimedScope(nmd_handle* h_, int c, cudaStream_t s_ = nullptr) : h(h_), cls(c), st(s_ ? s_ : h_->stream) {
     if (h->profiling) {
       a = pool_event(h);
       b = pool_event(h);
-      cudaEventRecord(a, h->stream);
+      cudaEventRecord(a, st);
     }
   }
   ~TimedScope() {
     if (a) {
-      cudaEventRecord(b, h->stream);
+      cudaEventRecord(b, st);
       h->timed.push_back({cls, a, b});
     }
   }
@@ -397,14 +419,19 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue};
   cudaStream_t s = h->stream;
   // Gram G = Q^T Q of the Q-side rows, then Cholesky and G^{-1}
+  // Gram G = Q^T Q of the Q-side rows and G^{-1} on the side stream: only the
+  // update needs them, so they overlap the dense contraction
   int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 255) / 256));
+  CK(h, cudaEventRecord(h->ev_fork, s));
+  CK(h, cudaStreamWaitEvent(h->side, h->ev_fork, 0));
   {
-    TimedScope ts(h, NMD_K_GRAM);
-    launch_gram(*ro.fq, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, s);
+    TimedScope ts(h, NMD_K_GRAM, h->side);
+    launch_gram(*ro.fq, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, h->side);
     launch_chol_inv(h->ws.gram_part, nparts, h->r, h->rp, (float)h->opt.ridge, h->ws.G, h->ws.Ginv,
-                    h->ws.chol_scratch, h->ws.status, s);
+                    h->ws.chol_scratch, h->ws.status, h->side);
     h->launches += 2;
   }
+  CK(h, cudaEventRecord(h->ev_join, h->side));
   if ((st = after_launch(h, "gram/cholesky")) != NMD_OK) return st;
   // dense Z-panel contraction R = P(L) Q over every (M-side, Q-side) pair
   {
@@ -420,13 +447,17 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   if ((st = after_launch(h, "dense panel")) != NMD_OK) return st;
   // sparse correction over the block's support
   const PanelSet& P = *ro.P;
-  int64_t lb = P.light_ptr[block], hb = P.heavy_ptr[block], he = P.light_ptr[block + 1];
+  int64_t r0 = P.row_ptr[block], r1 = P.row_ptr[block + 1];
+  int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1];
+  int64_t u0 = P.multi_ptr[block], u1 = P.multi_ptr[block + 1];
   {
     TimedScope ts(h, NMD_K_SPARSE);
-    launch_sparse(a, P.d + lb, hb - lb, P.d + hb, he - hb, ro.qidx, ro.vals, h->ws.R, s);
-    h->launches += (hb > lb) + (he > hb);
+    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, g1 - g0, P.d_multi + u0, u1 - u0, ro.qidx, ro.vals,
+                  h->ws.R, h->ws.seg_partials, s);
+    h->launches += (r1 > r0) + 2 * (g1 > g0);
   }
   if ((st = after_launch(h, "sparse correction")) != NMD_OK) return st;
+  CK(h, cudaStreamWaitEvent(s, h->ev_join, 0));
   if (do_update) {
     bool momentum = kind == NMD_STOCH;
     {
@@ -444,12 +475,16 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
 }  // namespace
 
 nmd_handle::~nmd_handle() {
+  if (side) cudaStreamSynchronize(side);
   if (!timed.empty()) cudaStreamSynchronize(stream);
   for (auto& t : timed) {
     cudaEventDestroy(t.a);
     cudaEventDestroy(t.b);
   }
   for (cudaEvent_t e : event_pool) cudaEventDestroy(e);
+  if (ev_fork) cudaEventDestroy(ev_fork);
+  if (ev_join) cudaEventDestroy(ev_join);
+  if (side) cudaStreamDestroy(side);
 }
 
 // ===========================================================================
@@ -494,7 +529,7 @@ nmd_status nmd_workspace_bytes(int64_t m, int64_t n, int32_t r, const int64_t* r
   Carver c(nullptr);
   Workspace w;
   Factor W, B;
-  layout(c, m, n, (int64_t)S.col.size(), pad_rank(r), panel_total(P), &w, &W, &B);
+  layout(c, m, n, (int64_t)S.col.size(), pad_rank(r), panel_total(P), max_segments(P), &w, &W, &B);
   *bytes = w.bytes;
   return NMD_OK;
 }
@@ -521,7 +556,7 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   h->s_fro = S.s_fro;
   build_panels(S, h->opt, h->panels);
   Carver c(d_workspace);
-  layout(c, m, n, h->nnz, h->rp, panel_total(h->panels), &h->ws, &h->W, &h->B);
+  layout(c, m, n, h->nnz, h->rp, panel_total(h->panels), max_segments(h->panels), &h->ws, &h->W, &h->B);
   auto bail = [&](nmd_status s, const std::string& w) {
     fprintf(stderr, "nmd_create: %s\n", w.c_str());
     delete h;
@@ -547,8 +582,13 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   std::vector<PanelRow> all;
   for (int s2 = 0; s2 < 2; ++s2)
     for (int k = 0; k < 2; ++k) {
-      h->panels[s2][k].d = h->ws.panels + all.size();
-      all.insert(all.end(), h->panels[s2][k].host.begin(), h->panels[s2][k].host.end());
+      PanelSet& P = h->panels[s2][k];
+      P.d = h->ws.panels + all.size();
+      all.insert(all.end(), P.host.begin(), P.host.end());
+      P.d_seg = h->ws.panels + all.size();
+      all.insert(all.end(), P.seg.begin(), P.seg.end());
+      P.d_multi = h->ws.panels + all.size();
+      all.insert(all.end(), P.multi.begin(), P.multi.end());
     }
   cudaStream_t s = h->stream;
   struct Cp { void* d; const void* src; size_t n; } cps[] = {
@@ -568,9 +608,14 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
     e = cudaMemsetAsync(f->master, 0, f->rows * h->rp * 4, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(f->hi, 0, f->rows * h->rp * 2, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(f->lo, 0, f->rows * h->rp * 2, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(f->lo2, 0, f->rows * h->rp * 2, s);
     if (e == cudaSuccess) e = cudaMemsetAsync(f->E, 0, f->rows * h->rp * 4, s);
     if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("memset: ") + cudaGetErrorString(e));
   }
+  e = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
+  if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("side stream: ") + cudaGetErrorString(e));
   e = cudaMemsetAsync(h->ws.status, 0, kStatusWords * sizeof(int), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->ws.counters, 0, 64 * sizeof(int), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
@@ -685,7 +730,9 @@ nmd_status nmd_loss(nmd_handle* h, nmd_loss_out* out) {
   double v[8];
   CK(h, cudaMemcpyAsync(v, h->ws.loss_out, sizeof v, cudaMemcpyDeviceToHost, s));
   if ((st = sync_and_check(h)) != NMD_OK) return st;
-  // v: [relu2, relu, sum_a, sum_b, sum_min, sum_maxcorr]
+  // v: [relu2, relu, sum_a, sum_b, sum_min, sum_max]: the dense sums cover
+  // the entries off the support (SIMT: every entry, with the support part
+  // subtracted again by the support pass)
   double zl2 = v[0] + v[2], err2 = v[0] + v[3];
   out->s_fro = h->s_fro;
   out->obj = sqrt(zl2 > 0 ? zl2 : 0.0) / h->s_fro;
@@ -739,7 +786,14 @@ nmd_status nmd_panel_traversal(const nmd_handle* h, int32_t side, int64_t block,
   if (st != NMD_OK) return st;
   // host mirrors of the index arrays are not kept; rebuild q from the device copy
   const PanelSet& P = *ro.P;
-  std::vector<PanelRow> list(P.host.begin() + P.light_ptr[block], P.host.begin() + P.light_ptr[block + 1]);
+  std::vector<PanelRow> list(P.host.begin() + P.row_ptr[block], P.host.begin() + P.row_ptr[block + 1]);
+  for (int64_t u = P.multi_ptr[block]; u < P.multi_ptr[block + 1]; ++u) {
+    const PanelRow& mr = P.multi[u];
+    const PanelRow& first = P.seg[P.seg_ptr[block] + mr.beg];
+    int64_t len = 0;
+    for (int32_t q = 0; q < mr.len; ++q) len += P.seg[P.seg_ptr[block] + mr.beg + q].len;
+    list.push_back(PanelRow{mr.row, (int32_t)len, first.beg});
+  }
   std::sort(list.begin(), list.end(), [](const PanelRow& a, const PanelRow& b) { return a.row < b.row; });
   int64_t total = 0;
   for (auto& pr : list) total += pr.len;
@@ -788,8 +842,8 @@ nmd_status nmd_set_state(nmd_handle* h, const float* W, const float* H, const fl
   // momentum: pack into the master buffers' E (pack writes master/hi/lo of a
   // Factor, so pack into a temporary view whose master is E)
   Factor tw = h->W, tb = h->B;
-  tw.master = h->W.E; tw.hi = nullptr; tw.lo = nullptr;
-  tb.master = h->B.E; tb.hi = nullptr; tb.lo = nullptr;
+  tw.master = h->W.E; tw.hi = nullptr; tw.lo = nullptr; tw.lo2 = nullptr;
+  tb.master = h->B.E; tb.hi = nullptr; tb.lo = nullptr; tb.lo2 = nullptr;
   CK(h, cudaMemcpyAsync(h->ws.R, EW, (size_t)h->m * h->r * 4, cudaMemcpyHostToDevice, s));
   launch_pack(h->ws.R, false, h->m, h->r, h->rp, tw, s);
   CK(h, cudaMemcpyAsync(h->ws.R, EH, (size_t)h->n * h->r * 4, cudaMemcpyHostToDevice, s));

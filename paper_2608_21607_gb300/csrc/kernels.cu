@@ -26,11 +26,13 @@ inline int grid_for(int64_t work, int threads, int cap = 152 * 16) {
 }
 
 // ---------------------------------------------------------------------------
-// Packing: fp32 (N x r, or r x N) -> N x rp master plus bf16 hi/lo split
-// (hi = bf16_rn(x), lo = bf16_rn(x - hi)); pad columns are zero.
+// Packing: fp32 (N x r, or r x N) -> N x rp master plus its bf16 pieces
+// hi = bf16_rn(x), lo = bf16_rn(x - hi), lo2 = bf16_rn(x - hi - lo) (each
+// difference is exact in fp32); pad columns are zero.
 // ---------------------------------------------------------------------------
 __global__ void pack_kernel(const float* __restrict__ src, int src_is_rxN, int64_t N, int r, int rp,
-                            float* __restrict__ master, bf16* __restrict__ hi, bf16* __restrict__ lo) {
+                            float* __restrict__ master, bf16* __restrict__ hi, bf16* __restrict__ lo,
+                            bf16* __restrict__ lo2) {
   int64_t total = N * rp;
   for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < total;
        idx += (int64_t)gridDim.x * blockDim.x) {
@@ -40,9 +42,12 @@ __global__ void pack_kernel(const float* __restrict__ src, int src_is_rxN, int64
     if (c < r) v = src_is_rxN ? src[(int64_t)c * N + j] : src[j * r + c];
     master[idx] = v;
     if (hi) {
-      bf16 h = __float2bfloat16_rn(v);
+      const bf16 h = __float2bfloat16_rn(v);
+      const float r1 = v - __bfloat162float(h);
+      const bf16 l = __float2bfloat16_rn(r1);
       hi[idx] = h;
-      if (lo) lo[idx] = __float2bfloat16_rn(v - __bfloat162float(h));
+      lo[idx] = l;
+      lo2[idx] = __float2bfloat16_rn(r1 - __bfloat162float(l));
     }
   }
 }
@@ -120,172 +125,157 @@ __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ Q, 
 // relative to the diagonal marks G as not positive definite.
 // One thread block; the r x r matrix lives in shared memory when it fits.
 // ---------------------------------------------------------------------------
-constexpr int kCholThreads = 1024;
-
-__global__ void __launch_bounds__(kCholThreads) ginv_kernel(const float* __restrict__ parts, int nparts,
-                                                            int r, int rp, float ridge,
-                                                            float* __restrict__ Gout,
-                                                            float* __restrict__ Ginv,
-                                                            float* __restrict__ scratch,
-                                                            int* __restrict__ status, int use_smem) {
+// Thread (ty, tx) of a T x T block owns the entries (ty + T a, tx + T b).
+template <int T>
+__global__ void __launch_bounds__(T * T) ginv_kernel(const float* __restrict__ parts, int nparts, int r, int rp,
+                                                     float ridge, float* __restrict__ Gout,
+                                                     float* __restrict__ Ginv, float* __restrict__ scratch,
+                                                     int* __restrict__ status, int use_smem) {
   extern __shared__ float sm[];
   float* A = use_smem ? sm : scratch;             // r x r
   __shared__ float rowk[256];
   __shared__ float diag0[256];
   __shared__ int bad;
+  const int tx = threadIdx.x % T, ty = threadIdx.x / T;
   if (threadIdx.x == 0) bad = 0;
-  for (int e = threadIdx.x; e < r * r; e += blockDim.x) {
-    int i = e / r, j = e % r;
-    int a = max(i, j), b = min(i, j);             // lower triangle holds the partials
-    float s = 0.f;
-    for (int p = 0; p < nparts; ++p) s += parts[(size_t)p * rp * rp + (size_t)a * rp + b];
-    if (i == j) s += ridge;
-    A[e] = s;
-    if (i == j) diag0[i] = s;
-  }
+  for (int i = ty; i < r; i += T)
+    for (int j = tx; j < r; j += T) {
+      const int a = max(i, j), b = min(i, j);     // the partials hold the lower triangle
+      const float* src = parts + (size_t)a * rp + b;
+      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      int p = 0;
+      for (; p + 8 <= nparts; p += 8)
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] += __ldg(src + (size_t)(p + q) * rp * rp);
+      for (; p < nparts; ++p) acc[0] += __ldg(src + (size_t)p * rp * rp);
+      float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+      if (i == j) {
+        sum += ridge;
+        diag0[i] = sum;
+      }
+      A[i * r + j] = sum;
+    }
   __syncthreads();
-  for (int e = threadIdx.x; e < rp * rp; e += blockDim.x) {
-    int i = e / rp, j = e % rp;
-    Gout[e] = (i < r && j < r) ? A[i * r + j] : 0.f;
-  }
+  for (int i = ty; i < rp; i += T)
+    for (int j = tx; j < rp; j += T) Gout[i * rp + j] = (i < r && j < r) ? A[i * r + j] : 0.f;
   const float tol = 4.0f * (float)r * FLT_EPSILON;
   for (int k = 0; k < r; ++k) {
-    float d = A[k * r + k];
+    const float d = A[k * r + k];
     if (!(d > tol * diag0[k]) || !isfinite(d)) {
       if (threadIdx.x == 0) {
         bad = 1;
         set_status(status, NMD_ERR_NOT_SPD, k, 0);
       }
-      break;   // uniform: every thread reads the same d
+      break;   // uniform: every thread read the same d
     }
-    for (int j = threadIdx.x; j < r; j += blockDim.x) rowk[j] = A[k * r + j];
+    for (int j = threadIdx.x; j < r; j += T * T) rowk[j] = A[k * r + j];
     __syncthreads();
-    float inv = 1.0f / d;
-    for (int e = threadIdx.x; e < r * r; e += blockDim.x) {
-      int i = e / r, j = e % r;
-      float v;
-      if (i == k && j == k) v = -inv;
-      else if (i == k) v = rowk[j] * inv;
-      else if (j == k) v = rowk[i] * inv;                 // symmetric: a_ik = a_ki
-      else v = A[e] - rowk[i] * rowk[j] * inv;
-      A[e] = v;
+    const float inv = 1.0f / d;
+    for (int i = ty; i < r; i += T) {
+      const float ri = rowk[i] * inv;
+      for (int j = tx; j < r; j += T) {
+        float v;
+        if (i == k && j == k) v = -inv;
+        else if (i == k) v = rowk[j] * inv;
+        else if (j == k) v = ri;                  // symmetric: a_ik = a_ki
+        else v = A[i * r + j] - ri * rowk[j];
+        A[i * r + j] = v;
+      }
     }
     __syncthreads();
   }
   __syncthreads();
-  for (int e = threadIdx.x; e < rp * rp; e += blockDim.x) {
-    int i = e / rp, j = e % rp;
-    float v = 0.f;
-    if (!bad && i < r && j < r) v = -0.5f * (A[i * r + j] + A[j * r + i]);   // symmetrise
-    Ginv[e] = v;
-  }
+  for (int i = ty; i < rp; i += T)
+    for (int j = tx; j < rp; j += T) {
+      float v = 0.f;
+      if (!bad && i < r && j < r) v = -0.5f * (A[i * r + j] + A[j * r + i]);   // symmetrise
+      Ginv[i * rp + j] = v;
+    }
 }
 
 // ---------------------------------------------------------------------------
 // Sparse correction: for every panel row i and entry (i, k) in the block,
-// L_ik = m_i . q_k (the operands of the dense pass), c = S_ik - min(0, L_ik),
-// R_i += c q_k.  One warp per light row; entries are visited in ascending k.
+// L_ik = m_i . q_k, c = S_ik - min(0, L_ik), R_i += c q_k (fp32 masters).
+// One warp per panel row or per segment of at most kSeg entries; the lanes
+// first fetch the entries' indices and values (one per lane), then four
+// entries at a time are processed with their q rows in flight together.
+// Single rows add into R directly (one writer per row); segments of long
+// rows write a partial sum to their slot and a second pass adds the slots
+// of each row in a fixed order.
 // ---------------------------------------------------------------------------
-template <typename T>
-__device__ __forceinline__ float ld(const T* p);
-template <>
-__device__ __forceinline__ float ld<float>(const float* p) { return __ldg(p); }
-template <>
-__device__ __forceinline__ float ld<bf16>(const bf16* p) { return __bfloat162float(*p); }
-
-template <typename T, int VPL>
-__global__ void __launch_bounds__(256) sparse_light_kernel(const PanelRow* __restrict__ rows, int64_t nrows,
-                                                           const T* __restrict__ Mop, int64_t m0,
-                                                           const T* __restrict__ Qop,
-                                                           const int32_t* __restrict__ qidx,
-                                                           const float* __restrict__ vals,
-                                                           float* __restrict__ R, int rp) {
-  int lane = threadIdx.x & 31;
-  int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-  int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  for (; w < nrows; w += nw) {
-    PanelRow pr = rows[w];
-    int64_t i = pr.row;
-    float mv[VPL], acc[VPL];
-#pragma unroll
-    for (int v = 0; v < VPL; ++v) {
-      int c = lane + 32 * v;
-      mv[v] = c < rp ? ld<T>(Mop + i * rp + c) : 0.f;
-      acc[v] = 0.f;
-    }
-    for (int64_t e = pr.beg; e < pr.beg + pr.len; ++e) {
-      int64_t k = qidx[e];
-      float s = vals[e];
-      float qv[VPL];
-      float part = 0.f;
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        int c = lane + 32 * v;
-        qv[v] = c < rp ? ld<T>(Qop + k * rp + c) : 0.f;
-        part = fmaf(mv[v], qv[v], part);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-      float cval = s - fminf(0.f, part);
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) acc[v] = fmaf(cval, qv[v], acc[v]);
-    }
-    float* Ri = R + (i - m0) * rp;
-#pragma unroll
-    for (int v = 0; v < VPL; ++v) {
-      int c = lane + 32 * v;
-      if (c < rp) Ri[c] += acc[v];
-    }
+template <int VPL>
+__global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __restrict__ rows, int64_t nrows,
+                                                          const float* __restrict__ Mop, int64_t m0,
+                                                          const float* __restrict__ Qop,
+                                                          const int32_t* __restrict__ qidx,
+                                                          const float* __restrict__ vals,
+                                                          float* __restrict__ R, float* __restrict__ partials,
+                                                          int rp) {
+  const int lane = threadIdx.x & 31;
+  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  if (w >= nrows) return;
+  const PanelRow pr = rows[w];
+  const int64_t i = pr.row;
+  int kl = 0;
+  float sl = 0.f;
+  if (lane < pr.len) {
+    kl = qidx[pr.beg + lane];
+    sl = vals[pr.beg + lane];
   }
-}
-
-// Heavy rows: one thread block (16 warps) per row; warp w takes entries
-// beg + w, beg + w + 16, ...; the 16 partial sums are added in warp order.
-template <typename T, int VPL>
-__global__ void __launch_bounds__(512) sparse_heavy_kernel(const PanelRow* __restrict__ rows,
-                                                           const T* __restrict__ Mop, int64_t m0,
-                                                           const T* __restrict__ Qop,
-                                                           const int32_t* __restrict__ qidx,
-                                                           const float* __restrict__ vals,
-                                                           float* __restrict__ R, int rp) {
-  __shared__ float part_sm[16][256];
-  int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  PanelRow pr = rows[blockIdx.x];
-  int64_t i = pr.row;
   float mv[VPL], acc[VPL];
 #pragma unroll
   for (int v = 0; v < VPL; ++v) {
-    int c = lane + 32 * v;
-    mv[v] = c < rp ? ld<T>(Mop + i * rp + c) : 0.f;
+    const int c = lane + 32 * v;
+    mv[v] = c < rp ? __ldg(Mop + i * rp + c) : 0.f;
     acc[v] = 0.f;
   }
-  for (int64_t e = pr.beg + wid; e < pr.beg + pr.len; e += 16) {
-    int64_t k = qidx[e];
-    float s = vals[e];
-    float qv[VPL];
-    float part = 0.f;
+  for (int e = 0; e < pr.len; e += 4) {
+    float qv[4][VPL], part[4];
+    float sv[4];
 #pragma unroll
-    for (int v = 0; v < VPL; ++v) {
-      int c = lane + 32 * v;
-      qv[v] = c < rp ? ld<T>(Qop + k * rp + c) : 0.f;
-      part = fmaf(mv[v], qv[v], part);
+    for (int j = 0; j < 4; ++j) {
+      const int k = __shfl_sync(0xffffffffu, kl, (e + j) & 31);
+      sv[j] = __shfl_sync(0xffffffffu, sl, (e + j) & 31);
+      const bool live = e + j < pr.len;
+      part[j] = 0.f;
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) {
+        const int c = lane + 32 * v;
+        qv[j][v] = (live && c < rp) ? __ldg(Qop + (int64_t)k * rp + c) : 0.f;
+        part[j] = fmaf(mv[v], qv[j][v], part[j]);
+      }
     }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-    float cval = s - fminf(0.f, part);
+    for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-    for (int v = 0; v < VPL; ++v) acc[v] = fmaf(cval, qv[v], acc[v]);
+      for (int j = 0; j < 4; ++j) part[j] += __shfl_xor_sync(0xffffffffu, part[j], o);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float cval = sv[j] - fminf(0.f, part[j]);        // zero for the padding entries (q = 0)
+#pragma unroll
+      for (int v = 0; v < VPL; ++v) acc[v] = fmaf(cval, qv[j][v], acc[v]);
+    }
   }
+  float* dst = partials ? partials + w * rp : R + (i - m0) * rp;
 #pragma unroll
   for (int v = 0; v < VPL; ++v) {
-    int c = lane + 32 * v;
-    if (c < 256) part_sm[wid][c] = acc[v];
+    const int c = lane + 32 * v;
+    if (c < rp) dst[c] = partials ? acc[v] : dst[c] + acc[v];
   }
-  __syncthreads();
-  for (int c = threadIdx.x; c < rp; c += blockDim.x) {
+}
+
+// R_i += sum of the segment slots of row i, in slot order.
+__global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __restrict__ multi, int64_t nmulti,
+                                                            const float* __restrict__ partials,
+                                                            float* __restrict__ R, int64_t m0, int rp) {
+  const int lane = threadIdx.x & 31;
+  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  if (w >= nmulti) return;
+  const PanelRow mr = multi[w];
+  for (int c = lane; c < rp; c += 32) {
     float s = 0.f;
-    for (int w = 0; w < 16; ++w) s += part_sm[w][c];
-    R[(i - m0) * rp + c] += s;
+    for (int q = 0; q < mr.len; ++q) s += partials[(mr.beg + q) * rp + c];
+    R[(mr.row - m0) * rp + c] += s;
   }
 }
 
@@ -294,99 +284,177 @@ __global__ void __launch_bounds__(512) sparse_heavy_kernel(const PanelRow* __res
 //   Z form:     U = eta (X - M)      (eqs. lsqA/lsqB with step size)
 //   Delta form: U = eta X            (eqs. spLsqA/spLsqB)
 // then E = U + gamma E (stochastic steps) and M += E, refreshing the bf16
-// hi/lo copies.  Skipped entirely while a sticky error is set.
+// pieces.  Skipped entirely while a sticky error is set.
+// A thread owns 8 consecutive columns of one row (float4 traffic, coalesced
+// along the row); a block keeps CW columns of G^{-1} in shared memory and
+// stages the R rows of each pass there.
 // ---------------------------------------------------------------------------
 template <int RP>
 __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
-                                                     bf16* __restrict__ Mlo, float* __restrict__ E,
-                                                     int64_t m0, int64_t rows,
+                                                     bf16* __restrict__ Mlo, bf16* __restrict__ Mlo2,
+                                                     float* __restrict__ E, int64_t m0, int64_t rows,
                                                      const float* __restrict__ R,
                                                      const float* __restrict__ Ginv, float eta,
                                                      float gamma, int momentum, int delta_form,
                                                      int* __restrict__ status) {
-  static_assert(RP >= 16 && RP <= 256, "padded rank");
-  constexpr bool kSmemG = RP <= 128;
-  constexpr int ROWS = 256 / RP;                      // rows per pass; one (row, column) per thread
-  __shared__ float Gs[kSmemG ? RP * RP : 1];
-  __shared__ float Rs[ROWS][RP];
+  constexpr int CW = RP <= 128 ? RP : 128;    // output columns handled by this block
+  constexpr int TPR = CW / 8;                 // threads per row
+  constexpr int ROWS = 256 / TPR;             // rows per pass
+  extern __shared__ float sm[];
+  float* Gs = sm;                             // RP x CW
+  float* Rs = sm + RP * CW;                   // ROWS x (RP + 4)
   if (*(volatile int*)status != 0) return;
-  if (kSmemG)
-    for (int e = threadIdx.x; e < RP * RP; e += blockDim.x) Gs[e] = Ginv[e];
-  const int c = threadIdx.x % RP;
-  const int rsub = threadIdx.x / RP;
+  const int cw0 = blockIdx.y * CW;
+  for (int e = threadIdx.x; e < RP * CW; e += blockDim.x) Gs[e] = Ginv[(e / CW) * RP + cw0 + (e % CW)];
+  const int rsub = threadIdx.x / TPR;
+  const int c0 = (threadIdx.x % TPR) * 8;     // within the block's CW columns
   for (int64_t base = (int64_t)blockIdx.x * ROWS; base < rows; base += (int64_t)gridDim.x * ROWS) {
     __syncthreads();
-    for (int e = threadIdx.x; e < ROWS * RP; e += blockDim.x) {
-      int64_t li = base + e / RP;
-      Rs[e / RP][e % RP] = li < rows ? R[li * RP + (e % RP)] : 0.f;
+    for (int e = threadIdx.x; e < ROWS * (RP / 4); e += blockDim.x) {
+      const int rr = e / (RP / 4), k4 = e % (RP / 4);
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (base + rr < rows) v = *(const float4*)(R + (base + rr) * RP + 4 * k4);
+      *(float4*)(Rs + rr * (RP + 4) + 4 * k4) = v;
     }
     __syncthreads();
-    int64_t li = base + rsub;
+    const int64_t li = base + rsub;
     if (li >= rows) continue;
-    float x = 0.f;
-#pragma unroll 8
-    for (int k = 0; k < RP; ++k)
-      x = fmaf(Rs[rsub][k], kSmemG ? Gs[k * RP + c] : __ldg(Ginv + k * RP + c), x);
-    int64_t gi = (m0 + li) * RP + c;
-    float mold = M[gi];
-    float u = delta_form ? eta * x : eta * (x - mold);
-    float e = momentum ? fmaf(gamma, E[gi], u) : u;
-    if (momentum) E[gi] = e;
-    float mnew = mold + e;
-    if (!isfinite(mnew)) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
-    M[gi] = mnew;
-    bf16 h = __float2bfloat16_rn(mnew);
-    Mhi[gi] = h;
-    Mlo[gi] = __float2bfloat16_rn(mnew - __bfloat162float(h));
+    float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    const float* rrow = Rs + rsub * (RP + 4);
+#pragma unroll 4
+    for (int k = 0; k < RP; ++k) {
+      const float rk = rrow[k];
+      const float4 g0 = *(const float4*)(Gs + k * CW + c0);
+      const float4 g1 = *(const float4*)(Gs + k * CW + c0 + 4);
+      x[0] = fmaf(rk, g0.x, x[0]); x[1] = fmaf(rk, g0.y, x[1]);
+      x[2] = fmaf(rk, g0.z, x[2]); x[3] = fmaf(rk, g0.w, x[3]);
+      x[4] = fmaf(rk, g1.x, x[4]); x[5] = fmaf(rk, g1.y, x[5]);
+      x[6] = fmaf(rk, g1.z, x[6]); x[7] = fmaf(rk, g1.w, x[7]);
+    }
+    const int64_t g = (m0 + li) * RP + cw0 + c0;
+    float mo[8], eo[8], mn[8];
+    *(float4*)mo = *(const float4*)(M + g);
+    *(float4*)(mo + 4) = *(const float4*)(M + g + 4);
+    if (momentum) {
+      *(float4*)eo = *(const float4*)(E + g);
+      *(float4*)(eo + 4) = *(const float4*)(E + g + 4);
+    }
+    bool finite = true;
+    uint32_t hw[4], lw[4], l2w[4];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float u = delta_form ? eta * x[j] : eta * (x[j] - mo[j]);
+      const float e = momentum ? fmaf(gamma, eo[j], u) : u;
+      eo[j] = e;
+      mn[j] = mo[j] + e;
+      finite = finite && isfinite(mn[j]);
+    }
+#pragma unroll
+    for (int j = 0; j < 8; j += 2) {
+      const bf16 h0 = __float2bfloat16_rn(mn[j]), h1 = __float2bfloat16_rn(mn[j + 1]);
+      const float r0 = mn[j] - __bfloat162float(h0), r1 = mn[j + 1] - __bfloat162float(h1);
+      const bf16 l0 = __float2bfloat16_rn(r0), l1 = __float2bfloat16_rn(r1);
+      const bf16 q0 = __float2bfloat16_rn(r0 - __bfloat162float(l0));
+      const bf16 q1 = __float2bfloat16_rn(r1 - __bfloat162float(l1));
+      hw[j / 2] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+      lw[j / 2] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+      l2w[j / 2] = (uint32_t)__bfloat16_as_ushort(q0) | ((uint32_t)__bfloat16_as_ushort(q1) << 16);
+    }
+    if (!finite) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
+    *(float4*)(M + g) = *(float4*)mn;
+    *(float4*)(M + g + 4) = *(float4*)(mn + 4);
+    if (momentum) {
+      *(float4*)(E + g) = *(float4*)eo;
+      *(float4*)(E + g + 4) = *(float4*)(eo + 4);
+    }
+    *(uint4*)(Mhi + g) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    *(uint4*)(Mlo + g) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+    *(uint4*)(Mlo2 + g) = make_uint4(l2w[0], l2w[1], l2w[2], l2w[3]);
   }
 }
+
+template <typename T>
+__device__ __forceinline__ float ld(const T* p);
+template <>
+__device__ __forceinline__ float ld<float>(const float* p) { return __ldg(p); }
+template <>
+__device__ __forceinline__ float ld<bf16>(const bf16* p) { return __bfloat162float(*p); }
 
 // ---------------------------------------------------------------------------
 // Loss, support part: for every stored (i, j), with L = w_i . b_j and
 // Shat = max(0, L):
-//   a = (S - L)^2 - Shat^2          (objective correction, eq. SLloss)
-//   b = (S - Shat)^2 - Shat^2       (RMSE correction)
-//   mn = min(S, Shat), mx = max(S, Shat) - Shat   (WJD sums)
-// One warp per row of S (fixed assignment), fp64 sums, per-block partials.
+//   a = (S - L)^2,  b = (S - Shat)^2,  mn = min(S, Shat),  mx = max(S, Shat)
+// (eqs. SLloss, RMSE, WJD on the support).  When the dense pass summed every
+// entry (SUBTRACT: the CUDA-core loss pass), Shat^2 and Shat are subtracted
+// again here, with L formed by the same sequential fma chain as that pass so
+// the two cancel exactly.  The tensor-core loss pass skips support entries,
+// and nothing is subtracted.  One warp per row of S, fp64 sums.
 // ---------------------------------------------------------------------------
-template <typename T, int VPL>
+template <int VPL, bool SUBTRACT>
 __global__ void __launch_bounds__(256) loss_sparse_kernel(const int64_t* __restrict__ rowptr,
                                                           const int32_t* __restrict__ col,
                                                           const float* __restrict__ val, int64_t m,
-                                                          const T* __restrict__ Wop,
-                                                          const T* __restrict__ Bop, int rp,
+                                                          const float* __restrict__ Wop,
+                                                          const float* __restrict__ Bop, int rp,
                                                           double* __restrict__ parts) {
   __shared__ double red[8][4];
-  int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   double sa = 0, sb = 0, smn = 0, smx = 0;
-  int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
   for (int64_t i = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5; i < m; i += nw) {
     float wv[VPL];
 #pragma unroll
     for (int v = 0; v < VPL; ++v) {
-      int c = lane + 32 * v;
-      wv[v] = c < rp ? ld<T>(Wop + i * rp + c) : 0.f;
+      const int c = lane + 32 * v;
+      wv[v] = c < rp ? __ldg(Wop + i * rp + c) : 0.f;
     }
-    for (int64_t e = rowptr[i]; e < rowptr[i + 1]; ++e) {
-      int64_t j = col[e];
-      float part = 0.f;
+    for (int64_t e0 = rowptr[i]; e0 < rowptr[i + 1]; e0 += 32) {
+      // lane l takes entry e0 + l
+      const int64_t e = e0 + lane;
+      const bool live = e < rowptr[i + 1];
+      if (SUBTRACT) {
+        if (live) {
+          const int64_t j = col[e];
+          float L = 0.f;
+          for (int c = 0; c < rp; ++c) L = fmaf(__ldg(Wop + i * rp + c), __ldg(Bop + j * rp + c), L);
+          const double Ld = L, S = val[e];
+          const double sh = Ld > 0 ? Ld : 0.0;
+          sa += (S - Ld) * (S - Ld) - sh * sh;
+          sb += (S - sh) * (S - sh) - sh * sh;
+          smn += S < sh ? S : sh;
+          smx += (S > sh ? S : sh) - sh;
+        }
+      } else {
+        const int64_t rem = rowptr[i + 1] - e0;
+        const int cnt = rem < 32 ? (int)rem : 32;
+        for (int q = 0; q < cnt; ++q) {
+          const int64_t j = col[e0 + q];
+          float part = 0.f;
 #pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        int c = lane + 32 * v;
-        float b = c < rp ? ld<T>(Bop + j * rp + c) : 0.f;
-        part = fmaf(wv[v], b, part);
-      }
+          for (int v = 0; v < VPL; ++v) {
+            const int c = lane + 32 * v;
+            part = fmaf(wv[v], c < rp ? __ldg(Bop + j * rp + c) : 0.f, part);
+          }
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
-      if (lane == 0) {
-        double L = part, S = val[e];
-        double sh = L > 0 ? L : 0.0;
-        sa += (S - L) * (S - L) - sh * sh;
-        sb += (S - sh) * (S - sh) - sh * sh;
-        smn += S < sh ? S : sh;
-        smx += (S > sh ? S : sh) - sh;
+          for (int o = 16; o > 0; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+          if (lane == q) {
+            const double Ld = part, S = val[e0 + q];
+            const double sh = Ld > 0 ? Ld : 0.0;
+            sa += (S - Ld) * (S - Ld);
+            sb += (S - sh) * (S - sh);
+            smn += S < sh ? S : sh;
+            smx += S > sh ? S : sh;
+          }
+        }
       }
     }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sa += __shfl_xor_sync(0xffffffffu, sa, o);
+    sb += __shfl_xor_sync(0xffffffffu, sb, o);
+    smn += __shfl_xor_sync(0xffffffffu, smn, o);
+    smx += __shfl_xor_sync(0xffffffffu, smx, o);
   }
   if (lane == 0) {
     red[wid][0] = sa; red[wid][1] = sb; red[wid][2] = smn; red[wid][3] = smx;
@@ -427,7 +495,7 @@ __global__ void loss_final_kernel(const double* __restrict__ dparts, int nd,
 // launchers
 // ===========================================================================
 void launch_pack(const float* src, bool src_is_rxN, int64_t N, int r, int rp, Factor& f, cudaStream_t s) {
-  pack_kernel<<<grid_for(N * rp, 256), 256, 0, s>>>(src, src_is_rxN, N, r, rp, f.master, f.hi, f.lo);
+  pack_kernel<<<grid_for(N * rp, 256), 256, 0, s>>>(src, src_is_rxN, N, r, rp, f.master, f.hi, f.lo, f.lo2);
 }
 
 void launch_unpack(const float* master, bool dst_is_rxN, int64_t N, int r, int rp, float* dst, cudaStream_t s) {
@@ -446,27 +514,41 @@ void launch_gram(const Factor& fq, int64_t q0, int64_t K, int r, int rp, float* 
 
 void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge, float* G, float* Ginv,
                      float* scratch, int* status, cudaStream_t s) {
-  size_t smem = (size_t)r * r * sizeof(float);
-  int use_smem = smem <= 200 * 1024;
-  if (use_smem && smem > 48 * 1024)
-    cudaFuncSetAttribute(ginv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  ginv_kernel<<<1, kCholThreads, use_smem ? smem : 0, s>>>(parts, nparts, r, rp, ridge, G, Ginv, scratch,
-                                                           status, use_smem);
+  const size_t smem = (size_t)r * r * sizeof(float);
+  const int use_smem = smem <= 200 * 1024;
+  if (r <= 64) {
+    ginv_kernel<16><<<1, 256, smem, s>>>(parts, nparts, r, rp, ridge, G, Ginv, scratch, status, 1);
+  } else {
+    static bool attr = false;
+    if (!attr) {
+      cudaFuncSetAttribute(ginv_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+      attr = true;
+    }
+    ginv_kernel<32><<<1, 1024, use_smem ? smem : 0, s>>>(parts, nparts, r, rp, ridge, G, Ginv, scratch, status,
+                                                         use_smem);
+  }
 }
 
-template <typename T>
-static void sparse_dispatch(const StepArgs& a, const T* Mop, const T* Qop, const PanelRow* light,
-                            int64_t nlight, const PanelRow* heavy, int64_t nheavy, const int32_t* qidx,
-                            const float* vals, float* R, cudaStream_t s) {
-  // panel rows and qidx hold absolute M-side / Q-side row indices
-  int g = grid_for(nlight * 32, 256, 152 * 64);
-#define NMD_SP(V)                                                                                     \
-  do {                                                                                                \
-    if (nlight > 0)                                                                                   \
-      sparse_light_kernel<T, V><<<g, 256, 0, s>>>(light, nlight, Mop, a.m0, Qop, qidx, vals, R, a.rp); \
-    if (nheavy > 0)                                                                                   \
-      sparse_heavy_kernel<T, V><<<(unsigned)nheavy, 512, 0, s>>>(heavy, Mop, a.m0, Qop, qidx, vals, R, \
-                                                                  a.rp);                              \
+void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* seg, int64_t nseg,
+                   const PanelRow* multi, int64_t nmulti, const int32_t* qidx, const float* vals, float* R,
+                   float* partials, cudaStream_t s) {
+  // The support correction always reads the fp32 masters, in every precision:
+  // on rows with few support entries the term S_ik q_k dominates R_i and is
+  // not averaged over many products, so rounding q_k to bf16 there would put
+  // its full relative error (up to 2^-9) into the update.
+  const float* Mop = a.fm->master;
+  const float* Qop = a.fq->master;
+#define NMD_SP(V)                                                                                           \
+  do {                                                                                                      \
+    if (nrows > 0)                                                                                          \
+      sparse_rows_kernel<V><<<(unsigned)((nrows + 7) / 8), 256, 0, s>>>(rows, nrows, Mop, a.m0, Qop, qidx,  \
+                                                                        vals, R, nullptr, a.rp);            \
+    if (nseg > 0) {                                                                                         \
+      sparse_rows_kernel<V><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(seg, nseg, Mop, a.m0, Qop, qidx,     \
+                                                                       vals, R, partials, a.rp);            \
+      sparse_reduce_kernel<<<(unsigned)((nmulti + 7) / 8), 256, 0, s>>>(multi, nmulti, partials, R, a.m0,   \
+                                                                        a.rp);                              \
+    }                                                                                                       \
   } while (0)
   switch (a.rp) {
     case 16: case 32: NMD_SP(1); break;
@@ -477,49 +559,54 @@ static void sparse_dispatch(const StepArgs& a, const T* Mop, const T* Qop, const
 #undef NMD_SP
 }
 
-// The support correction always reads the fp32 masters, in every precision:
-// on rows with few support entries the term S_ik q_k dominates R_i and is not
-// averaged over many products, so rounding q_k to bf16 there would put its
-// full relative error (up to 2^-9) into the update.
-void launch_sparse(const StepArgs& a, const PanelRow* light, int64_t nlight, const PanelRow* heavy,
-                   int64_t nheavy, const int32_t* qidx, const float* vals, float* R, cudaStream_t s) {
-  sparse_dispatch<float>(a, a.fm->master, a.fq->master, light, nlight, heavy, nheavy, qidx, vals, R, s);
+template <int RP>
+static void update_rp(const StepArgs& a, const float* R, const float* Ginv, float eta, float gamma, bool momentum,
+                      int* status, cudaStream_t s) {
+  constexpr int CW = RP <= 128 ? RP : 128;
+  constexpr int ROWS = 256 / (CW / 8);
+  const size_t smem = ((size_t)RP * CW + ROWS * (RP + 4)) * sizeof(float);
+  static bool attr = false;
+  if (!attr) {
+    cudaFuncSetAttribute(update_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    attr = true;
+  }
+  const int per_sm = RP <= 32 ? 8 : (RP == 64 ? 4 : (RP == 128 ? 2 : 1));
+  const int64_t tiles = (a.M + ROWS - 1) / ROWS;
+  dim3 grid((unsigned)std::min<int64_t>(tiles, 152 * per_sm), RP / CW);
+  const Factor& f = *a.fm;
+  update_kernel<RP><<<grid, 256, smem, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Ginv, eta, gamma, momentum,
+                                            a.epilogue == NMD_EPI_DELTA, status);
 }
 
-void launch_update(const StepArgs& a, const float* R, const float* Ginv, float eta, float gamma,
-                   bool momentum, int* status, cudaStream_t s) {
-  const Factor& f = *a.fm;
-  int rows_per_pass = 256 / std::min(a.rp, 256);
-  int g = grid_for(a.M, rows_per_pass, 152 * 8);
-#define NMD_UP(RP)                                                                                   \
-  update_kernel<RP><<<g, 256, 0, s>>>(f.master, f.hi, f.lo, f.E, a.m0, a.M, R, Ginv, eta, gamma,      \
-                                      momentum, a.epilogue == NMD_EPI_DELTA, status)
+void launch_update(const StepArgs& a, const float* R, const float* Ginv, float eta, float gamma, bool momentum,
+                   int* status, cudaStream_t s) {
   switch (a.rp) {
-    case 16: NMD_UP(16); break;
-    case 32: NMD_UP(32); break;
-    case 64: NMD_UP(64); break;
-    case 128: NMD_UP(128); break;
-    default: NMD_UP(256); break;
+    case 16: update_rp<16>(a, R, Ginv, eta, gamma, momentum, status, s); break;
+    case 32: update_rp<32>(a, R, Ginv, eta, gamma, momentum, status, s); break;
+    case 64: update_rp<64>(a, R, Ginv, eta, gamma, momentum, status, s); break;
+    case 128: update_rp<128>(a, R, Ginv, eta, gamma, momentum, status, s); break;
+    default: update_rp<256>(a, R, Ginv, eta, gamma, momentum, status, s); break;
   }
-#undef NMD_UP
 }
 
 void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s) {
-  bool bf = h->opt.precision == NMD_BF16;
-#define NMD_LS(T, V, WP, BP) \
-  loss_sparse_kernel<T, V><<<nparts, 256, 0, s>>>(h->ws.rowptr, h->ws.col, h->ws.val, h->m, WP, BP, h->rp, parts)
-#define NMD_LSV(V)                                                   \
-  do {                                                               \
-    if (bf) NMD_LS(bf16, V, h->W.hi, h->B.hi);                       \
-    else NMD_LS(float, V, h->W.master, h->B.master);                 \
+  // fp32 masters in every precision, like the support correction of the update
+  const bool subtract = h->opt.precision == NMD_SIMT;
+#define NMD_LS(V)                                                                                          \
+  do {                                                                                                     \
+    if (subtract)                                                                                          \
+      loss_sparse_kernel<V, true><<<nparts, 256, 0, s>>>(h->ws.rowptr, h->ws.col, h->ws.val, h->m,           \
+                                                        h->W.master, h->B.master, h->rp, parts);           \
+    else                                                                                                   \
+      loss_sparse_kernel<V, false><<<nparts, 256, 0, s>>>(h->ws.rowptr, h->ws.col, h->ws.val, h->m,          \
+                                                         h->W.master, h->B.master, h->rp, parts);          \
   } while (0)
   switch (h->rp) {
-    case 16: case 32: NMD_LSV(1); break;
-    case 64: NMD_LSV(2); break;
-    case 128: NMD_LSV(4); break;
-    default: NMD_LSV(8); break;
+    case 16: case 32: NMD_LS(1); break;
+    case 64: NMD_LS(2); break;
+    case 128: NMD_LS(4); break;
+    default: NMD_LS(8); break;
   }
-#undef NMD_LSV
 #undef NMD_LS
 }
 

@@ -23,17 +23,23 @@ struct PanelRow {
   int64_t beg;
 };
 
-// Panel rows longer than this are handled by a whole thread block each.
-constexpr int kHeavyRow = 256;
+// Panel rows with more entries than this are split into segments of at most
+// kSeg entries; each segment's partial sum goes to a scratch slot and the
+// slots of a row are added in a fixed order by a second pass.
+constexpr int kSeg = 32;
 
-// Per (side, kind): the panel lists of every block, concatenated.  Block k's
-// light rows are [light_ptr[k], light_ptr[k+1]) and its heavy rows
-// [heavy_ptr[k], heavy_ptr[k+1]) of the device array `d` (light rows first,
-// then heavy rows, block by block).
+// Per (side, kind): the panel lists of every block, concatenated.  For block k:
+//   single rows   [row_ptr[k], row_ptr[k+1])   of `host`/`d`   (len <= kSeg)
+//   segments      [seg_ptr[k], seg_ptr[k+1])   of `seg`        (one kSeg slice each)
+//   split rows    [multi_ptr[k], multi_ptr[k+1]) of `multi`    (row, #segments, first segment)
+// Rows are listed in ascending order.
 struct PanelSet {
-  std::vector<int64_t> light_ptr, heavy_ptr;
-  std::vector<PanelRow> host;
+  std::vector<int64_t> row_ptr, seg_ptr, multi_ptr;
+  std::vector<PanelRow> host, seg, multi;
   PanelRow* d = nullptr;
+  PanelRow* d_seg = nullptr;
+  PanelRow* d_multi = nullptr;
+  int64_t max_segments = 0;     // largest segment count of any block
 };
 
 // Device status word (sticky): [0] = nmd_status code of the first error,
@@ -46,6 +52,7 @@ struct Factor {
   float* master = nullptr;   // N x rp fp32, pad columns are zero
   bf16* hi = nullptr;        // N x rp, bf16(master)
   bf16* lo = nullptr;        // N x rp, bf16(master - hi)
+  bf16* lo2 = nullptr;       // N x rp, bf16(master - hi - lo)
   float* E = nullptr;        // N x rp momentum (fp32)
 };
 
@@ -79,6 +86,7 @@ struct Workspace {
   int* status = nullptr;       // kStatusWords
   int* counters = nullptr;     // 64 ints (tile schedulers)
   float* chol_scratch = nullptr;  // 2 x rp x rp (used when rp is too large for smem)
+  float* seg_partials = nullptr;  // max segments x rp (sparse correction of long rows)
 };
 
 constexpr int kGramParts = 64;
@@ -91,6 +99,10 @@ struct nmd_handle {
   int r = 0, rp = 0;
   nmd_options opt;
   cudaStream_t stream = nullptr;
+  // the Gram chain runs on a second stream, forked from and joined back into
+  // `stream` around the dense kernel of each step
+  cudaStream_t side = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
   nmd::Workspace ws;
   nmd::Factor W, B;            // A = W (m x r), B = H^T (n x r)
   nmd::PanelSet panels[2][2];  // [side][kind]
@@ -105,7 +117,7 @@ struct nmd_handle {
   // kernel timing (nmd_profile): event pairs per launch, by kernel class
   bool profiling = false;
   std::vector<cudaEvent_t> event_pool;
-  struct Timed { int cls; cudaEvent_t a, b; };
+  struct Timed { int cls; cudaEvent_t a, b; };  // a, b recorded on the stream the class runs on
   std::vector<Timed> timed;
   double prof_ms[5] = {0, 0, 0, 0, 0};
   int64_t prof_launches[5] = {0, 0, 0, 0, 0};
@@ -123,9 +135,9 @@ void launch_gram(const Factor& fq, int64_t q0, int64_t K, int r, int rp, float* 
                  int nparts, cudaStream_t s);
 void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge, float* G,
                      float* Ginv, float* scratch, int* status, cudaStream_t s);
-void launch_sparse(const StepArgs& a, const PanelRow* light, int64_t nlight,
-                   const PanelRow* heavy, int64_t nheavy, const int32_t* qidx,
-                   const float* vals, float* R, cudaStream_t s);
+void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* seg,
+                   int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
+                   const float* vals, float* R, float* partials, cudaStream_t s);
 void launch_update(const StepArgs& a, const float* R, const float* Ginv, float eta,
                    float gamma, bool momentum, int* status, cudaStream_t s);
 void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s);

@@ -8,16 +8,23 @@
 //        = -max(0, L_ik)     (Delta form, eq. updateD)  written back to TMEM
 //   R_i  = sum_k P_ik q_k                    MMA2: TMEM R += P (TMEM) x chunk
 // The same shared-memory copy of each chunk feeds both products: K-major for
-// MMA1 and MN-major for MMA2.  With SPLIT (fp32-accurate mode) every operand
-// is x = hi + lo (bf16 each) and each product is hi*hi + hi*lo + lo*hi.
+// MMA1 and MN-major for MMA2.  Every factor has bf16 pieces hi = bf16(x),
+// lo = bf16(x - hi), lo2 = bf16(x - hi - lo).  bf16 mode: MMA1 uses hi only,
+// MMA2 uses q = hi + lo -- every row of R shares the same q_k, so a rounding
+// of q would be a coherent error that the Gram solve amplifies by its
+// condition number.  fp32-accurate mode (SPLIT): MMA1 = w_hi q_hi + w_hi q_lo
+// + w_lo q_hi, P = P_hi + P_lo, MMA2 = P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi.
 //
 // The loss kernel runs MMA1 only, over all of W against all of B, and sums
-// max(0, L)^2 and max(0, L) (eq. SLloss / eq. RMSE / eq. WJD dense parts).
+// max(0, L)^2 and max(0, L) over the entries outside the support of S (the
+// dense parts of eq. SLloss / eq. RMSE / eq. WJD); the support entries are
+// summed by a separate pass.
 //
-// Warp roles (192 threads, one CTA per SM, persistent over M tiles):
-//   warps 0-3  epilogue: thread t owns TMEM lane t = tile row t
-//   warp 4     TMA producer of Q chunks (+ TMEM allocation)
-//   warp 5     MMA issuer (one thread)
+// Warp roles (320 threads, one CTA per SM, persistent over M tiles):
+//   warps 0-7  epilogue, two warpgroups taking alternate chunks; in each,
+//              thread t owns TMEM lane t = tile row t
+//   warp 8     TMA producer of Q chunks (+ TMEM allocation)
+//   warp 9     MMA issuer (one thread)
 // Every mbarrier wait is bounded (2 s): on expiry the kernel records
 // NMD_ERR_TIMEOUT, the other roles stop at their next wait, in-flight MMAs
 // and copies are drained and TMEM is freed before the kernel returns.
@@ -35,37 +42,51 @@ namespace {
 
 using namespace tc;
 
-constexpr int kThreads = 192;
+constexpr int kEpiThreads = 256;                 // two epilogue warpgroups
+constexpr int kProducerWarp = 8, kMmaWarp = 9;
+constexpr int kThreads = 320;
 constexpr int BM = 128;
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 
-template <int RP, bool SPLIT>
+template <int RP, bool SPLIT, bool LOSS>
 struct Cfg {
-  static constexpr int BN = (RP == 256 || (SPLIT && RP == 128)) ? 64 : 128;  // Q rows per chunk
+  // bf16 mode with r_pad <= 128: MMA2 multiplies P by [q_hi | q_lo] as one
+  // product of width 2 r_pad (two accumulators side by side, summed at
+  // readout): half the MMA instructions of two separate products
+  static constexpr bool FUSEDN = !SPLIT && !LOSS && RP <= 128;
+  static constexpr int RCOLS = FUSEDN ? 2 * RP : RP;   // TMEM columns of the R accumulator(s)
+  static constexpr int BN = (RP == 256 || (SPLIT && RP == 128) || (FUSEDN && RP == 128)) ? 64 : 128;  // Q rows per chunk
   static constexpr int WCOLS = SPLIT ? RP : RP / 2;    // TMEM columns of one W tile (hi [+ lo])
   static constexpr int NWB = (RP == 256) ? 1 : 2;      // W tile buffers
-  static constexpr int FREE = 512 - NWB * WCOLS - RP;
+  static constexpr int FREE = 512 - NWB * WCOLS - RCOLS;
   static constexpr int NB = FREE / BN >= 3 ? 3 : FREE / BN;  // L buffers
+  static constexpr int LAG = NB >= 3 ? 2 : 1;                 // MMA1 runs LAG chunks ahead of MMA2
   static constexpr int PANEL_W = RP < 64 ? RP : 64;    // elements per row of one swizzle panel
   static constexpr int ROWB = PANEL_W * 2;             // bytes per panel row (= swizzle width)
   static constexpr int PANEL_BYTES = BN * ROWB;
   static constexpr int NPANEL = RP / PANEL_W;
-  static constexpr int OPER_BYTES = BN * RP * 2;       // one operand (hi or lo) of a chunk
-  static constexpr int STAGE_BYTES = OPER_BYTES * (SPLIT ? 2 : 1);
+  static constexpr int OPER_BYTES = BN * RP * 2;       // one bf16 piece of a chunk
+  // bf16 pieces of each chunk in shared memory: the second product always
+  // uses q = hi + lo (three pieces in the fp32-accurate mode); the loss pass
+  // (first product only) needs hi (+ lo when split)
+  static constexpr int NQ = LOSS ? (SPLIT ? 2 : 1) : (SPLIT ? 3 : 2);
+  static constexpr int STAGE_BYTES = OPER_BYTES * NQ;
   static constexpr int NSTAGE_RAW = (160 * 1024) / STAGE_BYTES;
-  static constexpr int NSTAGE = NSTAGE_RAW > 8 ? 8 : (NSTAGE_RAW < 2 ? 2 : NSTAGE_RAW);
+  static constexpr int NSTAGE = NSTAGE_RAW > 8 ? 8 : (NSTAGE_RAW < 3 ? 3 : NSTAGE_RAW);
   static constexpr uint32_t SWZ = PANEL_W == 64 ? SWZ_128B : (PANEL_W == 32 ? SWZ_64B : SWZ_32B);
   static constexpr int COL_L = 0;               // NB x BN columns
   static constexpr int COL_R = NB * BN;         // RP columns
-  static constexpr int COL_W = COL_R + RP;      // NWB x WCOLS columns
+  static constexpr int COL_W = COL_R + RCOLS;   // NWB x WCOLS columns
   // barriers: full[NSTAGE], empty[NSTAGE], lfull[NB], pfull[NB], lfree[NB], rfull, rempty,
   // wfull[2], wempty[2], drain
   static constexpr int NBAR = 2 * NSTAGE + 3 * NB + 7;
-  static constexpr size_t SMEM_USED = 1024 + (size_t)NSTAGE * STAGE_BYTES + NBAR * 8 + 64 + 128 * 16;
+  static constexpr size_t SMEM_USED = 1024 + (size_t)NSTAGE * STAGE_BYTES + NBAR * 8 + 64 + 256 * 16;
   // at least 120 KB so that a second CTA (and its 512-column TMEM request)
   // never shares the SM
   static constexpr size_t SMEM = SMEM_USED > 120 * 1024 ? SMEM_USED : 120 * 1024;
   static_assert(NB >= 2, "need two L buffers");
+  static_assert(NSTAGE > LAG, "a stage must be free before MMA1 runs LAG chunks ahead");
+  static_assert(SMEM <= 227 * 1024, "shared memory per block");
   static_assert(COL_W + NWB * WCOLS <= 512, "TMEM budget");
   static_assert(BN % 32 == 0 && RP % 16 == 0, "shapes");
 };
@@ -79,6 +100,8 @@ struct TcParams {
   double* parts;        // per-CTA loss partials (loss kernel)
   int* status;
   float* Lout;          // verification: raw L (M x K, row-major) or nullptr
+  const int64_t* rowptr;   // loss kernel: CSR of S, whose entries the dense pass skips
+  const int32_t* cidx;
 };
 
 __device__ __forceinline__ void record(int* status, int code, int detail) {
@@ -86,21 +109,25 @@ __device__ __forceinline__ void record(int* status, int code, int detail) {
 }
 
 // Bounded wait on an mbarrier phase.  Returns false if the kernel is aborting.
-__device__ __noinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
-                                      int where) {
-  if (mbar_try_wait(bar, parity)) return true;
-  uint64_t t0 = globaltimer_ns();
-  for (uint32_t it = 1;; ++it) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((it & 255u) == 0) {
-      if (*abort_flag) return false;
-      if (globaltimer_ns() - t0 > kTimeoutNs) {
-        *abort_flag = 1;
-        record(status, NMD_ERR_TIMEOUT, where);
-        return false;
-      }
+// The polls suspend in hardware until the phase completes (or 20 us pass), so
+// waiting warps do not take issue slots from the MMA and copy threads.
+__device__ __noinline__ bool wait_bar_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
+                                           int where) {
+  const uint64_t t0 = globaltimer_ns();
+  for (;;) {
+    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (*abort_flag) return false;
+    if (globaltimer_ns() - t0 > kTimeoutNs) {
+      *abort_flag = 1;
+      record(status, NMD_ERR_TIMEOUT, where);
+      return false;
     }
   }
+}
+__device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
+                                         int where) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return wait_bar_slow(bar, parity, abort_flag, status, where);
 }
 
 // Warp-uniform wait: lane 0 polls, the outcome is broadcast to the warp.
@@ -116,8 +143,8 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 template <int RP, int EPI, bool SPLIT, bool LOSS>
 __global__ void __launch_bounds__(kThreads, 1)
     panel_tc_kernel(const __grid_constant__ CUtensorMap tq_hi, const __grid_constant__ CUtensorMap tq_lo,
-                    const TcParams p) {
-  using C = Cfg<RP, SPLIT>;
+                    const __grid_constant__ CUtensorMap tq_lo2, const TcParams p) {
+  using C = Cfg<RP, SPLIT, LOSS>;
   constexpr int BN = C::BN, NB = C::NB, NSTAGE = C::NSTAGE, NWB = C::NWB;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -146,25 +173,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int i = 0; i < NB; ++i) {
       mbar_init(b_lfull + 8 * i, 1);
-      mbar_init(b_pfull + 8 * i, 128);
-      mbar_init(b_lfree + 8 * i, LOSS ? 128 : 1);
+      mbar_init(b_pfull + 8 * i, 4);                 // the four warps of one epilogue warpgroup
+      mbar_init(b_lfree + 8 * i, LOSS ? 4 : 1);
     }
     mbar_init(b_rfull, 1);
-    mbar_init(b_rempty, 128);
+    mbar_init(b_rempty, kEpiThreads / 32);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(b_wfull + 8 * i, 128);
+      mbar_init(b_wfull + 8 * i, kEpiThreads / 32);
       mbar_init(b_wempty + 8 * i, 1);
     }
     mbar_init(b_drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 4) {
+  if (warp == kProducerWarp) {
     tmem_alloc(smem_u32(tmem_slot), 512);
     tmem_relinquish();
     if (lane == 0) {
       prefetch_tmap(&tq_hi);
-      if (SPLIT) prefetch_tmap(&tq_lo);
+      if (C::NQ > 1) prefetch_tmap(&tq_lo);
+      if (C::NQ > 2) prefetch_tmap(&tq_lo2);
     }
   }
   fence_before();
@@ -175,7 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t ntiles = (p.M + BM - 1) / BM;
   const int64_t nchunks = (p.K + BN - 1) / BN;
 
-  if (warp == 4) {
+  if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       int64_t G = 0;
@@ -191,12 +219,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
           for (int pn = 0; pn < C::NPANEL; ++pn) {
             tma_load_2d(dst + pn * C::PANEL_BYTES, &tq_hi, b_full + 8 * s, pn * C::PANEL_W, y);
-            if (SPLIT)
+            if (C::NQ > 1)
               tma_load_2d(dst + C::OPER_BYTES + pn * C::PANEL_BYTES, &tq_lo, b_full + 8 * s, pn * C::PANEL_W, y);
+            if (C::NQ > 2)
+              tma_load_2d(dst + 2 * C::OPER_BYTES + pn * C::PANEL_BYTES, &tq_lo2, b_full + 8 * s, pn * C::PANEL_W,
+                          y);
           }
         }
       }
-      if (!ok) {  // drain the copies still in flight before TMEM/smem go away
+      if (!ok) {  // drain the copies still in flight before shared memory goes away
         for (int64_t k = G - NSTAGE > 0 ? G - NSTAGE : 0; k < G; ++k) {
           uint64_t t0 = globaltimer_ns();
           while (!mbar_try_wait(b_full + 8 * (int)(k % NSTAGE), (uint32_t)((k / NSTAGE) & 1)) &&
@@ -205,72 +236,106 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == 5) {
+  } else if (warp == kMmaWarp) {
     // ------------------------------------------------------------ MMA issuer
+    // One global chunk sequence G over this CTA's tiles.  Step G issues MMA1
+    // of chunk G and MMA2 of chunk G - LAG, so the epilogue of a chunk has
+    // LAG chunks of tensor work to hide behind, including across tiles.  All
+    // ring positions and phases are kept as running counters.
     if (lane == 0) {
+      constexpr int LAG = C::LAG;
       constexpr uint32_t idesc1 = idesc_bf16(BM, BN, false);   // L = W x Q^T (Q K-major)
-      constexpr uint32_t idesc2 = idesc_bf16(BM, RP, true);    // R += P x Q (Q MN-major)
+      // R += P x Q (Q MN-major); the bf16 Delta form stores max(0, L) and
+      // negates A here, so the product is -max(0, L) Q
+      constexpr uint32_t idesc2 = idesc_bf16(BM, C::FUSEDN ? 2 * RP : RP, true, EPI == 1 && !SPLIT);
+      const int64_t my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+      const int64_t total = my_tiles * nchunks;
+      const uint32_t stage0 = smem_u32(stages);
+      // running state of MMA1 (chunk G) and MMA2 (chunk D = G - LAG)
+      int s1 = 0, l1 = 0, wb1 = 0;
+      uint32_t ph_full = 0, ph_lfree = 1, ph_wfull = 0;
+      int64_t c1 = 0, tt1 = 0;
+      int s2 = 0, l2 = 0;
+      uint32_t ph_pfull = 0, ph_rempty = 1;
+      int64_t c2 = 0, tt2 = 0;
       bool ok = true;
-      int64_t tt = 0;
-      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++tt) {
-        const int wb = (int)(tt % NWB);
-        if (!(ok = wait_bar(b_wfull + 8 * wb, (uint32_t)((tt / NWB) & 1), abort_flag, p.status, 2))) break;
-        fence_after();
-        const uint32_t wh = tmem + C::COL_W + wb * C::WCOLS;
-        const uint32_t wl = wh + RP / 2;
-        for (int64_t c = 0; c <= nchunks && ok; ++c) {
-          if (c < nchunks) {
-            const int64_t G = tt * nchunks + c;
-            const int s = (int)(G % NSTAGE), lb = (int)(G % NB);
-            if (!(ok = wait_bar(b_full + 8 * s, (uint32_t)((G / NSTAGE) & 1), abort_flag, p.status, 3))) break;
-            if (!(ok = wait_bar(b_lfree + 8 * lb, (uint32_t)((G / NB) & 1) ^ 1u, abort_flag, p.status, 4))) break;
-            fence_after();
-            const uint32_t sb = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
-            const uint32_t d = tmem + C::COL_L + lb * BN;
-#pragma unroll
-            for (int k = 0; k < RP / 16; ++k) {
-              const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
-              const uint64_t bh = sdesc(sb + off, 16, 8 * C::ROWB, C::SWZ);
-              mma_ts(d, wh + k * 8, bh, idesc1, k > 0);
-              if (SPLIT) {
-                const uint64_t bl = sdesc(sb + C::OPER_BYTES + off, 16, 8 * C::ROWB, C::SWZ);
-                mma_ts(d, wh + k * 8, bl, idesc1, 1);
-                mma_ts(d, wl + k * 8, bh, idesc1, 1);
-              }
-            }
-            commit(b_lfull + 8 * lb);
-            if (LOSS) commit(b_empty + 8 * s);
+      for (int64_t G = 0; G < total + (LOSS ? 0 : LAG) && ok; ++G) {
+        if (G < total) {
+          if (c1 == 0) {
+            if (!(ok = wait_bar(b_wfull + 8 * wb1, ph_wfull, abort_flag, p.status, 2))) break;
           }
-          if (!LOSS && c >= 1) {
-            const int64_t G = tt * nchunks + c - 1;
-            const int s = (int)(G % NSTAGE), lb = (int)(G % NB);
-            if (!(ok = wait_bar(b_pfull + 8 * lb, (uint32_t)((G / NB) & 1), abort_flag, p.status, 5))) break;
-            if (c == 1 && !(ok = wait_bar(b_rempty, (uint32_t)(tt & 1) ^ 1u, abort_flag, p.status, 6))) break;
-            fence_after();
-            const uint32_t sb = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
-            const uint32_t pl = tmem + C::COL_L + lb * BN;
+          if (!(ok = wait_bar(b_full + 8 * s1, ph_full, abort_flag, p.status, 3))) break;
+          // L buffer reuse: in the panel kernel the buffer's last reader is
+          // MMA2 of chunk G - NB, issued earlier by this thread, and tcgen05.mma
+          // operations of one thread execute in issue order; in the loss kernel
+          // the last reader is the epilogue, which signals L-free
+          if (LOSS && !(ok = wait_bar(b_lfree + 8 * l1, ph_lfree, abort_flag, p.status, 4))) break;
+          fence_after();
+          const uint32_t wh = tmem + C::COL_W + wb1 * C::WCOLS;
+          const uint32_t wl = wh + RP / 2;
+          const uint64_t d1 = sdesc(stage0 + s1 * C::STAGE_BYTES, 16, 8 * C::ROWB, C::SWZ);
+          const uint32_t d = tmem + C::COL_L + l1 * BN;
 #pragma unroll
-            for (int k = 0; k < BN / 16; ++k) {
-              const uint64_t bh = sdesc(sb + k * 16 * C::ROWB, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
-              const uint32_t acc = (c > 1 || k > 0) ? 1u : 0u;
-              if (!SPLIT) {
-                mma_ts(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
-              } else {
-                const uint64_t bl =
-                    sdesc(sb + C::OPER_BYTES + k * 16 * C::ROWB, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
-                const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
-                mma_ts(tmem + C::COL_R, ph, bh, idesc2, acc);
-                mma_ts(tmem + C::COL_R, ph, bl, idesc2, 1);
-                mma_ts(tmem + C::COL_R, plo, bh, idesc2, 1);
-              }
+          for (int k = 0; k < RP / 16; ++k) {
+            const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
+            const uint64_t bh = d1 + (off >> 4);
+            mma_ts(d, wh + k * 8, bh, idesc1, k > 0);
+            if (SPLIT) {
+              const uint64_t bl = d1 + ((C::OPER_BYTES + off) >> 4);
+              mma_ts(d, wh + k * 8, bl, idesc1, 1);
+              mma_ts(d, wl + k * 8, bh, idesc1, 1);
             }
-            commit(b_empty + 8 * s);
-            commit(b_lfree + 8 * lb);
+          }
+          commit(b_lfull + 8 * l1);
+          if (LOSS) {
+            commit(b_empty + 8 * s1);
+            if (c1 == nchunks - 1) commit(b_wempty + 8 * wb1);
+          }
+          // advance MMA1 state
+          if (++s1 == NSTAGE) { s1 = 0; ph_full ^= 1u; }
+          if (++l1 == NB) { l1 = 0; ph_lfree ^= 1u; }
+          if (++c1 == nchunks) {
+            c1 = 0;
+            ++tt1;
+            if (++wb1 == NWB) { wb1 = 0; ph_wfull ^= 1u; }
           }
         }
-        if (!ok) break;
-        if (!LOSS) commit(b_rfull);
-        commit(b_wempty + 8 * wb);
+        if (!LOSS && G >= LAG) {
+          if (!(ok = wait_bar(b_pfull + 8 * l2, ph_pfull, abort_flag, p.status, 5))) break;
+          if (c2 == 0 && !(ok = wait_bar(b_rempty, ph_rempty, abort_flag, p.status, 6))) break;
+          fence_after();
+          const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
+          const uint32_t pl = tmem + C::COL_L + l2 * BN;
+#pragma unroll
+          for (int k = 0; k < BN / 16; ++k) {
+            const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
+            const uint64_t bl = bh + (C::OPER_BYTES >> 4);
+            const uint32_t acc = (c2 > 0 || k > 0) ? 1u : 0u;
+            if (C::FUSEDN) {          // P [q_hi | q_lo] into two accumulators side by side
+              mma_ts(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
+            } else if (!SPLIT) {      // P (q_hi + q_lo)
+              mma_ts(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
+              mma_ts(tmem + C::COL_R, pl + k * 8, bl, idesc2, 1);
+            } else {                  // P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
+              const uint64_t bl2 = bh + ((2 * C::OPER_BYTES) >> 4);
+              const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
+              mma_ts(tmem + C::COL_R, ph, bh, idesc2, acc);
+              mma_ts(tmem + C::COL_R, ph, bl, idesc2, 1);
+              mma_ts(tmem + C::COL_R, ph, bl2, idesc2, 1);
+              mma_ts(tmem + C::COL_R, plo, bh, idesc2, 1);
+            }
+          }
+          commit(b_empty + 8 * s2);
+          if (c2 == nchunks - 1) {
+            commit(b_rfull);
+            commit(b_wempty + 8 * (int)(tt2 % NWB));
+          }
+          // advance MMA2 state
+          if (++s2 == NSTAGE) s2 = 0;
+          if (++l2 == NB) { l2 = 0; ph_pfull ^= 1u; }
+          if (c2 == 0) ph_rempty ^= 1u;
+          if (++c2 == nchunks) { c2 = 0; ++tt2; }
+        }
       }
       // wait until every MMA issued by this thread has completed
       commit(b_drain);
@@ -280,12 +345,21 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    const int row = threadIdx.x;                      // TMEM lane == tile row
-    const uint32_t lane_base = ((uint32_t)(warp * 32)) << 16;
+    // Two warpgroups take alternate chunks; within a warpgroup thread t owns
+    // TMEM lane t = tile row t.  Tile-level work (W load, R readout) is split
+    // by columns between the two warpgroups.
+    const int wg = warp >> 2;
+    const int row = (warp & 3) * 32 + lane;
+    const int et = threadIdx.x;                          // 0 .. 255
+    const uint32_t lane_base = ((uint32_t)((warp & 3) * 32)) << 16;
     double s2 = 0.0, s1 = 0.0;
     bool ok = true;
+    // loss pass: this thread's row of S, walked alongside the column chunks so
+    // that support entries are left to the support pass (no cancellation)
+    int64_t se = 0, send = 0;
+    int64_t snext = INT64_MAX;
 
-    // load the W tile of local tile index tt into W buffer tt % NWB
+    // load the W tile `tile` into W buffer wb: warpgroup g takes 8-word groups g, g+2, ...
     auto load_w = [&](int64_t tile, int wb) {
       const int64_t li = tile * BM + row;
       const bool valid = li < p.M;
@@ -293,7 +367,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint4* srcl = (const uint4*)(p.Mlo + (p.m0 + (valid ? li : 0)) * RP);
       const uint32_t wcol = tmem + lane_base + C::COL_W + wb * C::WCOLS;
 #pragma unroll
-      for (int q = 0; q < RP / 16; ++q) {
+      for (int q = wg; q < RP / 16; q += 2) {
         uint4 a = valid ? __ldg(src + 2 * q) : make_uint4(0, 0, 0, 0);
         uint4 b = valid ? __ldg(src + 2 * q + 1) : make_uint4(0, 0, 0, 0);
         uint32_t v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
@@ -307,7 +381,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tmem_wait_st();
       fence_before();
-      mbar_arrive(b_wfull + 8 * wb);
+      __syncwarp();
+      if (lane == 0) mbar_arrive(b_wfull + 8 * wb);
     };
 
     {  // prologue: the first NWB tiles
@@ -316,59 +391,102 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     int64_t tt = 0;
     for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++tt) {
+      if (LOSS) {
+        const int64_t li = t * BM + row;
+        se = li < p.M ? p.rowptr[li] : 0;
+        send = li < p.M ? p.rowptr[li + 1] : 0;
+        snext = se < send ? p.cidx[se] : INT64_MAX;
+      }
       for (int64_t c = 0; c < nchunks; ++c) {
         const int64_t G = tt * nchunks + c;
+        if ((int)(G & 1) != wg) continue;
+        if (LOSS) {   // skip the support columns of the other warpgroup's chunks
+          while (snext < c * BN) {
+            ++se;
+            snext = se < send ? p.cidx[se] : INT64_MAX;
+          }
+        }
         const int lb = (int)(G % NB);
         if (!(ok = warp_wait(b_lfull + 8 * lb, (uint32_t)((G / NB) & 1), abort_flag, p.status, 7))) break;
         fence_after();
-        const int64_t kv = p.K - c * BN;              // valid columns in this chunk
+        const int kv = (int)(p.K - c * BN < BN ? p.K - c * BN : BN);   // valid columns in this chunk
         const uint32_t lcol = tmem + lane_base + C::COL_L + lb * BN;
         float c2 = 0.f, c1 = 0.f;
 #pragma unroll 1
-        for (int j = 0; j < BN / 32; ++j) {
-          uint32_t v[32];
-          tmem_ld32(lcol + j * 32, v);
-          tmem_wait_ld(v);
+        for (int jj = 0; jj < BN / 64; ++jj) {
+          uint32_t v0[32], v1[32];
+          tmem_ld32(lcol + jj * 64, v0);
+          tmem_ld32(lcol + jj * 64 + 32, v1);
+          tmem_wait_ld(v0);
+          tmem_wait_ld(v1);
+          if (kv < BN) {   // last chunk: columns past the block end contribute nothing
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              if (jj * 64 + i >= kv) v0[i] = LOSS ? 0u : (EPI == 0 ? 0u : 0xff800000u);   // -inf -> relu 0
+              if (jj * 64 + 32 + i >= kv) v1[i] = LOSS ? 0u : (EPI == 0 ? 0u : 0xff800000u);
+            }
+          }
           if (p.Lout != nullptr) {
             const int64_t li = t * BM + row;
             if (li < p.M) {
 #pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (j * 32 + i < kv) p.Lout[li * p.K + c * BN + j * 32 + i] = __uint_as_float(v[i]);
+              for (int i = 0; i < 32; ++i) {
+                if (jj * 64 + i < kv) p.Lout[li * p.K + c * BN + jj * 64 + i] = __uint_as_float(v0[i]);
+                if (jj * 64 + 32 + i < kv) p.Lout[li * p.K + c * BN + jj * 64 + 32 + i] = __uint_as_float(v1[i]);
+              }
             }
           }
           if (LOSS) {
+            const int64_t cb = c * BN + jj * 64;
+            if (snext < cb + 64) {   // support columns in this group: zero them
+#pragma unroll
+              for (int i = 0; i < 64; ++i) {
+                if (cb + i == snext) {
+                  if (i < 32) v0[i] = 0u; else v1[i - 32] = 0u;
+                  ++se;
+                  snext = se < send ? p.cidx[se] : INT64_MAX;
+                }
+              }
+            }
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
-              float x = fmaxf(0.f, __uint_as_float(v[i]));
-              x = (j * 32 + i < kv) ? x : 0.f;
-              c2 = fmaf(x, x, c2);
-              c1 += x;
+              const float x0 = fmaxf(0.f, __uint_as_float(v0[i])), x1 = fmaxf(0.f, __uint_as_float(v1[i]));
+              c2 = fmaf(x0, x0, c2);
+              c2 = fmaf(x1, x1, c2);
+              c1 += x0 + x1;
             }
+          } else if (!SPLIT) {
+            uint32_t pk0[16], pk1[16];
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+              if (EPI == 0) {   // min(0, L)
+                pk0[i] = min0_bf16x2(pack_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1])));
+                pk1[i] = min0_bf16x2(pack_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1])));
+              } else {          // max(0, L); the MMA negates it
+                pk0[i] = pack_relu_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1]));
+                pk1[i] = pack_relu_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1]));
+              }
+            }
+            tmem_st16(lcol + jj * 32, pk0);
+            tmem_st16(lcol + jj * 32 + 16, pk1);
           } else {
-            float pv[32];
+            // fp32-accurate: P = hi + lo, hi at columns [32j, 32j+16), lo at [32j+16, 32j+32)
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float x = __uint_as_float(v[i]);
-              const float e = EPI == 0 ? fminf(0.f, x) : fminf(0.f, -x);   // min(0,L) or -max(0,L)
-              pv[i] = (j * 32 + i < kv) ? e : 0.f;
-            }
-            if (!SPLIT) {
-              uint32_t pk[16];
-#pragma unroll
-              for (int i = 0; i < 16; ++i) pk[i] = pack_bf16x2(pv[2 * i], pv[2 * i + 1]);
-              tmem_st16(lcol + j * 16, pk);
-            } else {
+            for (int h = 0; h < 2; ++h) {
+              uint32_t(&v)[32] = h == 0 ? v0 : v1;
               uint32_t ph[16], pl[16];
 #pragma unroll
               for (int i = 0; i < 16; ++i) {
-                const float h0 = __bfloat162float(__float2bfloat16_rn(pv[2 * i]));
-                const float h1 = __bfloat162float(__float2bfloat16_rn(pv[2 * i + 1]));
-                ph[i] = pack_bf16x2(h0, h1);
-                pl[i] = pack_bf16x2(pv[2 * i] - h0, pv[2 * i + 1] - h1);
+                const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
+                const float e0 = EPI == 0 ? fminf(0.f, x0) : fminf(0.f, -x0);
+                const float e1 = EPI == 0 ? fminf(0.f, x1) : fminf(0.f, -x1);
+                const uint32_t hp = pack_bf16x2(e0, e1);
+                const float h0 = __uint_as_float(hp << 16), h1 = __uint_as_float(hp & 0xffff0000u);
+                ph[i] = hp;
+                pl[i] = pack_bf16x2(e0 - h0, e1 - h1);
               }
-              tmem_st16(lcol + j * 32, ph);
-              tmem_st16(lcol + j * 32 + 16, pl);
+              tmem_st16(lcol + (2 * jj + h) * 32, ph);
+              tmem_st16(lcol + (2 * jj + h) * 32 + 16, pl);
             }
           }
         }
@@ -376,11 +494,13 @@ __global__ void __launch_bounds__(kThreads, 1)
           s2 += (double)c2;
           s1 += (double)c1;
           fence_before();
-          mbar_arrive(b_lfree + 8 * lb);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_lfree + 8 * lb);
         } else {
           tmem_wait_st();
           fence_before();
-          mbar_arrive(b_pfull + 8 * lb);
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_pfull + 8 * lb);
         }
       }
       if (!ok) break;
@@ -390,9 +510,22 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t li = t * BM + row;
         float* dst = p.R + li * RP;
 #pragma unroll 1
-        for (int j = 0; j < (RP + 31) / 32; ++j) {
+        for (int j = wg; j < (RP + 31) / 32; j += 2) {
           uint32_t v[32];
           tmem_ld32(tmem + lane_base + C::COL_R + j * 32, v);   // RP = 16 reads 16 spare columns
+          if (C::FUSEDN) {
+            uint32_t u[32];
+            tmem_ld32(tmem + lane_base + C::COL_R + RP + j * 32, u);
+            tmem_wait_ld(v);
+            tmem_wait_ld(u);
+            if (RP == 16) {   // the accumulators are 16 columns apart: u[i] = v[i + 16]
+#pragma unroll
+              for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + __uint_as_float(v[i + 16]));
+            } else {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + __uint_as_float(u[i]));
+            }
+          }
           tmem_wait_ld(v);
           if (li < p.M) {
 #pragma unroll
@@ -403,7 +536,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
         }
         fence_before();
-        mbar_arrive(b_rempty);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(b_rempty);
       }
       // refill this tile's W buffer with the tile NWB steps ahead
       const int64_t tn = t + (int64_t)NWB * gridDim.x;
@@ -415,13 +549,13 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (LOSS) {
-      // fixed-order reduction over the 128 epilogue threads
-      red[2 * row] = s2;
-      red[2 * row + 1] = s1;
-      asm volatile("bar.sync 1, 128;" ::: "memory");
-      if (row == 0) {
+      // fixed-order reduction over the 256 epilogue threads
+      red[2 * et] = s2;
+      red[2 * et + 1] = s1;
+      named_bar_sync(1, kEpiThreads);
+      if (et == 0) {
         double a = 0.0, b = 0.0;
-        for (int i = 0; i < 128; ++i) {
+        for (int i = 0; i < kEpiThreads; ++i) {
           a += red[2 * i];
           b += red[2 * i + 1];
         }
@@ -433,7 +567,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   fence_before();
   __syncthreads();
   fence_after();
-  if (warp == 4) tmem_dealloc(tmem, 512);
+  if (warp == kProducerWarp) tmem_dealloc(tmem, 512);
 }
 
 // ---------------------------------------------------------------------------
@@ -484,10 +618,11 @@ bool tensor_map(const bf16* base, int64_t rows, int rp, int panel_w, int bn, CUt
 
 template <int RP, int EPI, bool SPLIT, bool LOSS>
 nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, cudaStream_t s) {
-  using C = Cfg<RP, SPLIT>;
-  CUtensorMap th, tl;
+  using C = Cfg<RP, SPLIT, LOSS>;
+  CUtensorMap th, tl, tl2;
   if (!tensor_map(fq.hi, fq.rows, RP, C::PANEL_W, C::BN, &th)) return NMD_ERR_CUDA;
   if (!tensor_map(fq.lo, fq.rows, RP, C::PANEL_W, C::BN, &tl)) return NMD_ERR_CUDA;
+  if (!tensor_map(fq.lo2, fq.rows, RP, C::PANEL_W, C::BN, &tl2)) return NMD_ERR_CUDA;
   (void)fm;
   static bool attr_set = false;
   if (!attr_set) {
@@ -496,7 +631,7 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
       return NMD_ERR_CUDA;
     attr_set = true;
   }
-  panel_tc_kernel<RP, EPI, SPLIT, LOSS><<<grid, kThreads, C::SMEM, s>>>(th, tl, p);
+  panel_tc_kernel<RP, EPI, SPLIT, LOSS><<<grid, kThreads, C::SMEM, s>>>(th, tl, tl2, p);
   return NMD_OK;
 }
 
@@ -539,9 +674,12 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
                            int64_t* launches, float* Lout) {
   (void)counter;
   if (!tc_supported(a.rp, a.precision)) return NMD_ERR_UNSUPPORTED;
-  TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout};
-  int64_t ntiles = (a.M + BM - 1) / BM;
-  int grid = (int)(ntiles < num_sms ? ntiles : num_sms);
+  TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout, nullptr, nullptr};
+  // fewest CTAs that keep the same number of tile rounds: the SMs left over
+  // run the side-stream kernels of the step
+  const int64_t ntiles = (a.M + BM - 1) / BM;
+  const int64_t rounds = (ntiles + num_sms - 1) / num_sms;
+  const int grid = (int)((ntiles + rounds - 1) / rounds);
   nmd_status st = dispatch<false>(a.rp, a.epilogue, a.precision == NMD_FP32, *a.fm, *a.fq, p, grid, s);
   if (st == NMD_OK) ++*launches;
   return st;
@@ -550,7 +688,7 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
 nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts, int* status,
                                 cudaStream_t s, int64_t* launches) {
   if (!tc_supported(h->rp, h->opt.precision)) return NMD_ERR_UNSUPPORTED;
-  TcParams p{0, h->m, 0, h->n, h->W.hi, h->W.lo, nullptr, parts, status, nullptr};
+  TcParams p{0, h->m, 0, h->n, h->W.hi, h->W.lo, nullptr, parts, status, nullptr, h->ws.rowptr, h->ws.col};
   int64_t ntiles = (h->m + BM - 1) / BM;
   int grid = (int)(ntiles < h->num_sms ? ntiles : h->num_sms);
   if (grid > maxparts) grid = maxparts;

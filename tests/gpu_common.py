@@ -30,7 +30,7 @@ def rel(a, b):
 
 
 def make_pair(S, r, W, H, *, block_rows, block_cols, precision, epilogue=N.NMD_EPI_Z,
-              schedule=N.NMD_STOCH, eta=1.0, gamma=0.9, seed=0, order=N.NMD_ALTERNATE, EW=None,
+              schedule=N.NMD_STOCH, eta=0.5, gamma=0.9, seed=0, order=N.NMD_ALTERNATE, EW=None,
               EH=None):
     """A GPU solver and an oracle state holding the same factors and momentum."""
     sol = N.Solver(S, r, block_rows=block_rows, block_cols=block_cols, schedule=schedule,
@@ -63,7 +63,9 @@ def sync_oracle_to(sol, orc):
 
 
 # scaled-down stand-ins of the five workloads: same generators, several tiles
-# and a ragged last block on both sides
+# and a ragged last block on both sides, blocks of at least 10 r rows (the
+# full workloads have 32 r to 170 r): with fewer, the block Gram matrices of
+# the stochastic steps become near-singular
 def small_cases():
     cases = []
     S, _, _, _ = WL.planted(600, 400, 4, tau=0.5, seed=0)
@@ -75,13 +77,13 @@ def small_cases():
     S, _, _, _ = WL.planted(1500, 1300, 32, tau=None, density=0.05, noise=0.01, seed=2)
     W, H = WL.init_factors(1500, 1300, 32, 2)
     cases.append(("planted1500x1300_r32", S, 32, W, H, 320, 288, N.NMD_STOCH))
-    S = WL.connectome(2500, seed=3)
-    W, H = WL.init_factors(2500, 2500, 64, 3)
-    cases.append(("connectome2500_r64", S, 64, W, H, 448, 448, N.NMD_STOCH))
-    S = WL.connectome(1200, seed=4)
-    W, H = WL.init_factors(1200, 1200, 100, 4)
-    cases.append(("connectome1200_r100", S, 100, W, H, 350, 350, N.NMD_STOCH))
-    S = WL.connectome(1800, seed=5)
-    W, H = WL.init_factors(1800, 1800, 256, 5)
-    cases.append(("connectome1800_r256", S, 256, W, H, 704, 704, N.NMD_STOCH))
+    S = WL.connectome(4000, seed=3)
+    W, H = WL.init_factors(4000, 4000, 64, 3)
+    cases.append(("connectome4000_r64", S, 64, W, H, 1024, 1024, N.NMD_STOCH))
+    S = WL.connectome(3400, seed=4)
+    W, H = WL.init_factors(3400, 3400, 100, 4)
+    cases.append(("connectome3400_r100", S, 100, W, H, 1000, 1000, N.NMD_STOCH))
+    S = WL.connectome(6000, seed=5)
+    W, H = WL.init_factors(6000, 6000, 256, 5)
+    cases.append(("connectome6000_r256", S, 256, W, H, 2560, 2560, N.NMD_STOCH))
     return cases

@@ -34,7 +34,7 @@ def cases():
 
 
 CASE_NAMES = ["planted600x400_r4_exact", "identity1000_r3", "planted1500x1300_r32",
-              "connectome2500_r64", "connectome1200_r100", "connectome1800_r256"]
+              "connectome4000_r64", "connectome3400_r100", "connectome6000_r256"]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -104,8 +104,42 @@ def test_block_terms_parity(name, epi, prec):
 @pytest.mark.parametrize("prec", PRECISIONS, ids=lambda p: PREC_NAMES[p])
 @pytest.mark.parametrize("epi", EPILOGUES, ids=["zform", "delta"])
 @pytest.mark.parametrize("name", CASE_NAMES)
+def test_trajectory_parity(name, epi, prec):
+    """Every block step of the first two sweeps of the workload's own schedule,
+    each from the GPU's current state (teacher forcing): updated factors,
+    momentum and, after each sweep, the losses."""
+    sol, orc = _pair(name, prec, epi)
+    worst = 0.0
+    for sweep in range(2):
+        for side, block, kind in orc.sweep_steps(sweep):
+            sync_oracle_to(sol, orc)
+            M, E, (m0, m1), Q, _, _ = orc._roles(side, block, kind)
+            G = Q.T @ Q
+            ev = np.linalg.eigvalsh(G)
+            sol.block_update(side, block, kind)
+            orc.block_update(side, block, kind)
+            W, H, EW, EH, _ = sol.get_state()
+            got = (W if M is orc.A else H.T)[m0:m1]
+            err = rel(got, M[m0:m1])
+            worst = max(worst, err)
+            assert err <= TOL[prec], (sweep, side, kind, block, err, "kappa(G) = %.1f" % (ev[-1] / ev[0]))
+            if kind == O.STOCH:
+                gotE = (EW if M is orc.A else EH.T)[m0:m1]
+                assert rel(gotE, E[m0:m1]) <= 10 * TOL[prec]
+        sync_oracle_to(sol, orc)
+        g, o = sol.loss(), orc.loss()
+        for k in ("obj", "rmse", "wjd"):
+            assert abs(g[k] - o[k]) <= TOL[prec] * max(abs(o[k]), 1e-3), (sweep, k, g[k], o[k])
+
+
+@pytest.mark.parametrize("prec", PRECISIONS, ids=lambda p: PREC_NAMES[p])
+@pytest.mark.parametrize("epi", EPILOGUES, ids=["zform", "delta"])
+@pytest.mark.parametrize("name", CASE_NAMES)
 def test_block_update_parity(name, epi, prec):
-    """Updated factors and momentum after one step from an identical state."""
+    """Updated factors and momentum after one step from an identical state,
+    for all four kinds of step in turn.  The sequence (exact steps on a
+    stochastic workload) drives the block Gram matrices to condition numbers
+    in the thousands, a stress test of the accuracy of the second product."""
     sol, orc = _pair(name, prec, epi, momentum=True, eta=0.9, gamma=0.8)
     for side, kind in KINDS:
         K = _nblocks(orc, side)
@@ -184,10 +218,12 @@ def test_identity_omega_point_is_fixed(prec):
     H0 = np.stack([np.cos(th), np.sin(th), np.ones(n)], 0).astype(np.float32)
     sol = N.Solver(WL.identity(n), 3, block_rows=16, block_cols=16, precision=prec, gamma=0.9)
     sol.set_factors(W0, H0)
+    # factor entries of size 200 whose products cancel to 0 or 1: fp32
+    # rounding alone moves L by ~1e-5 and a sweep by ~1e-4 relative
     assert sol.loss()["obj"] < (1e-4 if prec == N.NMD_SIMT else 2e-3)
     sol.sweep()
     W, H = sol.get_factors()
-    assert rel(W @ H, W0.astype(np.float64) @ H0) < (1e-4 if prec == N.NMD_SIMT else 2e-3)
+    assert rel(W @ H, W0.astype(np.float64) @ H0) < 1e-3
 
 
 def test_not_spd_is_reported_and_update_skipped():
@@ -230,7 +266,7 @@ def test_bad_block_index_rejected():
 
 @pytest.mark.parametrize("prec", PRECISIONS, ids=lambda p: PREC_NAMES[p])
 def test_deterministic_and_resumable(prec):
-    _, S, r, W, H, br, bc, _ = cases()["connectome2500_r64"]
+    _, S, r, W, H, br, bc, _ = cases()["connectome4000_r64"]
     a = N.Solver(S, r, block_rows=br, block_cols=bc, precision=prec)
     b = N.Solver(S, r, block_rows=br, block_cols=bc, precision=prec)
     a.set_factors(W, H)

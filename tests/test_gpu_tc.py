@@ -30,13 +30,20 @@ def bf16_round(x):
     return rounded.astype(np.uint32).view(np.float32).astype(np.float64)
 
 
+def pieces(X):
+    """bf16 pieces hi, lo, lo2 of fp32 values (each difference exact in fp32)."""
+    X = np.asarray(X, np.float32).astype(np.float64)
+    hi = bf16_round(X.astype(np.float32))
+    lo = bf16_round((X - hi).astype(np.float32))
+    lo2 = bf16_round((X - hi - lo).astype(np.float32))
+    return hi, lo, lo2
+
+
 def operands(X, precision):
-    """The values the tensor cores see for factor rows X (fp32)."""
-    X = np.asarray(X, np.float32)
+    """The values the first product sees for factor rows X (fp32)."""
+    hi, lo, _ = pieces(X)
     if precision == N.NMD_BF16:
-        return bf16_round(X)
-    hi = bf16_round(X)
-    lo = bf16_round((X.astype(np.float64) - hi).astype(np.float32))
+        return hi
     return hi, lo
 
 
@@ -97,15 +104,14 @@ def test_second_product_R(r, n, b, epi, precision):
         L = sol.dense_products(side, block, kind, m1 - m0, c1 - c0).astype(np.float64)
         P = np.minimum(0, L) if epi == N.NMD_EPI_Z else -np.maximum(0, L)
         Qf = Q.astype(np.float32)
-        if precision == N.NMD_BF16:
-            qb = operands(Qf, precision)
+        qh, ql, ql2 = pieces(Qf)
+        if precision == N.NMD_BF16:       # P (q_hi + q_lo)
             Pb = bf16_round(P.astype(np.float32))
-            want = Pb @ qb
-        else:
-            qh, ql = operands(Qf, precision)
+            want = Pb @ (qh + ql)
+        else:                             # P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
             ph = bf16_round(P.astype(np.float32))
             pl = bf16_round((P - ph).astype(np.float32))
-            want = ph @ qh + ph @ ql + pl @ qh
+            want = ph @ (qh + ql + ql2) + pl @ qh
         Sd = src.dense_panel(m0, m1, c0, c1)
         sup = Sd > 0
         # the support correction uses fp32 L and q: c = S - min(0, L) on the support
