@@ -221,6 +221,24 @@ typedef enum { NMD_K_DENSE = 0, NMD_K_SPARSE = 1, NMD_K_GRAM = 2, NMD_K_UPDATE =
 nmd_status nmd_profile(nmd_handle* h, int on);
 nmd_status nmd_profile_read(nmd_handle* h, int32_t kernel_class, double* ms, int64_t* launches);
 
+/* Gram matrix G = Q^T Q (r x r, row-major, written to d_G) of the K rows of a
+ * caller's device matrix Q (row stride ld >= r floats), computed without any
+ * device allocation and without a handle or workspace.  The paper has no
+ * counterpart of this call; it exists for callers that cannot allocate
+ * device memory at the point of the call -- code running inside a
+ * framework or plugin that owns the whole device pool, or a real-time loop
+ * that forbids cudaMalloc -- and so cannot provide the workspace that
+ * nmd_create needs.  The partial sums go to a 2 MiB array in the library's
+ * static device memory, which every GPU that loads the library holds until
+ * the process exits.  Limits: r <= 128 (NMD_ERR_WORKSPACE beyond), K >= 1.
+ * The first call on a device looks up that array's device address (with the
+ * device current); make that first call before any stream capture.  All
+ * calls share the array, so calls that overlap on the GPU (other streams,
+ * other threads) race and must be serialised by the caller.  Asynchronous on
+ * `stream` (a cudaStream_t, NULL = legacy default stream); the result equals
+ * the Gram matrix of nmd_block_terms to fp32 rounding (summation order). */
+nmd_status nmd_gram_noalloc(const float* d_Q, int64_t K, int32_t r, int64_t ld, float* d_G, void* stream);
+
 /* Number of kernel launches this handle has issued (for launch accounting). */
 int64_t nmd_launch_count(const nmd_handle* h);
 

@@ -31,7 +31,7 @@ EXPORTS = [
     "nmd_get_factors", "nmd_block_update", "nmd_sweep", "nmd_block_order", "nmd_loss", "nmd_sync",
     "nmd_block_terms", "nmd_dense_products", "nmd_panel_traversal", "nmd_get_state", "nmd_set_state",
     "nmd_launch_count", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
-    "nmd_destroy",
+    "nmd_destroy", "nmd_gram_noalloc",
 ]
 
 
@@ -92,6 +92,7 @@ def lib() -> C.CDLL:
             "nmd_status_string": (C.c_char_p, [C.c_int]),
             "nmd_last_error": (C.c_char_p, [_P]),
             "nmd_destroy": (None, [_P]),
+            "nmd_gram_noalloc": (C.c_int, [_P, C.c_int64, C.c_int32, C.c_int64, _P, _P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -244,6 +245,12 @@ def nmd_profile_read(h, kernel_class: int):
     n = C.c_int64(0)
     _check(h, lib().nmd_profile_read(h, kernel_class, C.byref(ms), C.byref(n)), "nmd_profile_read")
     return ms.value, n.value
+
+
+def nmd_gram_noalloc(d_Q, K: int, r: int, ld: int, d_G, stream_ptr: int) -> int:
+    """G = Q^T Q of a device matrix with no device allocation (static scratch);
+    returns the status code."""
+    return lib().nmd_gram_noalloc(_ptr(d_Q), K, r, ld, _ptr(d_G), stream_ptr)
 
 
 def nmd_destroy(h):
