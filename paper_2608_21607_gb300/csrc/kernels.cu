@@ -273,8 +273,14 @@ __global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __re
   if (w >= nmulti) return;
   const PanelRow mr = multi[w];
   for (int c = lane; c < rp; c += 32) {
-    float s = 0.f;
-    for (int q = 0; q < mr.len; ++q) s += partials[(mr.beg + q) * rp + c];
+    // eight independent loads in flight, combined in a fixed order
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    int q = 0;
+    for (; q + 8 <= mr.len; q += 8)
+#pragma unroll
+      for (int u = 0; u < 8; ++u) acc[u] += __ldg(partials + (mr.beg + q + u) * rp + c);
+    for (; q < mr.len; ++q) acc[0] += __ldg(partials + (mr.beg + q) * rp + c);
+    const float s = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
     R[(mr.row - m0) * rp + c] += s;
   }
 }
@@ -285,9 +291,11 @@ __global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __re
 //   Delta form: U = eta X            (eqs. spLsqA/spLsqB)
 // then E = U + gamma E (stochastic steps) and M += E, refreshing the bf16
 // pieces.  Skipped entirely while a sticky error is set.
-// A thread owns 8 consecutive columns of one row (float4 traffic, coalesced
-// along the row); a block keeps CW columns of G^{-1} in shared memory and
-// stages the R rows of each pass there.
+// X = R G^{-1} is a small GEMM per tile of 64 rows: a block keeps CW columns
+// of G^{-1} in shared memory, stages the tile's R transposed (k-major), and
+// thread (ty, tx) of 16 x 16 computes rows 4 ty .. 4 ty + 3 and columns
+// CPT tx .. CPT tx + CPT - 1 (CPT = CW / 16) with 128-bit shared loads, then
+// applies the elementwise update to those entries.
 // ---------------------------------------------------------------------------
 template <int RP>
 __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
@@ -298,78 +306,101 @@ __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ M, bf16
                                                      float gamma, int momentum, int delta_form,
                                                      int* __restrict__ status) {
   constexpr int CW = RP <= 128 ? RP : 128;    // output columns handled by this block
-  constexpr int TPR = CW / 8;                 // threads per row
-  constexpr int ROWS = 256 / TPR;             // rows per pass
+  constexpr int CPT = CW / 16;                // columns per thread (1, 2, 4 or 8)
+  constexpr int TR = 64;                      // rows per tile
+  constexpr int LDR = TR + 4;                 // row stride of the transposed R tile
   extern __shared__ float sm[];
   float* Gs = sm;                             // RP x CW
-  float* Rs = sm + RP * CW;                   // ROWS x (RP + 4)
+  float* Rt = sm + RP * CW;                   // RP x LDR: Rt[k * LDR + row] = R[row][k]
   if (*(volatile int*)status != 0) return;
   const int cw0 = blockIdx.y * CW;
   for (int e = threadIdx.x; e < RP * CW; e += blockDim.x) Gs[e] = Ginv[(e / CW) * RP + cw0 + (e % CW)];
-  const int rsub = threadIdx.x / TPR;
-  const int c0 = (threadIdx.x % TPR) * 8;     // within the block's CW columns
-  for (int64_t base = (int64_t)blockIdx.x * ROWS; base < rows; base += (int64_t)gridDim.x * ROWS) {
+  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+  for (int64_t base = (int64_t)blockIdx.x * TR; base < rows; base += (int64_t)gridDim.x * TR) {
     __syncthreads();
-    for (int e = threadIdx.x; e < ROWS * (RP / 4); e += blockDim.x) {
-      const int rr = e / (RP / 4), k4 = e % (RP / 4);
+    for (int e = threadIdx.x; e < TR * (RP / 4); e += blockDim.x) {
+      const int rr = e / (RP / 4), k4 = 4 * (e % (RP / 4));
       float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (base + rr < rows) v = *(const float4*)(R + (base + rr) * RP + 4 * k4);
-      *(float4*)(Rs + rr * (RP + 4) + 4 * k4) = v;
+      if (base + rr < rows) v = *(const float4*)(R + (base + rr) * RP + k4);
+      Rt[(k4 + 0) * LDR + rr] = v.x;
+      Rt[(k4 + 1) * LDR + rr] = v.y;
+      Rt[(k4 + 2) * LDR + rr] = v.z;
+      Rt[(k4 + 3) * LDR + rr] = v.w;
     }
     __syncthreads();
-    const int64_t li = base + rsub;
-    if (li >= rows) continue;
-    float x[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    const float* rrow = Rs + rsub * (RP + 4);
+    float x[4][CPT];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) x[i][j] = 0.f;
 #pragma unroll 4
     for (int k = 0; k < RP; ++k) {
-      const float rk = rrow[k];
-      const float4 g0 = *(const float4*)(Gs + k * CW + c0);
-      const float4 g1 = *(const float4*)(Gs + k * CW + c0 + 4);
-      x[0] = fmaf(rk, g0.x, x[0]); x[1] = fmaf(rk, g0.y, x[1]);
-      x[2] = fmaf(rk, g0.z, x[2]); x[3] = fmaf(rk, g0.w, x[3]);
-      x[4] = fmaf(rk, g1.x, x[4]); x[5] = fmaf(rk, g1.y, x[5]);
-      x[6] = fmaf(rk, g1.z, x[6]); x[7] = fmaf(rk, g1.w, x[7]);
-    }
-    const int64_t g = (m0 + li) * RP + cw0 + c0;
-    float mo[8], eo[8], mn[8];
-    *(float4*)mo = *(const float4*)(M + g);
-    *(float4*)(mo + 4) = *(const float4*)(M + g + 4);
-    if (momentum) {
-      *(float4*)eo = *(const float4*)(E + g);
-      *(float4*)(eo + 4) = *(const float4*)(E + g + 4);
-    }
-    bool finite = true;
-    uint32_t hw[4], lw[4], l2w[4];
+      const float4 a = *(const float4*)(Rt + k * LDR + 4 * ty);
+      float b[CPT];
+      if (CPT >= 4) {
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const float u = delta_form ? eta * x[j] : eta * (x[j] - mo[j]);
-      const float e = momentum ? fmaf(gamma, eo[j], u) : u;
-      eo[j] = e;
-      mn[j] = mo[j] + e;
-      finite = finite && isfinite(mn[j]);
+        for (int j = 0; j < CPT; j += 4) {
+          const float4 g = *(const float4*)(Gs + k * CW + CPT * tx + j);
+          b[j] = g.x; b[j + 1] = g.y; b[j + 2] = g.z; b[j + 3] = g.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) b[j] = Gs[k * CW + CPT * tx + j];
+      }
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) {
+        x[0][j] = fmaf(a.x, b[j], x[0][j]);
+        x[1][j] = fmaf(a.y, b[j], x[1][j]);
+        x[2][j] = fmaf(a.z, b[j], x[2][j]);
+        x[3][j] = fmaf(a.w, b[j], x[3][j]);
+      }
     }
 #pragma unroll
-    for (int j = 0; j < 8; j += 2) {
-      const bf16 h0 = __float2bfloat16_rn(mn[j]), h1 = __float2bfloat16_rn(mn[j + 1]);
-      const float r0 = mn[j] - __bfloat162float(h0), r1 = mn[j + 1] - __bfloat162float(h1);
-      const bf16 l0 = __float2bfloat16_rn(r0), l1 = __float2bfloat16_rn(r1);
-      const bf16 q0 = __float2bfloat16_rn(r0 - __bfloat162float(l0));
-      const bf16 q1 = __float2bfloat16_rn(r1 - __bfloat162float(l1));
-      hw[j / 2] = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-      lw[j / 2] = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
-      l2w[j / 2] = (uint32_t)__bfloat16_as_ushort(q0) | ((uint32_t)__bfloat16_as_ushort(q1) << 16);
+    for (int i = 0; i < 4; ++i) {
+      const int64_t li = base + 4 * ty + i;
+      if (li >= rows) break;
+      const int64_t g = (m0 + li) * RP + cw0 + CPT * tx;
+      bool finite = true;
+      if (CPT == 1) {
+        const float mo = M[g];
+        const float eo = momentum ? E[g] : 0.f;
+        const float u = delta_form ? eta * x[i][0] : eta * (x[i][0] - mo);
+        const float e = momentum ? fmaf(gamma, eo, u) : u;
+        const float nv = mo + e;
+        finite = isfinite(nv);
+        M[g] = nv;
+        if (momentum) E[g] = e;
+        const bf16 h = __float2bfloat16_rn(nv);
+        const float r1 = nv - __bfloat162float(h);
+        const bf16 l = __float2bfloat16_rn(r1);
+        Mhi[g] = h;
+        Mlo[g] = l;
+        Mlo2[g] = __float2bfloat16_rn(r1 - __bfloat162float(l));
+      }
+#pragma unroll
+      for (int j = 0; j + 1 < CPT; j += 2) {
+        const float2 mo = *(const float2*)(M + g + j);
+        float2 eo = make_float2(0.f, 0.f);
+        if (momentum) eo = *(const float2*)(E + g + j);
+        const float u0 = delta_form ? eta * x[i][j] : eta * (x[i][j] - mo.x);
+        const float u1 = delta_form ? eta * x[i][j + 1] : eta * (x[i][j + 1] - mo.y);
+        const float e0 = momentum ? fmaf(gamma, eo.x, u0) : u0;
+        const float e1 = momentum ? fmaf(gamma, eo.y, u1) : u1;
+        const float n0 = mo.x + e0, n1 = mo.y + e1;
+        finite = finite && isfinite(n0) && isfinite(n1);
+        *(float2*)(M + g + j) = make_float2(n0, n1);
+        if (momentum) *(float2*)(E + g + j) = make_float2(e0, e1);
+        const bf16 h0 = __float2bfloat16_rn(n0), h1 = __float2bfloat16_rn(n1);
+        const float r0 = n0 - __bfloat162float(h0), r1 = n1 - __bfloat162float(h1);
+        const bf16 l0 = __float2bfloat16_rn(r0), l1 = __float2bfloat16_rn(r1);
+        const bf16 q0 = __float2bfloat16_rn(r0 - __bfloat162float(l0));
+        const bf16 q1 = __float2bfloat16_rn(r1 - __bfloat162float(l1));
+        *(uint32_t*)(Mhi + g + j) = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
+        *(uint32_t*)(Mlo + g + j) = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
+        *(uint32_t*)(Mlo2 + g + j) = (uint32_t)__bfloat16_as_ushort(q0) | ((uint32_t)__bfloat16_as_ushort(q1) << 16);
+      }
+      if (!finite) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
     }
-    if (!finite) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
-    *(float4*)(M + g) = *(float4*)mn;
-    *(float4*)(M + g + 4) = *(float4*)(mn + 4);
-    if (momentum) {
-      *(float4*)(E + g) = *(float4*)eo;
-      *(float4*)(E + g + 4) = *(float4*)(eo + 4);
-    }
-    *(uint4*)(Mhi + g) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-    *(uint4*)(Mlo + g) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
-    *(uint4*)(Mlo2 + g) = make_uint4(l2w[0], l2w[1], l2w[2], l2w[3]);
   }
 }
 
@@ -563,19 +594,18 @@ template <int RP>
 static void update_rp(const StepArgs& a, const float* R, const float* Ginv, float eta, float gamma, bool momentum,
                       int* status, cudaStream_t s) {
   constexpr int CW = RP <= 128 ? RP : 128;
-  constexpr int ROWS = 256 / (CW / 8);
-  const size_t smem = ((size_t)RP * CW + ROWS * (RP + 4)) * sizeof(float);
+  const size_t smem = ((size_t)RP * CW + (size_t)RP * (64 + 4)) * sizeof(float);
   static bool attr = false;
   if (!attr) {
     cudaFuncSetAttribute(update_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     attr = true;
   }
-  const int per_sm = RP <= 32 ? 8 : (RP == 64 ? 4 : (RP == 128 ? 2 : 1));
-  const int64_t tiles = (a.M + ROWS - 1) / ROWS;
+  const int per_sm = RP <= 64 ? 2 : 1;
+  const int64_t tiles = (a.M + 63) / 64;
   dim3 grid((unsigned)std::min<int64_t>(tiles, 152 * per_sm), RP / CW);
   const Factor& f = *a.fm;
-  update_kernel<RP><<<grid, 256, smem, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Ginv, eta, gamma, momentum,
-                                            a.epilogue == NMD_EPI_DELTA, status);
+  update_kernel<RP><<<grid, 256, smem, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Ginv, eta, gamma,
+                                            momentum, a.epilogue == NMD_EPI_DELTA, status);
 }
 
 void launch_update(const StepArgs& a, const float* R, const float* Ginv, float eta, float gamma, bool momentum,
