@@ -26,7 +26,6 @@ import statistics
 import subprocess
 import sys
 import tempfile
-import threading
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -100,13 +99,6 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def dist_setup():
-    ws = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    return ws, rank, local
-
-
 def oracle_sample(wl, budget_s=20.0):
     """Time the fp64 oracle on block steps of the workload until the budget
     (at least one COL/STOCH and one ROW/STOCH step); Z entries per second."""
@@ -143,7 +135,8 @@ def main():
     args = ap.parse_args()
     assert args.warmup >= 3, "at least 3 warm-up steps"
 
-    ws, rank, local = dist_setup()
+    from paper_2608_21607_gb300.replicas import env as replica_env
+    ws, rank, local = replica_env()
     metric = "Z entries/s per full ALS sweep (2*m*n / sweep time)"
     from paper_2608_21607_gb300 import workloads as WLm
     gen, r, block = WORKLOADS[args.workload]
@@ -180,11 +173,9 @@ def main():
     from paper_2608_21607_gb300 import build as B
     from paper_2608_21607_gb300 import nmd as N
 
+    from paper_2608_21607_gb300.replicas import Replicas
     torch.cuda.set_device(local)
-    dist = None
-    if ws > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    rep = Replicas(device=torch.device("cuda", local))
     B.build()
     wl = WLm.workload(gen, seed=0)
     prec = {"bf16": N.NMD_BF16, "fp32": N.NMD_FP32}[args.precision]
@@ -196,8 +187,7 @@ def main():
 
     def barrier():
         torch.cuda.synchronize()
-        if dist is not None:
-            dist.barrier()
+        rep.barrier()
         torch.cuda.synchronize()
 
     # ---------------- device-resident timing ----------------
@@ -225,13 +215,9 @@ def main():
     sol.profile(False)
     clk = clocks.stop()
     barrier()
-    t_max = ms_total
-    if dist is not None:
-        t = torch.tensor([ms_total], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        t_max = float(t.item())
     entries = 2.0 * wl.m * wl.n
-    value = ws * entries * args.steps / (t_max / 1e3)
+    value, t_max_s = rep.job_rate(entries * args.steps, ms_total / 1e3)   # replicas: weak scaling
+    t_max = 1e3 * t_max_s
 
     # dense kernel roofline: 4 M K r algorithmic flops per launch (2 M K r for
     # L = M Q^T and 2 M K r for R = P Q), summed over the launches of a sweep
@@ -276,12 +262,8 @@ def main():
         for _ in range(args.steps):
             e2e_step()
         torch.cuda.synchronize()
-        e2e_s = time.perf_counter() - t0
-        if dist is not None:
-            t = torch.tensor([e2e_s], device="cuda", dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_s = float(t.item())
-        e2e = {"value": ws * entries * args.steps / e2e_s, "unit": "Z entries/s", "h2d_bytes_per_step": h2d,
+        e2e_value, e2e_s = rep.job_rate(entries * args.steps, time.perf_counter() - t0)
+        e2e = {"value": e2e_value, "unit": "Z entries/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": 1e3 * e2e_s / args.steps}
 
     cpu = None
@@ -304,8 +286,7 @@ def main():
                 "e2e": e2e, "roofline": roofline, "cpu_baseline": cpu, "clocks": clk,
                 "gpu_launches": launches}
         print(json.dumps(line))
-    if dist is not None:
-        dist.destroy_process_group()
+    rep.close()
     return 0
 
 

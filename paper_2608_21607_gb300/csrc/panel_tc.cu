@@ -20,11 +20,15 @@
 // dense parts of eq. SLloss / eq. RMSE / eq. WJD); the support entries are
 // summed by a separate pass.
 //
-// Warp roles (320 threads, one CTA per SM, persistent over M tiles):
+// Warp roles (352 threads, one CTA per SM, persistent over M tiles):
 //   warps 0-7  epilogue, two warpgroups taking alternate chunks; in each,
 //              thread t owns TMEM lane t = tile row t
 //   warp 8     TMA producer of Q chunks (+ TMEM allocation)
-//   warp 9     MMA issuer (one thread)
+//   warp 9     issues MMA1 (L = W Q^T) for every chunk
+//   warp 10    issues MMA2 (R += P Q) for every chunk
+// The two MMA warps run converged and predicate each tcgen05 operation on an
+// elected lane; with two issuers the bookkeeping of one (barrier polls,
+// commits) overlaps the other's products on the tensor core.
 // Every mbarrier wait is bounded (2 s): on expiry the kernel records
 // NMD_ERR_TIMEOUT, the other roles stop at their next wait, in-flight MMAs
 // and copies are drained and TMEM is freed before the kernel returns.
@@ -43,8 +47,8 @@ namespace {
 using namespace tc;
 
 constexpr int kEpiThreads = 256;                 // two epilogue warpgroups
-constexpr int kProducerWarp = 8, kMmaWarp = 9;
-constexpr int kThreads = 320;
+constexpr int kProducerWarp = 8, kMma1Warp = 9, kMma2Warp = 10;
+constexpr int kThreads = 352;
 constexpr int BM = 128;
 constexpr uint64_t kTimeoutNs = 2000000000ull;
 
@@ -60,7 +64,6 @@ struct Cfg {
   static constexpr int NWB = (RP == 256) ? 1 : 2;      // W tile buffers
   static constexpr int FREE = 512 - NWB * WCOLS - RCOLS;
   static constexpr int NB = FREE / BN >= 3 ? 3 : FREE / BN;  // L buffers
-  static constexpr int LAG = NB >= 3 ? 2 : 1;                 // MMA1 runs LAG chunks ahead of MMA2
   static constexpr int PANEL_W = RP < 64 ? RP : 64;    // elements per row of one swizzle panel
   static constexpr int ROWB = PANEL_W * 2;             // bytes per panel row (= swizzle width)
   static constexpr int PANEL_BYTES = BN * ROWB;
@@ -72,20 +75,20 @@ struct Cfg {
   static constexpr int NQ = LOSS ? (SPLIT ? 2 : 1) : (SPLIT ? 3 : 2);
   static constexpr int STAGE_BYTES = OPER_BYTES * NQ;
   static constexpr int NSTAGE_RAW = (160 * 1024) / STAGE_BYTES;
-  static constexpr int NSTAGE = NSTAGE_RAW > 8 ? 8 : (NSTAGE_RAW < 3 ? 3 : NSTAGE_RAW);
+  static constexpr int NSTAGE = NSTAGE_RAW > 8 ? 8 : (NSTAGE_RAW < 2 ? 2 : NSTAGE_RAW);
   static constexpr uint32_t SWZ = PANEL_W == 64 ? SWZ_128B : (PANEL_W == 32 ? SWZ_64B : SWZ_32B);
   static constexpr int COL_L = 0;               // NB x BN columns
   static constexpr int COL_R = NB * BN;         // RP columns
   static constexpr int COL_W = COL_R + RCOLS;   // NWB x WCOLS columns
   // barriers: full[NSTAGE], empty[NSTAGE], lfull[NB], pfull[NB], lfree[NB], rfull, rempty,
-  // wfull[2], wempty[2], drain
-  static constexpr int NBAR = 2 * NSTAGE + 3 * NB + 7;
+  // wfull[2], wempty[2], drain, drain2
+  static constexpr int NBAR = 2 * NSTAGE + 3 * NB + 8;
   static constexpr size_t SMEM_USED = 1024 + (size_t)NSTAGE * STAGE_BYTES + NBAR * 8 + 64 + 256 * 16;
   // at least 120 KB so that a second CTA (and its 512-column TMEM request)
   // never shares the SM
   static constexpr size_t SMEM = SMEM_USED > 120 * 1024 ? SMEM_USED : 120 * 1024;
   static_assert(NB >= 2, "need two L buffers");
-  static_assert(NSTAGE > LAG, "a stage must be free before MMA1 runs LAG chunks ahead");
+  static_assert(NSTAGE >= 2, "stages");
   static_assert(SMEM <= 227 * 1024, "shared memory per block");
   static_assert(COL_W + NWB * WCOLS <= 512, "TMEM budget");
   static_assert(BN % 32 == 0 && RP % 16 == 0, "shapes");
@@ -130,6 +133,17 @@ __device__ __forceinline__ bool wait_bar(uint32_t bar, uint32_t parity, volatile
   return wait_bar_slow(bar, parity, abort_flag, status, where);
 }
 
+// Wait for a converged warp: every lane tests the phase; if it has not
+// completed, lane 0 polls and the outcome is broadcast.
+__device__ __forceinline__ bool conv_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
+                                          int where) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
+  int ok = 0;
+  if ((threadIdx.x & 31) == 0) ok = wait_bar_slow(bar, parity, abort_flag, status, where);
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  return ok != 0;
+}
+
 // Warp-uniform wait: lane 0 polls, the outcome is broadcast to the warp.
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
                                           int where) {
@@ -164,6 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t b_wfull = b_rempty + 8;
   const uint32_t b_wempty = b_wfull + 16;
   const uint32_t b_drain = b_wempty + 16;
+  const uint32_t b_drain2 = b_drain + 8;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -183,6 +198,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(b_wempty + 8 * i, 1);
     }
     mbar_init(b_drain, 1);
+    mbar_init(b_drain2, 1);
     *abort_flag = 0;
     fence_mbar_init();
   }
@@ -236,112 +252,108 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-  } else if (warp == kMmaWarp) {
-    // ------------------------------------------------------------ MMA issuer
-    // One global chunk sequence G over this CTA's tiles.  Step G issues MMA1
-    // of chunk G and MMA2 of chunk G - LAG, so the epilogue of a chunk has
-    // LAG chunks of tensor work to hide behind, including across tiles.  All
-    // ring positions and phases are kept as running counters.
+  } else if (warp == kMma1Warp) {
+    // ------------------------------------------------------------ MMA1 issuer
+    // L[lb] = W tile x chunk^T for every chunk G of this CTA's tiles, in order.
+    constexpr uint32_t idesc1 = idesc_bf16(BM, BN, false);   // Q K-major
+    const int64_t my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
+    const int64_t total = my_tiles * nchunks;
+    const uint32_t stage0 = smem_u32(stages);
+    int s1 = 0, l1 = 0, wb1 = 0;
+    uint32_t ph_full = 0, ph_lfree = 1, ph_wfull = 0;
+    int64_t c1 = 0;
+    bool ok = true;
+    for (int64_t G = 0; G < total && ok; ++G) {
+      if (c1 == 0 && !(ok = conv_wait(b_wfull + 8 * wb1, ph_wfull, abort_flag, p.status, 2))) break;
+      if (!(ok = conv_wait(b_full + 8 * s1, ph_full, abort_flag, p.status, 3))) break;
+      if (!(ok = conv_wait(b_lfree + 8 * l1, ph_lfree, abort_flag, p.status, 4))) break;
+      fence_after();
+      const uint32_t wh = tmem + C::COL_W + wb1 * C::WCOLS;
+      const uint32_t wl = wh + RP / 2;
+      const uint64_t d1 = sdesc(stage0 + s1 * C::STAGE_BYTES, 16, 8 * C::ROWB, C::SWZ);
+      const uint32_t d = tmem + C::COL_L + l1 * BN;
+#pragma unroll
+      for (int k = 0; k < RP / 16; ++k) {
+        const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
+        const uint64_t bh = d1 + (off >> 4);
+        mma_ts_elect(d, wh + k * 8, bh, idesc1, k > 0);
+        if (SPLIT) {
+          const uint64_t bl = d1 + ((C::OPER_BYTES + off) >> 4);
+          mma_ts_elect(d, wh + k * 8, bl, idesc1, 1);
+          mma_ts_elect(d, wl + k * 8, bh, idesc1, 1);
+        }
+      }
+      commit_elect(b_lfull + 8 * l1);
+      if (LOSS) commit_elect(b_empty + 8 * s1);
+      if (c1 == nchunks - 1) commit_elect(b_wempty + 8 * wb1);
+      if (++s1 == NSTAGE) { s1 = 0; ph_full ^= 1u; }
+      if (++l1 == NB) { l1 = 0; ph_lfree ^= 1u; }
+      if (++c1 == nchunks) {
+        c1 = 0;
+        if (++wb1 == NWB) { wb1 = 0; ph_wfull ^= 1u; }
+      }
+    }
+    // wait until every MMA issued by this warp has completed
+    commit_elect(b_drain);
     if (lane == 0) {
-      constexpr int LAG = C::LAG;
-      constexpr uint32_t idesc1 = idesc_bf16(BM, BN, false);   // L = W x Q^T (Q K-major)
-      // R += P x Q (Q MN-major); the bf16 Delta form stores max(0, L) and
-      // negates A here, so the product is -max(0, L) Q
-      constexpr uint32_t idesc2 = idesc_bf16(BM, C::FUSEDN ? 2 * RP : RP, true, EPI == 1 && !SPLIT);
+      const uint64_t t0 = globaltimer_ns();
+      while (!mbar_try_wait(b_drain, 0) && globaltimer_ns() - t0 < 200000000ull) {
+      }
+    }
+    __syncwarp();
+  } else if (warp == kMma2Warp) {
+    // ------------------------------------------------------------ MMA2 issuer
+    // R += P[lb] x chunk for every chunk once its P is in TMEM; frees the
+    // shared-memory stage and the L buffer, and hands R over per tile.
+    if (!LOSS) {
+      constexpr uint32_t idesc2 = idesc_bf16(BM, C::FUSEDN ? 2 * RP : RP, true, EPI == 1 && !SPLIT);   // Q MN-major
       const int64_t my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
       const int64_t total = my_tiles * nchunks;
       const uint32_t stage0 = smem_u32(stages);
-      // running state of MMA1 (chunk G) and MMA2 (chunk D = G - LAG)
-      int s1 = 0, l1 = 0, wb1 = 0;
-      uint32_t ph_full = 0, ph_lfree = 1, ph_wfull = 0;
-      int64_t c1 = 0, tt1 = 0;
       int s2 = 0, l2 = 0;
       uint32_t ph_pfull = 0, ph_rempty = 1;
-      int64_t c2 = 0, tt2 = 0;
+      int64_t c2 = 0;
       bool ok = true;
-      for (int64_t G = 0; G < total + (LOSS ? 0 : LAG) && ok; ++G) {
-        if (G < total) {
-          if (c1 == 0) {
-            if (!(ok = wait_bar(b_wfull + 8 * wb1, ph_wfull, abort_flag, p.status, 2))) break;
-          }
-          if (!(ok = wait_bar(b_full + 8 * s1, ph_full, abort_flag, p.status, 3))) break;
-          // L buffer reuse: in the panel kernel the buffer's last reader is
-          // MMA2 of chunk G - NB, issued earlier by this thread, and tcgen05.mma
-          // operations of one thread execute in issue order; in the loss kernel
-          // the last reader is the epilogue, which signals L-free
-          if (LOSS && !(ok = wait_bar(b_lfree + 8 * l1, ph_lfree, abort_flag, p.status, 4))) break;
-          fence_after();
-          const uint32_t wh = tmem + C::COL_W + wb1 * C::WCOLS;
-          const uint32_t wl = wh + RP / 2;
-          const uint64_t d1 = sdesc(stage0 + s1 * C::STAGE_BYTES, 16, 8 * C::ROWB, C::SWZ);
-          const uint32_t d = tmem + C::COL_L + l1 * BN;
+      for (int64_t D = 0; D < total && ok; ++D) {
+        if (!(ok = conv_wait(b_pfull + 8 * l2, ph_pfull, abort_flag, p.status, 5))) break;
+        if (c2 == 0 && !(ok = conv_wait(b_rempty, ph_rempty, abort_flag, p.status, 6))) break;
+        fence_after();
+        const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
+        const uint32_t pl = tmem + C::COL_L + l2 * BN;
 #pragma unroll
-          for (int k = 0; k < RP / 16; ++k) {
-            const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
-            const uint64_t bh = d1 + (off >> 4);
-            mma_ts(d, wh + k * 8, bh, idesc1, k > 0);
-            if (SPLIT) {
-              const uint64_t bl = d1 + ((C::OPER_BYTES + off) >> 4);
-              mma_ts(d, wh + k * 8, bl, idesc1, 1);
-              mma_ts(d, wl + k * 8, bh, idesc1, 1);
-            }
-          }
-          commit(b_lfull + 8 * l1);
-          if (LOSS) {
-            commit(b_empty + 8 * s1);
-            if (c1 == nchunks - 1) commit(b_wempty + 8 * wb1);
-          }
-          // advance MMA1 state
-          if (++s1 == NSTAGE) { s1 = 0; ph_full ^= 1u; }
-          if (++l1 == NB) { l1 = 0; ph_lfree ^= 1u; }
-          if (++c1 == nchunks) {
-            c1 = 0;
-            ++tt1;
-            if (++wb1 == NWB) { wb1 = 0; ph_wfull ^= 1u; }
+        for (int k = 0; k < BN / 16; ++k) {
+          const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
+          const uint64_t bl = bh + (C::OPER_BYTES >> 4);
+          const uint32_t acc = (c2 > 0 || k > 0) ? 1u : 0u;
+          if (C::FUSEDN) {          // P [q_hi | q_lo] into two accumulators side by side
+            mma_ts_elect(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
+          } else if (!SPLIT) {      // P (q_hi + q_lo)
+            mma_ts_elect(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
+            mma_ts_elect(tmem + C::COL_R, pl + k * 8, bl, idesc2, 1);
+          } else {                  // P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
+            const uint64_t bl2 = bh + ((2 * C::OPER_BYTES) >> 4);
+            const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
+            mma_ts_elect(tmem + C::COL_R, ph, bh, idesc2, acc);
+            mma_ts_elect(tmem + C::COL_R, ph, bl, idesc2, 1);
+            mma_ts_elect(tmem + C::COL_R, ph, bl2, idesc2, 1);
+            mma_ts_elect(tmem + C::COL_R, plo, bh, idesc2, 1);
           }
         }
-        if (!LOSS && G >= LAG) {
-          if (!(ok = wait_bar(b_pfull + 8 * l2, ph_pfull, abort_flag, p.status, 5))) break;
-          if (c2 == 0 && !(ok = wait_bar(b_rempty, ph_rempty, abort_flag, p.status, 6))) break;
-          fence_after();
-          const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
-          const uint32_t pl = tmem + C::COL_L + l2 * BN;
-#pragma unroll
-          for (int k = 0; k < BN / 16; ++k) {
-            const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
-            const uint64_t bl = bh + (C::OPER_BYTES >> 4);
-            const uint32_t acc = (c2 > 0 || k > 0) ? 1u : 0u;
-            if (C::FUSEDN) {          // P [q_hi | q_lo] into two accumulators side by side
-              mma_ts(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
-            } else if (!SPLIT) {      // P (q_hi + q_lo)
-              mma_ts(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
-              mma_ts(tmem + C::COL_R, pl + k * 8, bl, idesc2, 1);
-            } else {                  // P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
-              const uint64_t bl2 = bh + ((2 * C::OPER_BYTES) >> 4);
-              const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
-              mma_ts(tmem + C::COL_R, ph, bh, idesc2, acc);
-              mma_ts(tmem + C::COL_R, ph, bl, idesc2, 1);
-              mma_ts(tmem + C::COL_R, ph, bl2, idesc2, 1);
-              mma_ts(tmem + C::COL_R, plo, bh, idesc2, 1);
-            }
-          }
-          commit(b_empty + 8 * s2);
-          if (c2 == nchunks - 1) {
-            commit(b_rfull);
-            commit(b_wempty + 8 * (int)(tt2 % NWB));
-          }
-          // advance MMA2 state
-          if (++s2 == NSTAGE) s2 = 0;
-          if (++l2 == NB) { l2 = 0; ph_pfull ^= 1u; }
-          if (c2 == 0) ph_rempty ^= 1u;
-          if (++c2 == nchunks) { c2 = 0; ++tt2; }
+        commit_elect(b_empty + 8 * s2);
+        commit_elect(b_lfree + 8 * l2);
+        if (c2 == nchunks - 1) commit_elect(b_rfull);
+        if (++s2 == NSTAGE) s2 = 0;
+        if (++l2 == NB) { l2 = 0; ph_pfull ^= 1u; }
+        if (c2 == 0) ph_rempty ^= 1u;
+        if (++c2 == nchunks) c2 = 0;
+      }
+      commit_elect(b_drain2);
+      if (lane == 0) {
+        const uint64_t t0 = globaltimer_ns();
+        while (!mbar_try_wait(b_drain2, 0) && globaltimer_ns() - t0 < 200000000ull) {
         }
       }
-      // wait until every MMA issued by this thread has completed
-      commit(b_drain);
-      uint64_t t0 = globaltimer_ns();
-      while (!mbar_try_wait(b_drain, 0) && globaltimer_ns() - t0 < 200000000ull) {
-      }
+      __syncwarp();
     }
   } else {
     // ------------------------------------------------------------ epilogue
