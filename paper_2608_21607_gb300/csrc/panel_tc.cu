@@ -59,11 +59,13 @@ struct Cfg {
   // readout): half the MMA instructions of two separate products
   static constexpr bool FUSEDN = !SPLIT && !LOSS && RP <= 128;
   static constexpr int RCOLS = FUSEDN ? 2 * RP : RP;   // TMEM columns of the R accumulator(s)
-  static constexpr int BN = (RP == 256 || (SPLIT && RP == 128) || (FUSEDN && RP == 128)) ? 64 : 128;  // Q rows per chunk
+  // Q rows per chunk.  64 where the TMEM budget would otherwise leave only
+  // two L buffers: more chunks in flight hide the epilogue's latency.
+  static constexpr int BN = (RP == 256 || (SPLIT && RP == 128) || FUSEDN) ? 64 : 128;
   static constexpr int WCOLS = SPLIT ? RP : RP / 2;    // TMEM columns of one W tile (hi [+ lo])
   static constexpr int NWB = (RP == 256) ? 1 : 2;      // W tile buffers
   static constexpr int FREE = 512 - NWB * WCOLS - RCOLS;
-  static constexpr int NB = FREE / BN >= 3 ? 3 : FREE / BN;  // L buffers
+  static constexpr int NB = FREE / BN >= 6 ? 6 : FREE / BN;  // L buffers
   static constexpr int PANEL_W = RP < 64 ? RP : 64;    // elements per row of one swizzle panel
   static constexpr int ROWB = PANEL_W * 2;             // bytes per panel row (= swizzle width)
   static constexpr int PANEL_BYTES = BN * ROWB;
