@@ -2,6 +2,7 @@
 // workspace layout, the block schedule of a sweep and the C ABI of nmd.h.
 #include <math.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <algorithm>
@@ -248,9 +249,14 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
     f->E = c.take<float>(N * rp);
   }
   w->R = c.take<float>(std::max(m, n) * rp);
+  w->R2 = c.take<float>(std::max(m, n) * rp);
+  w->Rs = c.take<float>(std::max(m, n) * rp);
+  w->Rs2 = c.take<float>(std::max(m, n) * rp);
   w->gram_part = c.take<float>((size_t)kGramParts * rp * rp);
   w->G = c.take<float>((size_t)rp * rp);
   w->Ginv = c.take<float>((size_t)rp * rp);
+  w->G2 = c.take<float>((size_t)rp * rp);
+  w->Ginv2 = c.take<float>((size_t)rp * rp);
   w->chol_scratch = c.take<float>((size_t)2 * rp * rp);
   w->seg_partials = c.take<float>((size_t)std::max<int64_t>(maxseg, 1) * rp);
   w->loss_part = c.take<double>((size_t)kLossParts * 8);
@@ -318,6 +324,9 @@ const char* status_name(int s) {
 nmd_status sync_and_check(nmd_handle* h) {
   CK(h, cudaStreamSynchronize(h->stream));
   if (h->side) CK(h, cudaStreamSynchronize(h->side));
+  if (h->aux) CK(h, cudaStreamSynchronize(h->aux));
+  if (h->hp) CK(h, cudaStreamSynchronize(h->hp));
+  h->pend[0].active = h->pend[1].active = false;
   int st[kStatusWords];
   CK(h, cudaMemcpy(st, h->ws.status, sizeof st, cudaMemcpyDeviceToHost));
   if (st[0] != 0) {
@@ -348,7 +357,7 @@ struct TimedScope {
   int cls;
   cudaStream_t st;
   cudaEvent_t a = nullptr, b = nullptr;
-  TimedScope(nmd_handle* h_, int c, cudaStream_t s_ = nullptr) : h(h_), cls(c), st(s_ ? s_ : h_->stream) {
+  TimedScope(nmd_handle* h_, int c, cudaStream_t s_ = nullptr) : h(h_), cls(c), st(s_ ? s_ : h_->cur) {
     if (h->profiling) {
       a = pool_event(h);
       b = pool_event(h);
@@ -363,16 +372,27 @@ struct TimedScope {
   }
 };
 
+// With NMD_TRACE set to a file name, every timed launch is also appended to
+// that file as "class start_ms end_ms", relative to the first launch of the
+// batch (a timeline across the streams).
 void collect_timing(nmd_handle* h) {
+  static const char* names[5] = {"dense", "sparse", "gram", "update", "loss"};
+  const char* path = getenv("NMD_TRACE");
+  FILE* tf = (path && !h->timed.empty()) ? fopen(path, "a") : nullptr;
   for (auto& t : h->timed) {
     float ms = 0.f;
     if (cudaEventElapsedTime(&ms, t.a, t.b) == cudaSuccess) {
       h->prof_ms[t.cls] += ms;
       h->prof_launches[t.cls] += 1;
     }
+    float t0 = 0.f, t1 = 0.f;
+    if (tf && cudaEventElapsedTime(&t0, h->timed[0].a, t.a) == cudaSuccess &&
+        cudaEventElapsedTime(&t1, h->timed[0].a, t.b) == cudaSuccess)
+      fprintf(tf, "%s %.4f %.4f\n", names[t.cls], t0, t1);
     h->event_pool.push_back(t.a);
     h->event_pool.push_back(t.b);
   }
+  if (tf) fclose(tf);
   h->timed.clear();
 }
 
@@ -412,59 +432,137 @@ nmd_status roles(nmd_handle* h, int side, int64_t block, int kind, Roles* R) {
   return NMD_OK;
 }
 
-nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_update) {
+int factor_id(const nmd_handle* h, const Factor* f) { return f == &h->W ? 0 : 1; }
+
+bool overlaps(int64_t x0, int64_t x1, int64_t y0, int64_t y1) { return x0 < y1 && y0 < x1 && x0 < x1 && y0 < y1; }
+
+// Order the main stream after the deferred update of factor f.
+nmd_status wait_pending(nmd_handle* h, int f) {
+  if (h->pend[f].active) {
+    h->pend[f].active = false;
+    CK(h, cudaStreamWaitEvent(h->cur, h->pend[f].ev, 0));
+  }
+  return NMD_OK;
+}
+
+nmd_status wait_all_pending(nmd_handle* h) {
+  nmd_status st = wait_pending(h, 0);
+  if (st == NMD_OK) st = wait_pending(h, 1);
+  return st;
+}
+
+// The step that follows the current one within a sweep (lets the update
+// defer the rows that step does not read).
+struct NextUse {
+  int side;
+  int64_t block;
+  int kind;
+};
+
+nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro, float* R, float* Rs,
+                              const float* Ginv, int64_t lo, int64_t hi, bool momentum, cudaStream_t s) {
+  if (hi <= lo) return NMD_OK;
+  StepArgs sub = a;
+  sub.m0 = ro.m0 + lo;
+  sub.M = hi - lo;
+  TimedScope ts(h, NMD_K_UPDATE, s);
+  launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, Ginv, (float)h->opt.eta, momentum ? (float)h->opt.gamma : 0.f,
+                momentum, h->ws.status, s);
+  h->launches++;
+  return NMD_OK;
+}
+
+nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_update,
+                    const NextUse* next = nullptr) {
   Roles ro;
   nmd_status st = roles(h, side, block, kind, &ro);
   if (st != NMD_OK) return st;
-  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue};
-  cudaStream_t s = h->stream;
-  // Gram G = Q^T Q of the Q-side rows, then Cholesky and G^{-1}
-  // Gram G = Q^T Q of the Q-side rows and G^{-1} on the side stream: only the
-  // update needs them, so they overlap the dense contraction
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms};
+  cudaStream_t s = h->cur;
+  // wait for deferred updates of rows this step reads or writes, and for
+  // those of two steps back (they read the copies of R and G^{-1} reused now)
+  const int fm = factor_id(h, ro.fm), fq = factor_id(h, ro.fq);
+  if ((st = wait_pending(h, fm)) != NMD_OK) return st;
+  const nmd_handle::Pending& pq = h->pend[fq];
+  if (pq.active && (overlaps(ro.q0, ro.q0 + ro.K, pq.a0, pq.a1) || overlaps(ro.q0, ro.q0 + ro.K, pq.b0, pq.b1)))
+    if ((st = wait_pending(h, fq)) != NMD_OK) return st;
+  if (h->pend[fq].active && h->pend[fq].step <= h->step_index - 2)
+    if ((st = wait_pending(h, fq)) != NMD_OK) return st;
+  const int par = (int)(h->step_index & 1);
+  float* R = par ? h->ws.R2 : h->ws.R;
+  float* Rs = par ? h->ws.Rs2 : h->ws.Rs;
+  float* G = par ? h->ws.G2 : h->ws.G;
+  float* Ginv = par ? h->ws.Ginv2 : h->ws.Ginv;
+  h->cur_R = R;
+  h->cur_Rs = Rs;
+  h->cur_G = G;
+  // The side stream computes G = Q^T Q of the Q-side rows, G^{-1}, and the
+  // support term Rs of R; the main stream the dense term of R.  Neither reads
+  // what the other writes, so they overlap; the update joins them.
   int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 255) / 256));
   CK(h, cudaEventRecord(h->ev_fork, s));
   CK(h, cudaStreamWaitEvent(h->side, h->ev_fork, 0));
   {
     TimedScope ts(h, NMD_K_GRAM, h->side);
     launch_gram(*ro.fq, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, h->side);
-    launch_chol_inv(h->ws.gram_part, nparts, h->r, h->rp, (float)h->opt.ridge, h->ws.G, h->ws.Ginv,
-                    h->ws.chol_scratch, h->ws.status, h->side);
+    launch_chol_inv(h->ws.gram_part, nparts, h->r, h->rp, (float)h->opt.ridge, G, Ginv, h->ws.chol_scratch,
+                    h->ws.status, h->side);
     h->launches += 2;
   }
-  CK(h, cudaEventRecord(h->ev_join, h->side));
   if ((st = after_launch(h, "gram/cholesky")) != NMD_OK) return st;
-  // dense Z-panel contraction R = P(L) Q over every (M-side, Q-side) pair
-  {
-    TimedScope ts(h, NMD_K_DENSE);
-    if (h->opt.precision == NMD_SIMT) {
-      launch_panel_simt(a, h->ws.R, s);
-      h->launches++;
-    } else {
-      st = launch_panel_tc(a, h->ws.R, h->ws.status, h->ws.counters, h->num_sms, s, &h->launches);
-    }
-  }
-  if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
-  if ((st = after_launch(h, "dense panel")) != NMD_OK) return st;
   // sparse correction over the block's support
   const PanelSet& P = *ro.P;
   int64_t r0 = P.row_ptr[block], r1 = P.row_ptr[block + 1];
   int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1];
   int64_t u0 = P.multi_ptr[block], u1 = P.multi_ptr[block + 1];
   {
-    TimedScope ts(h, NMD_K_SPARSE);
-    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, g1 - g0, P.d_multi + u0, u1 - u0, ro.qidx, ro.vals,
-                  h->ws.R, h->ws.seg_partials, s);
+    TimedScope ts(h, NMD_K_SPARSE, h->side);
+    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, g1 - g0, P.d_multi + u0, u1 - u0, ro.qidx, ro.vals, Rs,
+                  h->ws.seg_partials, h->side);
     h->launches += (r1 > r0) + 2 * (g1 > g0);
   }
   if ((st = after_launch(h, "sparse correction")) != NMD_OK) return st;
+  CK(h, cudaEventRecord(h->ev_join, h->side));
+  // dense Z-panel contraction R = P(L) Q over every (M-side, Q-side) pair
+  {
+    TimedScope ts(h, NMD_K_DENSE);
+    if (h->opt.precision == NMD_SIMT) {
+      launch_panel_simt(a, R, s);
+      h->launches++;
+    } else {
+      st = launch_panel_tc(a, R, h->ws.status, h->ws.counters, h->num_sms, s, &h->launches);
+    }
+  }
+  if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
+  if ((st = after_launch(h, "dense panel")) != NMD_OK) return st;
   CK(h, cudaStreamWaitEvent(s, h->ev_join, 0));
   if (do_update) {
-    bool momentum = kind == NMD_STOCH;
-    {
-      TimedScope ts(h, NMD_K_UPDATE);
-      launch_update(a, h->ws.R, h->ws.Ginv, (float)h->opt.eta, momentum ? (float)h->opt.gamma : 0.f,
-                    momentum, h->ws.status, s);
-      h->launches++;
+    const bool momentum = kind == NMD_STOCH;
+    // rows [lo, hi) (relative to m0) are updated on the main stream; when the
+    // next step reads only these rows of this factor and writes the other
+    // factor, the rest are updated on the aux stream, overlapping it
+    int64_t lo = 0, hi = ro.M;
+    if (next) {
+      Roles rn;
+      if (roles(h, next->side, next->block, next->kind, &rn) == NMD_OK && rn.fq == ro.fm && rn.fm != ro.fm) {
+        lo = std::min(std::max(rn.q0 - ro.m0, (int64_t)0), ro.M);
+        hi = std::max(std::min(rn.q0 + rn.K - ro.m0, ro.M), lo);
+      }
+    }
+    if ((st = launch_update_rows(h, a, ro, R, Rs, Ginv, lo, hi, momentum, s)) != NMD_OK) return st;
+    if (lo > 0 || hi < ro.M) {
+      CK(h, cudaEventRecord(h->ev_prio, s));
+      CK(h, cudaStreamWaitEvent(h->aux, h->ev_prio, 0));
+      if ((st = launch_update_rows(h, a, ro, R, Rs, Ginv, 0, lo, momentum, h->aux)) != NMD_OK) return st;
+      if ((st = launch_update_rows(h, a, ro, R, Rs, Ginv, hi, ro.M, momentum, h->aux)) != NMD_OK) return st;
+      nmd_handle::Pending& pm = h->pend[fm];
+      CK(h, cudaEventRecord(pm.ev, h->aux));
+      pm.active = true;
+      pm.step = h->step_index;
+      pm.a0 = ro.m0;
+      pm.a1 = ro.m0 + lo;
+      pm.b0 = ro.m0 + hi;
+      pm.b1 = ro.m0 + ro.M;
     }
     if ((st = after_launch(h, "update")) != NMD_OK) return st;
   }
@@ -476,6 +574,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
 
 nmd_handle::~nmd_handle() {
   if (side) cudaStreamSynchronize(side);
+  if (aux) cudaStreamSynchronize(aux);
   if (!timed.empty()) cudaStreamSynchronize(stream);
   for (auto& t : timed) {
     cudaEventDestroy(t.a);
@@ -485,6 +584,16 @@ nmd_handle::~nmd_handle() {
   if (ev_fork) cudaEventDestroy(ev_fork);
   if (ev_join) cudaEventDestroy(ev_join);
   if (side) cudaStreamDestroy(side);
+  if (ev_prio) cudaEventDestroy(ev_prio);
+  for (auto& p : pend)
+    if (p.ev) cudaEventDestroy(p.ev);
+  if (aux) cudaStreamDestroy(aux);
+  if (hp) {
+    cudaStreamSynchronize(hp);
+    cudaStreamDestroy(hp);
+  }
+  if (ev_in) cudaEventDestroy(ev_in);
+  if (ev_out) cudaEventDestroy(ev_out);
 }
 
 // ===========================================================================
@@ -553,6 +662,7 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   h->nnz = (int64_t)S.col.size();
   h->opt = *opts;
   h->stream = (cudaStream_t)stream;
+  h->cur = h->stream;
   h->s_fro = S.s_fro;
   build_panels(S, h->opt, h->panels);
   Carver c(d_workspace);
@@ -612,11 +722,21 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
     if (e == cudaSuccess) e = cudaMemsetAsync(f->E, 0, f->rows * h->rp * 4, s);
     if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("memset: ") + cudaGetErrorString(e));
   }
-  e = cudaStreamCreateWithFlags(&h->side, cudaStreamNonBlocking);
+  int least = 0, greatest = 0;
+  e = cudaDeviceGetStreamPriorityRange(&least, &greatest);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side, cudaStreamNonBlocking, greatest);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->hp, cudaStreamNonBlocking, greatest);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->aux, cudaStreamNonBlocking, least);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_in, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_prio, cudaEventDisableTiming);
+  for (int f = 0; f < 2 && e == cudaSuccess; ++f) e = cudaEventCreateWithFlags(&h->pend[f].ev, cudaEventDisableTiming);
   if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("side stream: ") + cudaGetErrorString(e));
   e = cudaMemsetAsync(h->ws.status, 0, kStatusWords * sizeof(int), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->ws.Rs, 0, std::max(m, n) * h->rp * sizeof(float), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(h->ws.Rs2, 0, std::max(m, n) * h->rp * sizeof(float), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(h->ws.counters, 0, 64 * sizeof(int), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return bail(NMD_ERR_CUDA, std::string("create: ") + cudaGetErrorString(e));
@@ -682,19 +802,33 @@ nmd_status nmd_sweep(nmd_handle* h) {
   int64_t Kr = nblocks(h->m, h->opt.block_rows), Kc = nblocks(h->n, h->opt.block_cols);
   std::vector<int64_t> pr = permutation(h->opt.seed, h->sweep_index, NMD_ROW, Kr);
   std::vector<int64_t> pc = permutation(h->opt.seed, h->sweep_index, NMD_COL, Kc);
-  nmd_status st = NMD_OK;
+  // the sweep's steps in order, so that each update knows the step after it
+  std::vector<NextUse> steps;
   if (h->opt.schedule == NMD_EXACT) {
-    for (int64_t t = 0; t < Kr && st == NMD_OK; ++t) st = run_step(h, NMD_ROW, pr[t], NMD_EXACT, true);
-    for (int64_t t = 0; t < Kc && st == NMD_OK; ++t) st = run_step(h, NMD_COL, pc[t], NMD_EXACT, true);
+    for (int64_t t = 0; t < Kr; ++t) steps.push_back({NMD_ROW, pr[t], NMD_EXACT});
+    for (int64_t t = 0; t < Kc; ++t) steps.push_back({NMD_COL, pc[t], NMD_EXACT});
   } else if (h->opt.order == NMD_PHASED) {
-    for (int64_t t = 0; t < Kc && st == NMD_OK; ++t) st = run_step(h, NMD_COL, pc[t], NMD_STOCH, true);
-    for (int64_t t = 0; t < Kr && st == NMD_OK; ++t) st = run_step(h, NMD_ROW, pr[t], NMD_STOCH, true);
+    for (int64_t t = 0; t < Kc; ++t) steps.push_back({NMD_COL, pc[t], NMD_STOCH});
+    for (int64_t t = 0; t < Kr; ++t) steps.push_back({NMD_ROW, pr[t], NMD_STOCH});
   } else {
-    for (int64_t t = 0; t < std::max(Kr, Kc) && st == NMD_OK; ++t) {
-      if (t < Kc) st = run_step(h, NMD_COL, pc[t], NMD_STOCH, true);
-      if (st == NMD_OK && t < Kr) st = run_step(h, NMD_ROW, pr[t], NMD_STOCH, true);
+    for (int64_t t = 0; t < std::max(Kr, Kc); ++t) {
+      if (t < Kc) steps.push_back({NMD_COL, pc[t], NMD_STOCH});
+      if (t < Kr) steps.push_back({NMD_ROW, pr[t], NMD_STOCH});
     }
   }
+  CK(h, cudaEventRecord(h->ev_in, h->stream));
+  CK(h, cudaStreamWaitEvent(h->hp, h->ev_in, 0));
+  h->cur = h->hp;
+  nmd_status st = NMD_OK;
+  for (size_t t = 0; t < steps.size() && st == NMD_OK; ++t)
+    st = run_step(h, steps[t].side, steps[t].block, steps[t].kind, true,
+                  t + 1 < steps.size() ? &steps[t + 1] : nullptr);
+  // `stream` continues after every kernel of the sweep, deferred ones included
+  nmd_status st2 = wait_all_pending(h);
+  h->cur = h->stream;
+  if (st == NMD_OK) st = st2;
+  CK(h, cudaEventRecord(h->ev_out, h->hp));
+  CK(h, cudaStreamWaitEvent(h->stream, h->ev_out, 0));
   if (st == NMD_OK) h->sweep_index++;
   return st;
 }
@@ -752,11 +886,14 @@ nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t k
   if (st != NMD_OK) return st;
   if ((st = run_step(h, side, block, kind, false)) != NMD_OK) return st;
   h->step_index--;
+  launch_combine(h->cur_R, h->cur_Rs, ro.M * h->rp, h->cur);
+  h->launches++;
+  if ((st = after_launch(h, "combine")) != NMD_OK) return st;
   if ((st = sync_and_check(h)) != NMD_OK) return st;
   if (rows) *rows = ro.M;
   cudaStream_t s = h->stream;
-  if (R) CK(h, cudaMemcpy2DAsync(R, h->r * 4, h->ws.R, h->rp * 4, h->r * 4, ro.M, cudaMemcpyDeviceToHost, s));
-  if (G) CK(h, cudaMemcpy2DAsync(G, h->r * 4, h->ws.G, h->rp * 4, h->r * 4, h->r, cudaMemcpyDeviceToHost, s));
+  if (R) CK(h, cudaMemcpy2DAsync(R, h->r * 4, h->cur_R, h->rp * 4, h->r * 4, ro.M, cudaMemcpyDeviceToHost, s));
+  if (G) CK(h, cudaMemcpy2DAsync(G, h->r * 4, h->cur_G, h->rp * 4, h->r * 4, h->r, cudaMemcpyDeviceToHost, s));
   CK(h, cudaStreamSynchronize(s));
   return NMD_OK;
 }
@@ -768,7 +905,7 @@ nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_
   nmd_status st = roles(h, side, block, kind, &ro);
   if (st != NMD_OK) return st;
   if (h->opt.precision == NMD_SIMT) return fail(h, NMD_ERR_UNSUPPORTED, "dense products hook needs a tensor-core precision");
-  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue};
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms};
   st = launch_panel_tc(a, h->ws.R, h->ws.status, h->ws.counters, h->num_sms, h->stream, &h->launches, d_L);
   if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
   if ((st = after_launch(h, "dense products")) != NMD_OK) return st;

@@ -193,17 +193,95 @@ __global__ void __launch_bounds__(T * T) ginv_kernel(const float* __restrict__ p
     }
 }
 
+// Register-resident variant for rp <= 128: thread t owns row t / 4 and the
+// rp / 4 contiguous columns (t % 4) rp / 4 ... of it.  Before pivot k the
+// owners of row k publish it to shared memory (two alternating buffers, one
+// barrier per pivot); every thread then updates its own entries from that
+// row alone, using the symmetry a_ik = a_ki.  Each update is written so that
+// (i, j) and (j, i) round identically (the product a_ik a_kj is formed
+// before the division), so the matrix stays exactly symmetric.  The partial
+// Gram matrices are summed in part order first.
+template <int RP>
+__global__ void __launch_bounds__(RP * 4) ginv_reg_kernel(const float* __restrict__ parts, int nparts, int r,
+                                                          float ridge, float* __restrict__ Gout,
+                                                          float* __restrict__ Ginv, int* __restrict__ status) {
+  constexpr int CPT = RP / 4;
+  __shared__ __align__(16) float rk[2][RP];
+  __shared__ float diag0[RP];
+  const int i = threadIdx.x / 4, c0 = (threadIdx.x % 4) * CPT;
+  // the partials hold the entries whose 64-row tile is >= their 64-column tile
+  const bool direct = (i / 64) >= (c0 / 64);
+  float a[CPT];
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) a[j] = 0.f;
+  for (int p = 0; p < nparts; ++p) {
+    const float* src = parts + (size_t)p * RP * RP;
+    if (direct) {
+#pragma unroll
+      for (int j = 0; j < CPT; j += 4) {
+        const float4 v = __ldg((const float4*)(src + i * RP + c0 + j));
+        a[j] += v.x; a[j + 1] += v.y; a[j + 2] += v.z; a[j + 3] += v.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) a[j] += __ldg(src + (c0 + j) * RP + i);
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < CPT; ++j)
+    if (c0 + j == i && i < r) {
+      a[j] += ridge;
+      diag0[i] = a[j];
+    }
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) Gout[i * RP + c0 + j] = (i < r && c0 + j < r) ? a[j] : 0.f;
+  const float tol = 4.0f * (float)r * FLT_EPSILON;
+  bool bad = false;
+  for (int k = 0; k < r; ++k) {
+    float* rb = rk[k & 1];
+    if (i == k) {
+#pragma unroll
+      for (int j = 0; j < CPT; j += 4) *(float4*)(rb + c0 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
+    }
+    __syncthreads();
+    const float d = rb[k];
+    if (!(d > tol * diag0[k]) || !isfinite(d)) {   // uniform: every thread read the same d
+      bad = true;
+      if (threadIdx.x == 0) set_status(status, NMD_ERR_NOT_SPD, k, 0);
+      break;
+    }
+    const float inv = 1.0f / d;
+    if (i == k) {
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) a[j] = (c0 + j == k) ? -inv : a[j] * inv;
+    } else {
+      const float ri = rb[i];
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) {
+        const float rj = rb[c0 + j];
+        a[j] = (c0 + j == k) ? ri * inv : fmaf(-(ri * rj), inv, a[j]);
+      }
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) Ginv[i * RP + c0 + j] = (!bad && i < r && c0 + j < r) ? -a[j] : 0.f;
+}
+
 // ---------------------------------------------------------------------------
 // Sparse correction: for every panel row i and entry (i, k) in the block,
 // L_ik = m_i . q_k, c = S_ik - min(0, L_ik), R_i += c q_k (fp32 masters).
 // One warp per panel row or per segment of at most kSeg entries; the lanes
-// first fetch the entries' indices and values (one per lane), then four
-// entries at a time are processed with their q rows in flight together.
-// Single rows add into R directly (one writer per row); segments of long
-// rows write a partial sum to their slot and a second pass adds the slots
-// of each row in a fixed order.
+// first fetch the entries' indices and values (one per lane), then NE
+// entries at a time (4 for single rows, which are mostly short; 8 for the
+// full segments of long rows) are processed with their q rows in flight
+// together; the accumulation order over the entries stays ascending.
+// The result goes to Rs, the support term of R, which holds zeros on every
+// other row (the update consumes it and clears it): single rows write their
+// row of Rs directly (one writer per row); segments of long rows write a
+// partial sum to their slot and a second pass adds the slots of each row in
+// a fixed order and writes the sum.
 // ---------------------------------------------------------------------------
-template <int VPL>
+template <int VPL, int NE>
 __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __restrict__ rows, int64_t nrows,
                                                           const float* __restrict__ Mop, int64_t m0,
                                                           const float* __restrict__ Qop,
@@ -229,11 +307,11 @@ __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __rest
     mv[v] = c < rp ? __ldg(Mop + i * rp + c) : 0.f;
     acc[v] = 0.f;
   }
-  for (int e = 0; e < pr.len; e += 4) {
-    float qv[4][VPL], part[4];
-    float sv[4];
+  for (int e = 0; e < pr.len; e += NE) {
+    float qv[NE][VPL], part[NE];
+    float sv[NE];
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < NE; ++j) {
       const int k = __shfl_sync(0xffffffffu, kl, (e + j) & 31);
       sv[j] = __shfl_sync(0xffffffffu, sl, (e + j) & 31);
       const bool live = e + j < pr.len;
@@ -248,9 +326,9 @@ __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __rest
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1)
 #pragma unroll
-      for (int j = 0; j < 4; ++j) part[j] += __shfl_xor_sync(0xffffffffu, part[j], o);
+      for (int j = 0; j < NE; ++j) part[j] += __shfl_xor_sync(0xffffffffu, part[j], o);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < NE; ++j) {
       const float cval = sv[j] - fminf(0.f, part[j]);        // zero for the padding entries (q = 0)
 #pragma unroll
       for (int v = 0; v < VPL; ++v) acc[v] = fmaf(cval, qv[j][v], acc[v]);
@@ -260,28 +338,36 @@ __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __rest
 #pragma unroll
   for (int v = 0; v < VPL; ++v) {
     const int c = lane + 32 * v;
-    if (c < rp) dst[c] = partials ? acc[v] : dst[c] + acc[v];
+    if (c < rp) dst[c] = acc[v];
   }
 }
 
-// R_i += sum of the segment slots of row i, in slot order.
-__global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __restrict__ multi, int64_t nmulti,
+// Rs_i = sum of the segment slots of row i.  One block per long row: thread
+// t handles column t % RP of the slots g, g + G, g + 2G, ... (g = t / RP,
+// G = 256 / RP groups) with eight loads in flight, and the G group sums are
+// added in group order, so the result is the same on every run.
+template <int RP>
+__global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __restrict__ multi,
                                                             const float* __restrict__ partials,
-                                                            float* __restrict__ R, int64_t m0, int rp) {
-  const int lane = threadIdx.x & 31;
-  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-  if (w >= nmulti) return;
-  const PanelRow mr = multi[w];
-  for (int c = lane; c < rp; c += 32) {
-    // eight independent loads in flight, combined in a fixed order
-    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    int q = 0;
-    for (; q + 8 <= mr.len; q += 8)
+                                                            float* __restrict__ R, int64_t m0) {
+  constexpr int G = 256 / RP;
+  __shared__ float gsum[256];
+  const PanelRow mr = multi[blockIdx.x];
+  const int c = threadIdx.x % RP, g = threadIdx.x / RP;
+  const float* src = partials + mr.beg * RP + c;
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  int q = g;
+  for (; q + 7 * G < mr.len; q += 8 * G)
 #pragma unroll
-      for (int u = 0; u < 8; ++u) acc[u] += __ldg(partials + (mr.beg + q + u) * rp + c);
-    for (; q < mr.len; ++q) acc[0] += __ldg(partials + (mr.beg + q) * rp + c);
-    const float s = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
-    R[(mr.row - m0) * rp + c] += s;
+    for (int u = 0; u < 8; ++u) acc[u] += __ldg(src + (int64_t)(q + u * G) * RP);
+  for (; q < mr.len; q += G) acc[0] += __ldg(src + (int64_t)q * RP);
+  gsum[threadIdx.x] = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+  __syncthreads();
+  if (g == 0) {
+    float v = gsum[c];
+#pragma unroll
+    for (int k = 1; k < G; ++k) v += gsum[k * RP + c];
+    R[(mr.row - m0) * RP + c] = v;
   }
 }
 
@@ -290,118 +376,217 @@ __global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __re
 //   Z form:     U = eta (X - M)      (eqs. lsqA/lsqB with step size)
 //   Delta form: U = eta X            (eqs. spLsqA/spLsqB)
 // then E = U + gamma E (stochastic steps) and M += E, refreshing the bf16
-// pieces.  Skipped entirely while a sticky error is set.
-// X = R G^{-1} is a small GEMM per tile of 64 rows: a block keeps CW columns
-// of G^{-1} in shared memory, stages the tile's R transposed (k-major), and
-// thread (ty, tx) of 16 x 16 computes rows 4 ty .. 4 ty + 3 and columns
-// CPT tx .. CPT tx + CPT - 1 (CPT = CW / 16) with 128-bit shared loads, then
-// applies the elementwise update to those entries.
+// pieces (the third piece only where the fp32-accurate mode reads it).
+// Skipped entirely while a sticky error is set.
+// X = R G^{-1} is a small GEMM per tile of TR rows.  A block keeps CW columns
+// of G^{-1} in shared memory; the tile's R rows (contiguous in global memory)
+// are copied into a double buffer with cp.async one tile ahead, and each
+// thread's M and E entries are loaded into registers before the product, so
+// the memory latency of both overlaps the arithmetic.  Thread (ty, tx) owns
+// rows 4 ty .. 4 ty + 3 and CPT columns: for CPT >= 4 the groups of four
+// columns 4 tx + 4 TX g (g < CPT / 4), so that a quarter warp reads 128
+// contiguous bytes of G^{-1} and a half warp writes whole 256-byte rows.
 // ---------------------------------------------------------------------------
+template <int RP>
+struct UpdCfg {
+  static constexpr int CW = RP <= 128 ? RP : 128;   // output columns per block
+  static constexpr int TR = RP <= 128 ? 64 : 32;    // rows per tile
+  static constexpr int TY = TR / 4;                  // row groups of four
+  static constexpr int TX = 256 / TY;                // column groups
+  static constexpr int CPT = CW / TX;                // columns per thread (1, 2, 4 or 8)
+  static constexpr size_t SMEM = ((size_t)RP * CW + 2 * (size_t)TR * RP) * sizeof(float);
+  static_assert(CPT >= 1 && (CPT < 4 || CPT % 4 == 0), "column split");
+};
+
+template <int CPT, int TX>
+__device__ __forceinline__ int upd_col(int tx, int j) {
+  if (CPT >= 4) return (j / 4) * 4 * TX + 4 * tx + (j % 4);
+  return CPT * tx + j;
+}
+
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem_dst)),
+               "l"(gsrc)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
 template <int RP>
 __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
                                                      bf16* __restrict__ Mlo, bf16* __restrict__ Mlo2,
                                                      float* __restrict__ E, int64_t m0, int64_t rows,
-                                                     const float* __restrict__ R,
+                                                     const float* __restrict__ R, float* __restrict__ Rs,
                                                      const float* __restrict__ Ginv, float eta,
-                                                     float gamma, int momentum, int delta_form,
+                                                     float gamma, int momentum, int delta_form, int write_lo2,
                                                      int* __restrict__ status) {
-  constexpr int CW = RP <= 128 ? RP : 128;    // output columns handled by this block
-  constexpr int CPT = CW / 16;                // columns per thread (1, 2, 4 or 8)
-  constexpr int TR = 64;                      // rows per tile
-  constexpr int LDR = TR + 4;                 // row stride of the transposed R tile
-  extern __shared__ float sm[];
-  float* Gs = sm;                             // RP x CW
-  float* Rt = sm + RP * CW;                   // RP x LDR: Rt[k * LDR + row] = R[row][k]
+  using C = UpdCfg<RP>;
+  constexpr int NV = C::TR * RP / 4 / 256;   // float4 of a tile per thread
+  constexpr int CW = C::CW, TR = C::TR, TX = C::TX, CPT = C::CPT;
+  extern __shared__ __align__(16) float sm[];
+  float* Gs = sm;                               // RP x CW
+  float* Rb = sm + RP * CW;                     // 2 x TR x RP, row-major like R
   if (*(volatile int*)status != 0) return;
   const int cw0 = blockIdx.y * CW;
-  for (int e = threadIdx.x; e < RP * CW; e += blockDim.x) Gs[e] = Ginv[(e / CW) * RP + cw0 + (e % CW)];
-  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
-  for (int64_t base = (int64_t)blockIdx.x * TR; base < rows; base += (int64_t)gridDim.x * TR) {
-    __syncthreads();
-    for (int e = threadIdx.x; e < TR * (RP / 4); e += blockDim.x) {
-      const int rr = e / (RP / 4), k4 = 4 * (e % (RP / 4));
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (base + rr < rows) v = *(const float4*)(R + (base + rr) * RP + k4);
-      Rt[(k4 + 0) * LDR + rr] = v.x;
-      Rt[(k4 + 1) * LDR + rr] = v.y;
-      Rt[(k4 + 2) * LDR + rr] = v.z;
-      Rt[(k4 + 3) * LDR + rr] = v.w;
+  const int tx = threadIdx.x % TX, ty = threadIdx.x / TX;
+  const int64_t ntiles = (rows + TR - 1) / TR;
+  const int64_t total = rows * RP;              // floats of R in this step
+  auto issue = [&](int64_t tile, int buf) {
+    const int64_t base = tile * TR * RP;
+    float* dst = Rb + buf * TR * RP;
+#pragma unroll
+    for (int u = 0; u < NV; ++u) {
+      const int e = threadIdx.x + 256 * u;
+      if (base + 4 * e < total) cp_async16(dst + 4 * e, R + base + 4 * e);
+    }
+  };
+  int64_t t = blockIdx.x;
+  if (t < ntiles) issue(t, 0);
+  cp_async_commit();
+  for (int e = threadIdx.x; e < RP * CW; e += 256) Gs[e] = Ginv[(e / CW) * RP + cw0 + (e % CW)];
+  int buf = 0;
+  for (; t < ntiles; t += gridDim.x, buf ^= 1) {
+    if (t + gridDim.x < ntiles) issue(t + gridDim.x, buf ^ 1);
+    cp_async_commit();
+    const int64_t base = t * TR;
+    // the support term of this tile, taken from Rs (which is left zero)
+    float4 sv[NV];
+#pragma unroll
+    for (int u = 0; u < NV; ++u) {
+      const int64_t o = base * RP + 4 * (threadIdx.x + 256 * u);
+      sv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (o < total) sv[u] = *(const float4*)(Rs + o);
+    }
+    // this thread's M and E entries, in flight during the product
+    float mo[4][CPT], eo[4][CPT];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int64_t li = base + 4 * ty + i;
+      const bool live = li < rows;
+      const float* mrow = M + (m0 + li) * RP + cw0;
+      const float* erow = E + (m0 + li) * RP + cw0;
+      if (CPT >= 4) {
+#pragma unroll
+        for (int j = 0; j < CPT; j += 4) {
+          const int c = upd_col<CPT, TX>(tx, j);
+          float4 v = make_float4(0.f, 0.f, 0.f, 0.f), w = v;
+          if (live) {
+            v = *(const float4*)(mrow + c);
+            if (momentum) w = *(const float4*)(erow + c);
+          }
+          mo[i][j] = v.x; mo[i][j + 1] = v.y; mo[i][j + 2] = v.z; mo[i][j + 3] = v.w;
+          eo[i][j] = w.x; eo[i][j + 1] = w.y; eo[i][j + 2] = w.z; eo[i][j + 3] = w.w;
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) {
+          const int c = upd_col<CPT, TX>(tx, j);
+          mo[i][j] = live ? mrow[c] : 0.f;
+          eo[i][j] = (live && momentum) ? erow[c] : 0.f;
+        }
+      }
+    }
+    cp_async_wait_1();
+    // add the support term to the entries this thread copied (its own copies
+    // have landed), clear Rs there (when one block covers all columns of the
+    // tile; otherwise the launcher clears it afterwards), then publish
+#pragma unroll
+    for (int u = 0; u < NV; ++u) {
+      const int e = threadIdx.x + 256 * u;
+      const int64_t o = base * RP + 4 * e;
+      if (o < total) {
+        float4* d = (float4*)(Rb + buf * TR * RP + 4 * e);
+        float4 v = *d;
+        v.x += sv[u].x; v.y += sv[u].y; v.z += sv[u].z; v.w += sv[u].w;
+        *d = v;
+        if (gridDim.y == 1) *(float4*)(Rs + o) = make_float4(0.f, 0.f, 0.f, 0.f);
+      }
     }
     __syncthreads();
+    const float* Rt = Rb + buf * TR * RP + (4 * ty) * RP;
     float x[4][CPT];
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
       for (int j = 0; j < CPT; ++j) x[i][j] = 0.f;
-#pragma unroll 4
-    for (int k = 0; k < RP; ++k) {
-      const float4 a = *(const float4*)(Rt + k * LDR + 4 * ty);
-      float b[CPT];
-      if (CPT >= 4) {
+#pragma unroll 2
+    for (int k = 0; k < RP; k += 4) {
+      float4 a[4];
 #pragma unroll
-        for (int j = 0; j < CPT; j += 4) {
-          const float4 g = *(const float4*)(Gs + k * CW + CPT * tx + j);
-          b[j] = g.x; b[j + 1] = g.y; b[j + 2] = g.z; b[j + 3] = g.w;
+      for (int i = 0; i < 4; ++i) a[i] = *(const float4*)(Rt + i * RP + k);
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        float b[CPT];
+        const float* grow = Gs + (k + kk) * CW;
+        if (CPT >= 4) {
+#pragma unroll
+          for (int j = 0; j < CPT; j += 4) {
+            const float4 g = *(const float4*)(grow + upd_col<CPT, TX>(tx, j));
+            b[j] = g.x; b[j + 1] = g.y; b[j + 2] = g.z; b[j + 3] = g.w;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < CPT; ++j) b[j] = grow[upd_col<CPT, TX>(tx, j)];
         }
-      } else {
 #pragma unroll
-        for (int j = 0; j < CPT; ++j) b[j] = Gs[k * CW + CPT * tx + j];
-      }
+        for (int i = 0; i < 4; ++i) {
+          const float av = kk == 0 ? a[i].x : kk == 1 ? a[i].y : kk == 2 ? a[i].z : a[i].w;
 #pragma unroll
-      for (int j = 0; j < CPT; ++j) {
-        x[0][j] = fmaf(a.x, b[j], x[0][j]);
-        x[1][j] = fmaf(a.y, b[j], x[1][j]);
-        x[2][j] = fmaf(a.z, b[j], x[2][j]);
-        x[3][j] = fmaf(a.w, b[j], x[3][j]);
+          for (int j = 0; j < CPT; ++j) x[i][j] = fmaf(av, b[j], x[i][j]);
+        }
       }
     }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int64_t li = base + 4 * ty + i;
       if (li >= rows) break;
-      const int64_t g = (m0 + li) * RP + cw0 + CPT * tx;
+      const int64_t g = (m0 + li) * RP + cw0;
       bool finite = true;
-      if (CPT == 1) {
-        const float mo = M[g];
-        const float eo = momentum ? E[g] : 0.f;
-        const float u = delta_form ? eta * x[i][0] : eta * (x[i][0] - mo);
-        const float e = momentum ? fmaf(gamma, eo, u) : u;
-        const float nv = mo + e;
-        finite = isfinite(nv);
-        M[g] = nv;
-        if (momentum) E[g] = e;
-        const bf16 h = __float2bfloat16_rn(nv);
-        const float r1 = nv - __bfloat162float(h);
-        const bf16 l = __float2bfloat16_rn(r1);
-        Mhi[g] = h;
-        Mlo[g] = l;
-        Mlo2[g] = __float2bfloat16_rn(r1 - __bfloat162float(l));
-      }
+      float nv[CPT], ev[CPT];
 #pragma unroll
-      for (int j = 0; j + 1 < CPT; j += 2) {
-        const float2 mo = *(const float2*)(M + g + j);
-        float2 eo = make_float2(0.f, 0.f);
-        if (momentum) eo = *(const float2*)(E + g + j);
-        const float u0 = delta_form ? eta * x[i][j] : eta * (x[i][j] - mo.x);
-        const float u1 = delta_form ? eta * x[i][j + 1] : eta * (x[i][j + 1] - mo.y);
-        const float e0 = momentum ? fmaf(gamma, eo.x, u0) : u0;
-        const float e1 = momentum ? fmaf(gamma, eo.y, u1) : u1;
-        const float n0 = mo.x + e0, n1 = mo.y + e1;
-        finite = finite && isfinite(n0) && isfinite(n1);
-        *(float2*)(M + g + j) = make_float2(n0, n1);
-        if (momentum) *(float2*)(E + g + j) = make_float2(e0, e1);
-        const bf16 h0 = __float2bfloat16_rn(n0), h1 = __float2bfloat16_rn(n1);
-        const float r0 = n0 - __bfloat162float(h0), r1 = n1 - __bfloat162float(h1);
-        const bf16 l0 = __float2bfloat16_rn(r0), l1 = __float2bfloat16_rn(r1);
-        const bf16 q0 = __float2bfloat16_rn(r0 - __bfloat162float(l0));
-        const bf16 q1 = __float2bfloat16_rn(r1 - __bfloat162float(l1));
-        *(uint32_t*)(Mhi + g + j) = (uint32_t)__bfloat16_as_ushort(h0) | ((uint32_t)__bfloat16_as_ushort(h1) << 16);
-        *(uint32_t*)(Mlo + g + j) = (uint32_t)__bfloat16_as_ushort(l0) | ((uint32_t)__bfloat16_as_ushort(l1) << 16);
-        *(uint32_t*)(Mlo2 + g + j) = (uint32_t)__bfloat16_as_ushort(q0) | ((uint32_t)__bfloat16_as_ushort(q1) << 16);
+      for (int j = 0; j < CPT; ++j) {
+        const float u = delta_form ? eta * x[i][j] : eta * (x[i][j] - mo[i][j]);
+        ev[j] = momentum ? fmaf(gamma, eo[i][j], u) : u;
+        nv[j] = mo[i][j] + ev[j];
+        finite = finite && isfinite(nv[j]);
+      }
+      uint32_t hw[CPT], lw[CPT], l2w[CPT];
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) {
+        const bf16 h = __float2bfloat16_rn(nv[j]);
+        const float r1 = nv[j] - __bfloat162float(h);
+        const bf16 l = __float2bfloat16_rn(r1);
+        hw[j] = __bfloat16_as_ushort(h);
+        lw[j] = __bfloat16_as_ushort(l);
+        l2w[j] = __bfloat16_as_ushort(__float2bfloat16_rn(r1 - __bfloat162float(l)));
+      }
+      if (CPT >= 4) {
+#pragma unroll
+        for (int j = 0; j < CPT; j += 4) {
+          const int c = upd_col<CPT, TX>(tx, j);
+          *(float4*)(M + g + c) = make_float4(nv[j], nv[j + 1], nv[j + 2], nv[j + 3]);
+          if (momentum) *(float4*)(E + g + c) = make_float4(ev[j], ev[j + 1], ev[j + 2], ev[j + 3]);
+          *(uint2*)(Mhi + g + c) = make_uint2(hw[j] | (hw[j + 1] << 16), hw[j + 2] | (hw[j + 3] << 16));
+          *(uint2*)(Mlo + g + c) = make_uint2(lw[j] | (lw[j + 1] << 16), lw[j + 2] | (lw[j + 3] << 16));
+          if (write_lo2)
+            *(uint2*)(Mlo2 + g + c) = make_uint2(l2w[j] | (l2w[j + 1] << 16), l2w[j + 2] | (l2w[j + 3] << 16));
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) {
+          const int c = upd_col<CPT, TX>(tx, j);
+          M[g + c] = nv[j];
+          if (momentum) E[g + c] = ev[j];
+          Mhi[g + c] = __ushort_as_bfloat16((unsigned short)hw[j]);
+          Mlo[g + c] = __ushort_as_bfloat16((unsigned short)lw[j]);
+          if (write_lo2) Mlo2[g + c] = __ushort_as_bfloat16((unsigned short)l2w[j]);
+        }
       }
       if (!finite) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
     }
+    __syncthreads();   // the buffer read above is refilled by the next iteration's copy
   }
+  asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 template <typename T>
@@ -547,8 +732,13 @@ void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge,
                      float* scratch, int* status, cudaStream_t s) {
   const size_t smem = (size_t)r * r * sizeof(float);
   const int use_smem = smem <= 200 * 1024;
-  if (r <= 64) {
-    ginv_kernel<16><<<1, 256, smem, s>>>(parts, nparts, r, rp, ridge, G, Ginv, scratch, status, 1);
+  if (rp <= 128) {
+    switch (rp) {
+      case 16: ginv_reg_kernel<16><<<1, 64, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
+      case 32: ginv_reg_kernel<32><<<1, 128, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
+      case 64: ginv_reg_kernel<64><<<1, 256, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
+      default: ginv_reg_kernel<128><<<1, 512, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
+    }
   } else {
     static bool attr = false;
     if (!attr) {
@@ -557,6 +747,18 @@ void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge,
     }
     ginv_kernel<32><<<1, 1024, use_smem ? smem : 0, s>>>(parts, nparts, r, rp, ridge, G, Ginv, scratch, status,
                                                          use_smem);
+  }
+}
+
+static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* partials, float* R, int64_t m0, int rp,
+                          cudaStream_t s) {
+  const unsigned grid = (unsigned)nmulti;
+  switch (rp) {
+    case 16: sparse_reduce_kernel<16><<<grid, 256, 0, s>>>(multi, partials, R, m0); break;
+    case 32: sparse_reduce_kernel<32><<<grid, 256, 0, s>>>(multi, partials, R, m0); break;
+    case 64: sparse_reduce_kernel<64><<<grid, 256, 0, s>>>(multi, partials, R, m0); break;
+    case 128: sparse_reduce_kernel<128><<<grid, 256, 0, s>>>(multi, partials, R, m0); break;
+    default: sparse_reduce_kernel<256><<<grid, 256, 0, s>>>(multi, partials, R, m0); break;
   }
 }
 
@@ -572,13 +774,12 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
 #define NMD_SP(V)                                                                                           \
   do {                                                                                                      \
     if (nrows > 0)                                                                                          \
-      sparse_rows_kernel<V><<<(unsigned)((nrows + 7) / 8), 256, 0, s>>>(rows, nrows, Mop, a.m0, Qop, qidx,  \
+      sparse_rows_kernel<V, 4><<<(unsigned)((nrows + 7) / 8), 256, 0, s>>>(rows, nrows, Mop, a.m0, Qop, qidx, \
                                                                         vals, R, nullptr, a.rp);            \
     if (nseg > 0) {                                                                                         \
-      sparse_rows_kernel<V><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(seg, nseg, Mop, a.m0, Qop, qidx,     \
+      sparse_rows_kernel<V, 8><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(seg, nseg, Mop, a.m0, Qop, qidx,  \
                                                                        vals, R, partials, a.rp);            \
-      sparse_reduce_kernel<<<(unsigned)((nmulti + 7) / 8), 256, 0, s>>>(multi, nmulti, partials, R, a.m0,   \
-                                                                        a.rp);                              \
+      launch_reduce(multi, nmulti, partials, R, a.m0, a.rp, s);                                             \
     }                                                                                                       \
   } while (0)
   switch (a.rp) {
@@ -590,33 +791,52 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
 #undef NMD_SP
 }
 
-template <int RP>
-static void update_rp(const StepArgs& a, const float* R, const float* Ginv, float eta, float gamma, bool momentum,
-                      int* status, cudaStream_t s) {
-  constexpr int CW = RP <= 128 ? RP : 128;
-  const size_t smem = ((size_t)RP * CW + (size_t)RP * (64 + 4)) * sizeof(float);
-  static bool attr = false;
-  if (!attr) {
-    cudaFuncSetAttribute(update_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    attr = true;
-  }
-  const int per_sm = RP <= 64 ? 2 : 1;
-  const int64_t tiles = (a.M + 63) / 64;
-  dim3 grid((unsigned)std::min<int64_t>(tiles, 152 * per_sm), RP / CW);
-  const Factor& f = *a.fm;
-  update_kernel<RP><<<grid, 256, smem, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Ginv, eta, gamma,
-                                            momentum, a.epilogue == NMD_EPI_DELTA, status);
+__global__ void zero_kernel(float4* __restrict__ p, int64_t n) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+    p[i] = make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
-void launch_update(const StepArgs& a, const float* R, const float* Ginv, float eta, float gamma, bool momentum,
-                   int* status, cudaStream_t s) {
-  switch (a.rp) {
-    case 16: update_rp<16>(a, R, Ginv, eta, gamma, momentum, status, s); break;
-    case 32: update_rp<32>(a, R, Ginv, eta, gamma, momentum, status, s); break;
-    case 64: update_rp<64>(a, R, Ginv, eta, gamma, momentum, status, s); break;
-    case 128: update_rp<128>(a, R, Ginv, eta, gamma, momentum, status, s); break;
-    default: update_rp<256>(a, R, Ginv, eta, gamma, momentum, status, s); break;
+template <int RP>
+static void update_rp(const StepArgs& a, const float* R, float* Rs, const float* Ginv, float eta, float gamma,
+                      bool momentum, int* status, cudaStream_t s) {
+  using C = UpdCfg<RP>;
+  static int per_sm = 0;
+  if (per_sm == 0) {
+    cudaFuncSetAttribute(update_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, update_kernel<RP>, 256, C::SMEM) != cudaSuccess ||
+        per_sm < 1)
+      per_sm = 1;
   }
+  const int64_t tiles = (a.M + C::TR - 1) / C::TR;
+  dim3 grid((unsigned)std::min<int64_t>(tiles, (int64_t)a.num_sms * per_sm), RP / C::CW);
+  const Factor& f = *a.fm;
+  update_kernel<RP><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, Ginv, eta, gamma,
+                                               momentum, a.epilogue == NMD_EPI_DELTA,
+                                               a.precision == NMD_FP32, status);
+  if (RP / C::CW > 1) zero_kernel<<<grid_for(a.M * RP / 4, 256), 256, 0, s>>>((float4*)Rs, a.M * RP / 4);
+}
+
+void launch_update(const StepArgs& a, const float* R, float* Rs, const float* Ginv, float eta, float gamma,
+                   bool momentum, int* status, cudaStream_t s) {
+  switch (a.rp) {
+    case 16: update_rp<16>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
+    case 32: update_rp<32>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
+    case 64: update_rp<64>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
+    case 128: update_rp<128>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
+    default: update_rp<256>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
+  }
+}
+
+// R += Rs, Rs = 0 over the first n floats (the terms of a step without update)
+__global__ void combine_kernel(float* __restrict__ R, float* __restrict__ Rs, int64_t n) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    R[i] += Rs[i];
+    Rs[i] = 0.f;
+  }
+}
+
+void launch_combine(float* R, float* Rs, int64_t n, cudaStream_t s) {
+  combine_kernel<<<grid_for(n, 256), 256, 0, s>>>(R, Rs, n);
 }
 
 void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s) {

@@ -64,6 +64,7 @@ struct StepArgs {
   int64_t m0, M, q0, K;
   int r, rp;
   int precision, epilogue;
+  int num_sms = 152;         // streaming multiprocessors of the device (grid sizing)
 };
 
 struct Workspace {
@@ -77,10 +78,20 @@ struct Workspace {
   float* valT = nullptr;
   // panel lists: [side][kind]
   PanelRow* panels = nullptr;
+  // R, G and G^{-1} exist twice: step t uses copy t % 2, so that the tail of
+  // step t's update can still read its copy while step t + 1 runs
   float* R = nullptr;          // max(m, n) x rp fp32 right-hand side / staging
+  float* R2 = nullptr;         // second copy of R
+  // the support term of R (sparse correction), kept zero outside the rows
+  // of the step in flight: written by the sparse kernels, added to R and
+  // cleared by the update; two copies like R
+  float* Rs = nullptr;
+  float* Rs2 = nullptr;
   float* gram_part = nullptr;  // kGramParts x rp x rp
-  float* G = nullptr;          // rp x rp (last Gram, for verification)
+  float* G = nullptr;          // rp x rp (Gram, for verification)
   float* Ginv = nullptr;       // rp x rp
+  float* G2 = nullptr;
+  float* Ginv2 = nullptr;
   double* loss_part = nullptr; // kLossParts x 8
   double* loss_out = nullptr;  // 8
   int* status = nullptr;       // kStatusWords
@@ -103,6 +114,27 @@ struct nmd_handle {
   // `stream` around the dense kernel of each step
   cudaStream_t side = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // Within a sweep, the rows of a step's update that the next step does not
+  // read are updated on `aux`, overlapping the next step.  pend[f] records,
+  // for factor f (0 = W, 1 = B), the rows such an update may still be
+  // writing and the event that marks its end.
+  cudaStream_t aux = nullptr;   // lowest priority
+  // a sweep runs on `hp` (highest priority, forked from and joined back into
+  // `stream`), so that the next step's kernels are scheduled ahead of the
+  // deferred updates; `cur` is the stream the current call issues to
+  cudaStream_t hp = nullptr;
+  cudaStream_t cur = nullptr;
+  cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+  cudaEvent_t ev_prio = nullptr;
+  struct Pending {
+    bool active = false;
+    int64_t step = 0;
+    int64_t a0 = 0, a1 = 0, b0 = 0, b1 = 0;   // rows [a0, a1) and [b0, b1) in flight
+    cudaEvent_t ev = nullptr;
+  } pend[2];
+  float* cur_R = nullptr;      // the copies of R, Rs and G the last step used
+  float* cur_Rs = nullptr;
+  float* cur_G = nullptr;
   nmd::Workspace ws;
   nmd::Factor W, B;            // A = W (m x r), B = H^T (n x r)
   nmd::PanelSet panels[2][2];  // [side][kind]
@@ -138,8 +170,9 @@ void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge,
 void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* seg,
                    int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
                    const float* vals, float* R, float* partials, cudaStream_t s);
-void launch_update(const StepArgs& a, const float* R, const float* Ginv, float eta,
+void launch_update(const StepArgs& a, const float* R, float* Rs, const float* Ginv, float eta,
                    float gamma, bool momentum, int* status, cudaStream_t s);
+void launch_combine(float* R, float* Rs, int64_t n, cudaStream_t s);
 void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s);
 void launch_loss_final(const double* dense_parts, int ndense, const double* sparse_parts,
                        int nsparse, double* out, cudaStream_t s);
