@@ -210,13 +210,18 @@ nmd_status nmd_get_state(nmd_handle* h, float* W, float* H, float* EW, float* EH
 nmd_status nmd_set_state(nmd_handle* h, const float* W, const float* H, const float* EW,
                          const float* EH, int64_t sweep_index);
 
-/* Kernel timing with CUDA events recorded on the handle's stream around each
- * launch.  nmd_profile(h, 1) clears the totals and starts recording,
- * nmd_profile(h, 0) stops.  nmd_profile_read synchronises and returns the
- * device time (ms) and launch count accumulated for one kernel class:
- * NMD_K_DENSE (the fused Z-panel kernel), NMD_K_SPARSE (support
- * correction), NMD_K_GRAM (Gram matrix + inverse), NMD_K_UPDATE (least
- * squares / momentum update), NMD_K_LOSS (dense loss pass). */
+/* Kernel timing with CUDA events recorded around each launch, on the stream
+ * the launch goes to (inside nmd_sweep the library's own streams, which
+ * overlap: class totals can add up to more than the elapsed time).
+ * nmd_profile(h, 1) clears the totals and starts recording, nmd_profile(h, 0)
+ * stops.  nmd_profile_read synchronises and returns the device time (ms) and
+ * launch count accumulated for one kernel class: NMD_K_DENSE (the fused
+ * Z-panel kernel), NMD_K_SPARSE (support correction), NMD_K_GRAM (Gram
+ * matrix + inverse), NMD_K_UPDATE (least squares / momentum update),
+ * NMD_K_LOSS (dense loss pass).  With the environment variable NMD_TRACE set
+ * to a file name, the launches timed since the last read are also appended
+ * to that file, one line "class start_ms end_ms" each, relative to the
+ * first of them (a timeline across the streams). */
 typedef enum { NMD_K_DENSE = 0, NMD_K_SPARSE = 1, NMD_K_GRAM = 2, NMD_K_UPDATE = 3, NMD_K_LOSS = 4 } nmd_kernel_class;
 nmd_status nmd_profile(nmd_handle* h, int on);
 nmd_status nmd_profile_read(nmd_handle* h, int32_t kernel_class, double* ms, int64_t* launches);

@@ -499,7 +499,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   // The side stream computes G = Q^T Q of the Q-side rows, G^{-1}, and the
   // support term Rs of R; the main stream the dense term of R.  Neither reads
   // what the other writes, so they overlap; the update joins them.
-  int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 255) / 256));
+  int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 127) / 128));
   CK(h, cudaEventRecord(h->ev_fork, s));
   CK(h, cudaStreamWaitEvent(h->side, h->ev_fork, 0));
   {

@@ -89,16 +89,17 @@ __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ Q, 
       int64_t k = kb + rr;
       bool ok = k < k1;
       Qa[rr][cc] = (ok && cc < wa) ? Q[(q0 + k) * rp + ta * 64 + cc] : 0.f;
-      Qb[rr][cc] = (ok && cc < wb) ? Q[(q0 + k) * rp + tb * 64 + cc] : 0.f;
+      if (ta != tb) Qb[rr][cc] = (ok && cc < wb) ? Q[(q0 + k) * rp + tb * 64 + cc] : 0.f;
     }
     __syncthreads();
+    const float(*Qs)[65] = ta != tb ? Qb : Qa;   // a diagonal tile reads one copy
 #pragma unroll 4
     for (int rr = 0; rr < 32; ++rr) {
       float a[4], b[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) a[i] = Qa[rr][ty * 4 + i];
 #pragma unroll
-      for (int j = 0; j < 4; ++j) b[j] = Qb[rr][tx * 4 + j];
+      for (int j = 0; j < 4; ++j) b[j] = Qs[rr][tx * 4 + j];
 #pragma unroll
       for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -214,6 +215,7 @@ __global__ void __launch_bounds__(RP * 4) ginv_reg_kernel(const float* __restric
   float a[CPT];
 #pragma unroll
   for (int j = 0; j < CPT; ++j) a[j] = 0.f;
+#pragma unroll 4
   for (int p = 0; p < nparts; ++p) {
     const float* src = parts + (size_t)p * RP * RP;
     if (direct) {
@@ -413,7 +415,7 @@ __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commi
 __device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
 
 template <int RP>
-__global__ void __launch_bounds__(256) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
+__global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
                                                      bf16* __restrict__ Mlo, bf16* __restrict__ Mlo2,
                                                      float* __restrict__ E, int64_t m0, int64_t rows,
                                                      const float* __restrict__ R, float* __restrict__ Rs,
@@ -441,9 +443,13 @@ __global__ void __launch_bounds__(256) update_kernel(float* __restrict__ M, bf16
     }
   };
   int64_t t = blockIdx.x;
+  // G^{-1} (its CW columns) and the first tile of R in one copy group
+  for (int e = threadIdx.x; e < RP * CW / 4; e += 256) {
+    const int k = (4 * e) / CW, c = (4 * e) % CW;
+    cp_async16(Gs + 4 * e, Ginv + k * RP + cw0 + c);
+  }
   if (t < ntiles) issue(t, 0);
   cp_async_commit();
-  for (int e = threadIdx.x; e < RP * CW; e += 256) Gs[e] = Ginv[(e / CW) * RP + cw0 + (e % CW)];
   int buf = 0;
   for (; t < ntiles; t += gridDim.x, buf ^= 1) {
     if (t + gridDim.x < ntiles) issue(t + gridDim.x, buf ^ 1);
