@@ -41,6 +41,24 @@ WORKLOADS = {
 }
 
 
+# DRAM bytes (read + write) of one dense-kernel launch, from the ncu capture
+# summarised in profiles/dense_panel_connectome_r64_bf16.md; valid only while
+# the kernel's sources hash to the digest recorded with it (else null)
+DENSE_TRAFFIC = {
+    # (workload, precision, epilogue): (bytes per launch, sha256 prefix of the kernel sources)
+    ("connectome-139255-r64", "bf16", "z"): (18910720 + 7680, "24a91da28205588e"),
+}
+
+
+def dense_source_digest():
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("panel_tc.cu", "tc_ptx.cuh"):
+        with open(os.path.join(ROOT, "paper_2608_21607_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
 def peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -229,9 +247,14 @@ def main():
     pk, pk_kind = peaks()
     peak = pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
     achieved = flops_sweep * args.steps / (dense_ms / 1e3) / 1e12 if dense_ms > 0 else None
+    traffic = None
+    rec = DENSE_TRAFFIC.get((wl.name, args.precision, args.epilogue))
+    if rec and rec[1] == dense_source_digest():
+        traffic = rec[0]
     roofline = {"bound": "tensor", "kernel": "panel_tc_kernel (fused Z-panel, tcgen05)",
                 "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": (achieved / peak) if achieved else None, "traffic": None,
+                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)",
                 "peak_kind": "%s bf16 dense, sustained" % pk_kind,
                 "flops_per_launch": flops_per_launch, "launches": dense_n,
                 "avg_launch_us": 1e3 * dense_ms / max(dense_n, 1),
