@@ -58,7 +58,13 @@ struct Cfg {
   // product of width 2 r_pad (two accumulators side by side, summed at
   // readout): half the MMA instructions of two separate products
   static constexpr bool FUSEDN = !SPLIT && !LOSS && RP <= 128;
-  static constexpr int RCOLS = FUSEDN ? 2 * RP : RP;   // TMEM columns of the R accumulator(s)
+  // fp32-accurate mode at r_pad = 256: W hi + lo take 256 TMEM columns, so a
+  // CTA accumulates one 128-column half of R (blockIdx.y selects it) and the
+  // first product is formed once per half
+  static constexpr bool RHALF = SPLIT && !LOSS && RP == 256;
+  static constexpr int NR = RHALF ? RP / 2 : RP;        // R columns of one CTA
+  // TMEM columns of the R accumulator(s); the loss pass has none
+  static constexpr int RCOLS = LOSS ? 0 : (FUSEDN ? 2 * RP : NR);
   // Q rows per chunk.  64 where the TMEM budget would otherwise leave only
   // two L buffers: more chunks in flight hide the epilogue's latency.
   static constexpr int BN = (RP == 256 || (SPLIT && RP == 128) || FUSEDN) ? 64 : 128;
@@ -120,7 +126,7 @@ __device__ __noinline__ bool wait_bar_slow(uint32_t bar, uint32_t parity, volati
                                            int where) {
   const uint64_t t0 = globaltimer_ns();
   for (;;) {
-    if (mbar_try_wait_sleep(bar, parity, 20000u)) return true;
+    if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
     if (globaltimer_ns() - t0 > kTimeoutNs) {
       *abort_flag = 1;
@@ -308,7 +314,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     // R += P[lb] x chunk for every chunk once its P is in TMEM; frees the
     // shared-memory stage and the L buffer, and hands R over per tile.
     if (!LOSS) {
-      constexpr uint32_t idesc2 = idesc_bf16(BM, C::FUSEDN ? 2 * RP : RP, true, EPI == 1 && !SPLIT);   // Q MN-major
+      constexpr uint32_t idesc2 = idesc_bf16(BM, C::FUSEDN ? 2 * RP : C::NR, true, EPI == 1 && !SPLIT);   // Q MN-major
+      // R columns [hcol, hcol + NR) of Q: their panels start hcol / PANEL_W panels in
+      const uint32_t hpan = C::RHALF ? (uint32_t)blockIdx.y * (C::NR / C::PANEL_W) * C::PANEL_BYTES : 0u;
       const int64_t my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
       const int64_t total = my_tiles * nchunks;
       const uint32_t stage0 = smem_u32(stages);
@@ -320,7 +328,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = conv_wait(b_pfull + 8 * l2, ph_pfull, abort_flag, p.status, 5))) break;
         if (c2 == 0 && !(ok = conv_wait(b_rempty, ph_rempty, abort_flag, p.status, 6))) break;
         fence_after();
-        const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
+        const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES + hpan, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
         const uint32_t pl = tmem + C::COL_L + l2 * BN;
 #pragma unroll
         for (int k = 0; k < BN / 16; ++k) {
@@ -522,9 +530,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = warp_wait(b_rfull, (uint32_t)(tt & 1), abort_flag, p.status, 8))) break;
         fence_after();
         const int64_t li = t * BM + row;
-        float* dst = p.R + li * RP;
+        float* dst = p.R + li * RP + (C::RHALF ? (int64_t)blockIdx.y * C::NR : 0);
 #pragma unroll 1
-        for (int j = wg; j < (RP + 31) / 32; j += 2) {
+        for (int j = wg; j < (C::NR + 31) / 32; j += 2) {
           uint32_t v[32];
           tmem_ld32(tmem + lane_base + C::COL_R + j * 32, v);   // RP = 16 reads 16 spare columns
           if (C::FUSEDN) {
@@ -544,7 +552,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (li < p.M) {
 #pragma unroll
             for (int i = 0; i < 32; i += 4)
-              if (j * 32 + i < RP)
+              if (j * 32 + i < C::NR)
                 *(float4*)(dst + j * 32 + i) = make_float4(__uint_as_float(v[i]), __uint_as_float(v[i + 1]),
                                                           __uint_as_float(v[i + 2]), __uint_as_float(v[i + 3]));
           }
@@ -645,19 +653,17 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
       return NMD_ERR_CUDA;
     attr_set = true;
   }
-  panel_tc_kernel<RP, EPI, SPLIT, LOSS><<<grid, kThreads, C::SMEM, s>>>(th, tl, tl2, p);
+  panel_tc_kernel<RP, EPI, SPLIT, LOSS><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u), kThreads, C::SMEM, s>>>(th, tl, tl2, p);
   return NMD_OK;
 }
 
 template <int RP, bool LOSS>
 nmd_status dispatch_rp(int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p, int grid,
                        cudaStream_t s) {
-  if (LOSS) return split ? run<RP, 0, (RP < 256), LOSS>(fm, fq, p, grid, s) : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
-  if (split) {
-    if (RP == 256) return NMD_ERR_UNSUPPORTED;
-    return epilogue == NMD_EPI_DELTA ? run<RP, 1, (RP < 256), LOSS>(fm, fq, p, grid, s)
-                                     : run<RP, 0, (RP < 256), LOSS>(fm, fq, p, grid, s);
-  }
+  if (LOSS) return split ? run<RP, 0, true, LOSS>(fm, fq, p, grid, s) : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
+  if (split)
+    return epilogue == NMD_EPI_DELTA ? run<RP, 1, true, LOSS>(fm, fq, p, grid, s)
+                                     : run<RP, 0, true, LOSS>(fm, fq, p, grid, s);
   return epilogue == NMD_EPI_DELTA ? run<RP, 1, false, LOSS>(fm, fq, p, grid, s)
                                    : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
 }
@@ -665,7 +671,6 @@ nmd_status dispatch_rp(int epilogue, bool split, const Factor& fm, const Factor&
 template <bool LOSS>
 nmd_status dispatch(int rp, int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p,
                     int grid, cudaStream_t s) {
-  if (split && rp == 256) return NMD_ERR_UNSUPPORTED;
   switch (rp) {
     case 16: return dispatch_rp<16, LOSS>(epilogue, split, fm, fq, p, grid, s);
     case 32: return dispatch_rp<32, LOSS>(epilogue, split, fm, fq, p, grid, s);
@@ -680,7 +685,6 @@ nmd_status dispatch(int rp, int epilogue, bool split, const Factor& fm, const Fa
 
 bool tc_supported(int rp, int precision) {
   if (precision == NMD_SIMT) return false;
-  if (precision == NMD_FP32 && rp == 256) return false;
   return rp == 16 || rp == 32 || rp == 64 || rp == 128 || rp == 256;
 }
 

@@ -44,8 +44,6 @@ def gpu():
 
 def _pair(name, precision, epilogue=N.NMD_EPI_Z, momentum=False, **kw):
     _, S, r, W, H, br, bc, sched = cases()[name]
-    if precision == N.NMD_FP32 and r > 128:
-        pytest.skip("fp32-accurate tensor-core path covers r <= 128")
     EW = EH = None
     if momentum:
         rng = np.random.default_rng(11)

@@ -62,8 +62,6 @@ RANKS = [(3, 1000, 192), (32, 700, 160), (64, 900, 200), (100, 600, 224), (256, 
 @pytest.mark.parametrize("precision", [N.NMD_BF16, N.NMD_FP32], ids=["bf16", "fp32"])
 @pytest.mark.parametrize("r,n,b", RANKS, ids=[str(x[0]) for x in RANKS])
 def test_first_product_L(r, n, b, precision):
-    if precision == N.NMD_FP32 and r > 128:
-        pytest.skip("fp32-accurate tensor-core path covers r <= 128")
     S = WL.connectome(n, seed=r)
     W, H = WL.init_factors(n, n, r, r)
     sol = N.Solver(S, r, block_rows=b, block_cols=b, precision=precision)
@@ -91,8 +89,6 @@ def test_first_product_L(r, n, b, precision):
 @pytest.mark.parametrize("epi", [N.NMD_EPI_Z, N.NMD_EPI_DELTA], ids=["zform", "delta"])
 @pytest.mark.parametrize("r,n,b", RANKS, ids=[str(x[0]) for x in RANKS])
 def test_second_product_R(r, n, b, epi, precision):
-    if precision == N.NMD_FP32 and r > 128:
-        pytest.skip("fp32-accurate tensor-core path covers r <= 128")
     S = WL.connectome(n, seed=r + 1)
     W, H = WL.init_factors(n, n, r, r + 1)
     sol = N.Solver(S, r, block_rows=b, block_cols=b, precision=precision, epilogue=epi)
