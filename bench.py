@@ -38,6 +38,7 @@ WORKLOADS = {
     "connectome_r256": ("connectome_r256", 256, 8192),
     "planted_medium": ("planted_medium", 32, 2048),
     "identity": ("identity", 3, 512),
+    "planted_tiny": ("planted_tiny", 4, 128),
 }
 
 
@@ -123,6 +124,7 @@ def oracle_sample(wl, budget_s=20.0):
     import numpy as np
     import oracle as O
     st = O.State(wl.S, wl.W0, wl.H0, O.Options(block_rows=wl.block_rows, block_cols=wl.block_cols,
+                                                 schedule=O.EXACT if wl.schedule == "exact" else O.STOCH,
                                                  eta=wl.eta, gamma=wl.gamma))
     steps = st.sweep_steps(0)
     entries, t_used, done = 0, 0.0, []
@@ -171,14 +173,14 @@ def main():
                 vals.append((v, nsteps, t))
         value = statistics.median(v for v, _, _ in vals)
         tsum = sum(t for _, _, t in vals)
-        sample = ("%d block steps of the sweep per timed step (first COL/STOCH and ROW/STOCH blocks of "
+        sample = ("%d block steps of the sweep per timed step (the first blocks of "
                   "sweep 0), fp64 oracle, numpy on %d host cores" % (vals[0][1], cores))
         line = {"impl": "reference", "metric": metric, "value": value, "unit": "Z entries/s",
                 "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
                 "ms_per_step": 1e3 * tsum / len(vals), "higher_is_better": True, "scaling": "weak",
                 "vs_baseline": None, "dtype": "f64", "data": "synthetic",
                 "config": {"workload": wl.name, "m": wl.m, "n": wl.n, "nnz": wl.S.nnz, "r": r,
-                           "block": block, "schedule": "stochastic", "parallelism": "host cores"},
+                           "block": block, "schedule": wl.schedule, "parallelism": "host cores"},
                 "cpu_baseline": {"value": value, "unit": "Z entries/s", "cores": cores, "kind": "oracle",
                                  "sample": sample},
                 "e2e": {"value": value, "unit": "Z entries/s", "h2d_bytes_per_step": 0,
@@ -198,7 +200,9 @@ def main():
     wl = WLm.workload(gen, seed=0)
     prec = {"bf16": N.NMD_BF16, "fp32": N.NMD_FP32}[args.precision]
     epi = {"z": N.NMD_EPI_Z, "delta": N.NMD_EPI_DELTA}[args.epilogue]
-    sol = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols, schedule=N.NMD_STOCH,
+    exact = wl.schedule == "exact"
+    sol = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols,
+                   schedule=N.NMD_EXACT if exact else N.NMD_STOCH,
                    eta=wl.eta, gamma=wl.gamma, precision=prec, epilogue=epi, seed=0)
     sol.set_factors(wl.W0, wl.H0)
     stream = sol.stream
@@ -216,16 +220,31 @@ def main():
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
+    # Workloads whose whole workspace fits in L2 (129 MB) are timed sweep by
+    # sweep with L2 flushed before each (a 512 MB write, outside the timed
+    # interval); the others already stream more than L2 per sweep.
+    ws_bytes = sol.workspace.numel() * sol.workspace.element_size()
+    flush = ws_bytes < 256 * 2**20
+    scratch = torch.empty(512 * 2**20, dtype=torch.uint8, device="cuda") if flush else None
     l0 = sol.launches
     sol.profile(True)
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
-        sol.sweep()
-    e1.record(stream)
+    ms_total = 0.0
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps if flush else 1)]
+    if flush:
+        for e0, e1 in ev:
+            with torch.cuda.stream(stream):
+                scratch.fill_(1)
+            e0.record(stream)
+            sol.sweep()
+            e1.record(stream)
+    else:
+        ev[0][0].record(stream)
+        for _ in range(args.steps):
+            sol.sweep()
+        ev[0][1].record(stream)
     sol.sync()
-    ms_total = e0.elapsed_time(e1)
+    ms_total = sum(e0.elapsed_time(e1) for e0, e1 in ev)
     launches = sol.launches - l0
     dense_ms, dense_n = sol.profile_read(N.NMD_K_DENSE)
     other = {name: sol.profile_read(k) for name, k in
@@ -302,10 +321,14 @@ def main():
                 "scaling": "weak", "vs_baseline": None, "dtype": args.precision if prec == N.NMD_BF16 else "f32",
                 "data": "synthetic",
                 "config": {"workload": wl.name, "m": wl.m, "n": wl.n, "nnz": wl.S.nnz, "r": wl.r,
-                           "block": wl.block_rows, "schedule": "stochastic, alternating", "eta": wl.eta,
+                           "block": wl.block_rows,
+                           "schedule": "exact (row blocks, then column blocks)" if exact else "stochastic, alternating",
+                           "eta": wl.eta,
                            "gamma": wl.gamma, "precision": args.precision,
                            "epilogue": args.epilogue, "parallelism": "replicas" if ws > 1 else "single GPU",
-                           "l2": "inputs larger than L2 (factors, momentum and operand copies ~260 MB)"},
+                           "workspace_mb": round(ws_bytes / 2**20, 1),
+                           "l2": ("workspace smaller than L2: L2 flushed (512 MB write) before each timed sweep"
+                                  if flush else "workspace larger than L2 (%.0f MB): no flush" % (ws_bytes / 2**20))},
                 "e2e": e2e, "roofline": roofline, "cpu_baseline": cpu, "clocks": clk,
                 "gpu_launches": launches}
         print(json.dumps(line))
