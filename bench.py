@@ -150,6 +150,8 @@ def main():
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="connectome_r64")
     ap.add_argument("--precision", choices=["bf16", "fp32"], default="bf16")
     ap.add_argument("--epilogue", choices=["z", "delta"], default="z")
+    ap.add_argument("--init", choices=["normal", "paper"], default="normal",
+                    help="factor start: iid N(0, 0.01), or the sign-structured start W > 0, H < 0")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing on the host")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg (profiling runs)")
     args = ap.parse_args()
@@ -204,7 +206,10 @@ def main():
     sol = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols,
                    schedule=N.NMD_EXACT if exact else N.NMD_STOCH,
                    eta=wl.eta, gamma=wl.gamma, precision=prec, epilogue=epi, seed=0)
-    sol.set_factors(wl.W0, wl.H0)
+    W0, H0 = wl.W0, wl.H0
+    if args.init == "paper":
+        W0, H0 = WLm.init_factors(wl.m, wl.n, wl.r, 0, signs="paper")
+    sol.set_factors(W0, H0)
     stream = sol.stream
 
     def barrier():
@@ -227,6 +232,7 @@ def main():
     flush = ws_bytes < 256 * 2**20
     scratch = torch.empty(512 * 2**20, dtype=torch.uint8, device="cuda") if flush else None
     l0 = sol.launches
+    sol.skip_count(reset=True)
     sol.profile(True)
     ms_total = 0.0
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -246,6 +252,7 @@ def main():
     sol.sync()
     ms_total = sum(e0.elapsed_time(e1) for e0, e1 in ev)
     launches = sol.launches - l0
+    skipped = sol.skip_count(reset=True)
     dense_ms, dense_n = sol.profile_read(N.NMD_K_DENSE)
     other = {name: sol.profile_read(k) for name, k in
              [("sparse", N.NMD_K_SPARSE), ("gram_inverse", N.NMD_K_GRAM), ("update", N.NMD_K_UPDATE)]}
@@ -283,8 +290,8 @@ def main():
         roofline["note"] = "fp32-accurate mode issues 3 bf16 MMAs per product; flops counted once"
 
     # ---------------- end to end through the public API, host buffers -------
-    Wh = torch.from_numpy(np.ascontiguousarray(wl.W0, np.float32)).pin_memory()
-    Hh = torch.from_numpy(np.ascontiguousarray(wl.H0, np.float32)).pin_memory()
+    Wh = torch.from_numpy(np.ascontiguousarray(W0, np.float32)).pin_memory()
+    Hh = torch.from_numpy(np.ascontiguousarray(H0, np.float32)).pin_memory()
     Wo = torch.empty_like(Wh).pin_memory()
     Ho = torch.empty_like(Hh).pin_memory()
     h2d = (Wh.numel() + Hh.numel()) * 4
@@ -325,7 +332,9 @@ def main():
                            "schedule": "exact (row blocks, then column blocks)" if exact else "stochastic, alternating",
                            "eta": wl.eta,
                            "gamma": wl.gamma, "precision": args.precision,
-                           "epilogue": args.epilogue, "parallelism": "replicas" if ws > 1 else "single GPU",
+                           "epilogue": args.epilogue, "init": args.init,
+                           "skipped_chunks_per_sweep": skipped / args.steps,
+                           "parallelism": "replicas" if ws > 1 else "single GPU",
                            "workspace_mb": round(ws_bytes / 2**20, 1),
                            "l2": ("workspace smaller than L2: L2 flushed (512 MB write) before each timed sweep"
                                   if flush else "workspace larger than L2 (%.0f MB): no flush" % (ws_bytes / 2**20))},

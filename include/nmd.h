@@ -247,6 +247,15 @@ nmd_status nmd_gram_noalloc(const float* d_Q, int64_t K, int32_t r, int64_t ld, 
 /* Number of kernel launches this handle has issued (for launch accounting). */
 int64_t nmd_launch_count(const nmd_handle* h);
 
+/* Delta form (epilogue NMD_EPI_DELTA): number of Q chunks (64 or 128 Q-side
+ * rows against a 128-row M tile) whose second product the tensor-core panel
+ * kernel skipped because max(0, L) was zero on the whole chunk -- the tile
+ * skipping of Sec. 4.3 (the rectified tile is sparse where the model is
+ * mostly negative).  The first chunk of every tile is always computed.
+ * Counts since creation or the last reset; synchronises; reset != 0 sets
+ * the count back to zero. */
+nmd_status nmd_skip_count(nmd_handle* h, int64_t* skipped, int32_t reset);
+
 const char* nmd_status_string(nmd_status s);
 const char* nmd_last_error(const nmd_handle* h);
 void nmd_destroy(nmd_handle* h);

@@ -624,6 +624,17 @@ const char* nmd_last_error(const nmd_handle* h) { return h ? h->last_error.c_str
 
 int64_t nmd_launch_count(const nmd_handle* h) { return h ? h->launches : 0; }
 
+nmd_status nmd_skip_count(nmd_handle* h, int64_t* skipped, int32_t reset) {
+  if (!h || !skipped) return NMD_ERR_INVALID;
+  nmd_status st = sync_and_check(h);
+  if (st != NMD_OK) return st;
+  unsigned long long v = 0;
+  CK(h, cudaMemcpy(&v, h->ws.counters, sizeof v, cudaMemcpyDeviceToHost));
+  *skipped = (int64_t)v;
+  if (reset) CK(h, cudaMemset(h->ws.counters, 0, sizeof v));
+  return NMD_OK;
+}
+
 nmd_status nmd_workspace_bytes(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
                                const int32_t* col_idx, const float* vals, const nmd_options* opts,
                                size_t* bytes) {

@@ -95,7 +95,7 @@ struct Workspace {
   double* loss_part = nullptr; // kLossParts x 8
   double* loss_out = nullptr;  // 8
   int* status = nullptr;       // kStatusWords
-  int* counters = nullptr;     // 64 ints (tile schedulers)
+  int* counters = nullptr;     // 64 ints; ints 0-1: skipped Delta-form chunks (u64)
   float* chol_scratch = nullptr;  // 2 x rp x rp (used when rp is too large for smem)
   float* seg_partials = nullptr;  // max segments x rp (sparse correction of long rows)
 };

@@ -91,7 +91,9 @@ struct Cfg {
   // barriers: full[NSTAGE], empty[NSTAGE], lfull[NB], pfull[NB], lfree[NB], rfull, rempty,
   // wfull[2], wempty[2], drain, drain2
   static constexpr int NBAR = 2 * NSTAGE + 3 * NB + 8;
-  static constexpr size_t SMEM_USED = 1024 + (size_t)NSTAGE * STAGE_BYTES + NBAR * 8 + 64 + 256 * 16;
+  // after the barriers: TMEM slot and abort flag (64 B), the loss reduction
+  // (256 x 16 B), and 4 flags per L buffer (Delta form: P nonzero per warp)
+  static constexpr size_t SMEM_USED = 1024 + (size_t)NSTAGE * STAGE_BYTES + NBAR * 8 + 64 + 256 * 16 + NB * 16;
   // at least 120 KB so that a second CTA (and its 512-column TMEM request)
   // never shares the SM
   static constexpr size_t SMEM = SMEM_USED > 120 * 1024 ? SMEM_USED : 120 * 1024;
@@ -113,6 +115,7 @@ struct TcParams {
   float* Lout;          // verification: raw L (M x K, row-major) or nullptr
   const int64_t* rowptr;   // loss kernel: CSR of S, whose entries the dense pass skips
   const int32_t* cidx;
+  unsigned long long* skips;   // Delta form: count of chunks whose second product was skipped (or nullptr)
 };
 
 __device__ __forceinline__ void record(int* status, int code, int detail) {
@@ -175,6 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint32_t* tmem_slot = (uint32_t*)(bars + C::NBAR);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
   double* red = (double*)(smem + (size_t)NSTAGE * C::STAGE_BYTES + C::NBAR * 8 + 64);
+  volatile uint32_t* pflag = (volatile uint32_t*)(red + 2 * kEpiThreads);   // [NB][4]
 
   const uint32_t b_full = smem_u32(bars);
   const uint32_t b_empty = b_full + 8 * NSTAGE;
@@ -328,10 +332,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = conv_wait(b_pfull + 8 * l2, ph_pfull, abort_flag, p.status, 5))) break;
         if (c2 == 0 && !(ok = conv_wait(b_rempty, ph_rempty, abort_flag, p.status, 6))) break;
         fence_after();
+        // Delta form: a chunk whose P is zero in every row adds nothing to R
+        // (Sec. 4.3); its MMAs are skipped, except for the first chunk of a
+        // tile, which initialises the accumulator
+        bool skip = false;
+        if (EPI == 1 && c2 > 0)
+          skip = (pflag[4 * l2] | pflag[4 * l2 + 1] | pflag[4 * l2 + 2] | pflag[4 * l2 + 3]) == 0u;
+        if (skip && p.skips != nullptr && lane == 0) atomicAdd(p.skips, 1ull);
         const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES + hpan, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
         const uint32_t pl = tmem + C::COL_L + l2 * BN;
 #pragma unroll
-        for (int k = 0; k < BN / 16; ++k) {
+        for (int k = 0; k < BN / 16 && !skip; ++k) {
           const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
           const uint64_t bl = bh + (C::OPER_BYTES >> 4);
           const uint32_t acc = (c2 > 0 || k > 0) ? 1u : 0u;
@@ -434,6 +445,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int kv = (int)(p.K - c * BN < BN ? p.K - c * BN : BN);   // valid columns in this chunk
         const uint32_t lcol = tmem + lane_base + C::COL_L + lb * BN;
         float c2 = 0.f, c1 = 0.f;
+        uint32_t nzacc = 0u;   // Delta form: OR of this thread's P words
 #pragma unroll 1
         for (int jj = 0; jj < BN / 64; ++jj) {
           uint32_t v0[32], v1[32];
@@ -487,6 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               } else {          // max(0, L); the MMA negates it
                 pk0[i] = pack_relu_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1]));
                 pk1[i] = pack_relu_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1]));
+                nzacc |= (pk0[i] | pk1[i]) & 0x7fff7fffu;   // -0 counts as zero
               }
             }
             tmem_st16(lcol + jj * 32, pk0);
@@ -506,6 +519,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float h0 = __uint_as_float(hp << 16), h1 = __uint_as_float(hp & 0xffff0000u);
                 ph[i] = hp;
                 pl[i] = pack_bf16x2(e0 - h0, e1 - h1);
+                if (EPI == 1) nzacc |= (ph[i] | pl[i]) & 0x7fff7fffu;   // -0 counts as zero
               }
               tmem_st16(lcol + (2 * jj + h) * 32, ph);
               tmem_st16(lcol + (2 * jj + h) * 32 + 16, pl);
@@ -519,6 +533,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(b_lfree + 8 * lb);
         } else {
+          if (EPI == 1) {   // published before the arrive (release) that MMA2 acquires
+            const bool nz = __any_sync(0xffffffffu, nzacc != 0u);
+            if (lane == 0) pflag[4 * lb + (warp & 3)] = nz ? 1u : 0u;
+          }
           tmem_wait_st();
           fence_before();
           __syncwarp();
@@ -690,9 +708,9 @@ bool tc_supported(int rp, int precision) {
 
 nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counter, int num_sms, cudaStream_t s,
                            int64_t* launches, float* Lout) {
-  (void)counter;
   if (!tc_supported(a.rp, a.precision)) return NMD_ERR_UNSUPPORTED;
-  TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout, nullptr, nullptr};
+  TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout, nullptr, nullptr,
+             (unsigned long long*)counter};
   // fewest CTAs that keep the same number of tile rounds: the SMs left over
   // run the side-stream kernels of the step
   const int64_t ntiles = (a.M + BM - 1) / BM;
@@ -706,7 +724,8 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
 nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts, int* status,
                                 cudaStream_t s, int64_t* launches) {
   if (!tc_supported(h->rp, h->opt.precision)) return NMD_ERR_UNSUPPORTED;
-  TcParams p{0, h->m, 0, h->n, h->W.hi, h->W.lo, nullptr, parts, status, nullptr, h->ws.rowptr, h->ws.col};
+  TcParams p{0, h->m, 0, h->n, h->W.hi, h->W.lo, nullptr, parts, status, nullptr, h->ws.rowptr, h->ws.col,
+             nullptr};
   int64_t ntiles = (h->m + BM - 1) / BM;
   int grid = (int)(ntiles < h->num_sms ? ntiles : h->num_sms);
   if (grid > maxparts) grid = maxparts;

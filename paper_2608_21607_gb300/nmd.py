@@ -30,7 +30,7 @@ EXPORTS = [
     "nmd_version", "nmd_default_options", "nmd_workspace_bytes", "nmd_create", "nmd_set_factors",
     "nmd_get_factors", "nmd_block_update", "nmd_sweep", "nmd_block_order", "nmd_loss", "nmd_sync",
     "nmd_block_terms", "nmd_dense_products", "nmd_panel_traversal", "nmd_get_state", "nmd_set_state",
-    "nmd_launch_count", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
+    "nmd_launch_count", "nmd_skip_count", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
     "nmd_destroy", "nmd_gram_noalloc",
 ]
 
@@ -87,6 +87,7 @@ def lib() -> C.CDLL:
             "nmd_get_state": (C.c_int, [_P, _P, _P, _P, _P, _i64p]),
             "nmd_set_state": (C.c_int, [_P, _P, _P, _P, _P, C.c_int64]),
             "nmd_launch_count": (C.c_int64, [_P]),
+            "nmd_skip_count": (C.c_int, [_P, C.POINTER(C.c_int64), C.c_int32]),
             "nmd_profile": (C.c_int, [_P, C.c_int]),
             "nmd_profile_read": (C.c_int, [_P, C.c_int32, C.POINTER(C.c_double), _i64p]),
             "nmd_status_string": (C.c_char_p, [C.c_int]),
@@ -236,6 +237,12 @@ def nmd_launch_count(h) -> int:
     return lib().nmd_launch_count(h)
 
 
+def nmd_skip_count(h, reset: bool = False) -> int:
+    v = C.c_int64(0)
+    _check(h, lib().nmd_skip_count(h, C.byref(v), 1 if reset else 0), "nmd_skip_count")
+    return int(v.value)
+
+
 def nmd_profile(h, on: bool):
     _check(h, lib().nmd_profile(h, int(on)), "nmd_profile")
 
@@ -357,3 +364,7 @@ class Solver:
     @property
     def launches(self) -> int:
         return nmd_launch_count(self.h)
+
+    def skip_count(self, reset: bool = False) -> int:
+        """Delta form: chunks whose second product was skipped (all-zero P)."""
+        return nmd_skip_count(self.h, reset)

@@ -91,11 +91,19 @@ def csr_from_dense(D: np.ndarray, dtype=np.float32) -> CSR:
     return CSR(m, n, row_ptr, cols.astype(np.int32), D[rows, cols].astype(dtype))
 
 
-def init_factors(m: int, n: int, r: int, seed: int, sigma: float = 0.1):
-    """W (m x r) and H (r x n) iid N(0, sigma^2), float32."""
+def init_factors(m: int, n: int, r: int, seed: int, sigma: float = 0.1, signs: str = "normal"):
+    """W (m x r) and H (r x n) iid N(0, sigma^2), float32.
+
+    signs="paper": the sign-structured start of Sec. 4.3, W = |N(0, sigma^2)|
+    and H = -|N(0, sigma^2)|, so that W H < 0 everywhere at the start (the
+    rectified matrix is empty)."""
     rng = np.random.default_rng([seed, 0xF0C7])
     W = (sigma * rng.standard_normal((m, r))).astype(np.float32)
     H = (sigma * rng.standard_normal((r, n))).astype(np.float32)
+    if signs == "paper":
+        W, H = np.abs(W), -np.abs(H)
+    elif signs != "normal":
+        raise ValueError("signs must be 'normal' or 'paper'")
     return W, H
 
 
