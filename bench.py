@@ -39,6 +39,7 @@ WORKLOADS = {
     "planted_medium": ("planted_medium", 32, 2048),
     "identity": ("identity", 3, 512),
     "planted_tiny": ("planted_tiny", 4, 128),
+    "connectome_dense_r64": ("connectome_dense_r64", 64, 4096),
 }
 
 
@@ -150,6 +151,8 @@ def main():
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="connectome_r64")
     ap.add_argument("--precision", choices=["bf16", "fp32"], default="bf16")
     ap.add_argument("--epilogue", choices=["z", "delta"], default="z")
+    ap.add_argument("--skip-zero-chunks", action="store_true",
+                    help="Delta form: skip the second product of chunks whose rectified tile is zero")
     ap.add_argument("--init", choices=["normal", "paper"], default="normal",
                     help="factor start: iid N(0, 0.01), or the sign-structured start W > 0, H < 0")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing on the host")
@@ -205,7 +208,8 @@ def main():
     exact = wl.schedule == "exact"
     sol = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols,
                    schedule=N.NMD_EXACT if exact else N.NMD_STOCH,
-                   eta=wl.eta, gamma=wl.gamma, precision=prec, epilogue=epi, seed=0)
+                   eta=wl.eta, gamma=wl.gamma, precision=prec, epilogue=epi, seed=0,
+                   skip_zero_chunks=args.skip_zero_chunks)
     W0, H0 = wl.W0, wl.H0
     if args.init == "paper":
         W0, H0 = WLm.init_factors(wl.m, wl.n, wl.r, 0, signs="paper")
@@ -333,6 +337,7 @@ def main():
                            "eta": wl.eta,
                            "gamma": wl.gamma, "precision": args.precision,
                            "epilogue": args.epilogue, "init": args.init,
+                           "skip_zero_chunks": args.skip_zero_chunks,
                            "skipped_chunks_per_sweep": skipped / args.steps,
                            "parallelism": "replicas" if ws > 1 else "single GPU",
                            "workspace_mb": round(ws_bytes / 2**20, 1),

@@ -90,6 +90,9 @@ typedef struct {
   int32_t precision;    /* nmd_precision */
   int32_t epilogue;     /* nmd_epilogue */
   uint64_t seed;        /* block-order seed */
+  int32_t skip_zero_chunks;  /* Delta form: skip the second product of Q chunks whose rectified
+                              * tile is zero (Sec. 4.3; see nmd_skip_count).  Default 0: the check
+                              * costs the dense kernel time when no chunk vanishes */
 } nmd_options;
 
 typedef struct {

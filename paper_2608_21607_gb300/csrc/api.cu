@@ -477,7 +477,8 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   Roles ro;
   nmd_status st = roles(h, side, block, kind, &ro);
   if (st != NMD_OK) return st;
-  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms};
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
+              h->opt.skip_zero_chunks != 0};
   cudaStream_t s = h->cur;
   // wait for deferred updates of rows this step reads or writes, and for
   // those of two steps back (they read the copies of R and G^{-1} reused now)
@@ -916,7 +917,8 @@ nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_
   nmd_status st = roles(h, side, block, kind, &ro);
   if (st != NMD_OK) return st;
   if (h->opt.precision == NMD_SIMT) return fail(h, NMD_ERR_UNSUPPORTED, "dense products hook needs a tensor-core precision");
-  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms};
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
+              h->opt.skip_zero_chunks != 0};
   st = launch_panel_tc(a, h->ws.R, h->ws.status, h->ws.counters, h->num_sms, h->stream, &h->launches, d_L);
   if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
   if ((st = after_launch(h, "dense products")) != NMD_OK) return st;

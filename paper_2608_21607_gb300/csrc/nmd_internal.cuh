@@ -65,6 +65,7 @@ struct StepArgs {
   int r, rp;
   int precision, epilogue;
   int num_sms = 152;         // streaming multiprocessors of the device (grid sizing)
+  bool skip_zero = false;    // Delta form: skip chunks whose rectified tile is zero
 };
 
 struct Workspace {

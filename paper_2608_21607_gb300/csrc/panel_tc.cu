@@ -116,6 +116,7 @@ struct TcParams {
   const int64_t* rowptr;   // loss kernel: CSR of S, whose entries the dense pass skips
   const int32_t* cidx;
   unsigned long long* skips;   // Delta form: count of chunks whose second product was skipped (or nullptr)
+  int skip_on;                 // Delta form: skip chunks whose rectified tile is zero
 };
 
 __device__ __forceinline__ void record(int* status, int code, int detail) {
@@ -165,7 +166,10 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   return ok != 0;
 }
 
-template <int RP, int EPI, bool SPLIT, bool LOSS>
+// SKIP (Delta form only): skip the second product of chunks whose rectified
+// tile is zero; a separate instantiation, so that the kernel without it
+// carries none of the checks.
+template <int RP, int EPI, bool SPLIT, bool LOSS, bool SKIP>
 __global__ void __launch_bounds__(kThreads, 1)
     panel_tc_kernel(const __grid_constant__ CUtensorMap tq_hi, const __grid_constant__ CUtensorMap tq_lo,
                     const __grid_constant__ CUtensorMap tq_lo2, const TcParams p) {
@@ -336,13 +340,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         // (Sec. 4.3); its MMAs are skipped, except for the first chunk of a
         // tile, which initialises the accumulator
         bool skip = false;
-        if (EPI == 1 && c2 > 0)
+        static_assert(!SKIP || (EPI == 1 && !LOSS), "skipping is a Delta-form option");
+        if (SKIP && c2 > 0)
           skip = (pflag[4 * l2] | pflag[4 * l2 + 1] | pflag[4 * l2 + 2] | pflag[4 * l2 + 3]) == 0u;
         if (skip && p.skips != nullptr && lane == 0) atomicAdd(p.skips, 1ull);
         const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES + hpan, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
         const uint32_t pl = tmem + C::COL_L + l2 * BN;
 #pragma unroll
-        for (int k = 0; k < BN / 16 && !skip; ++k) {
+        for (int k = 0; k < BN / 16 && !(SKIP && skip); ++k) {
           const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
           const uint64_t bl = bh + (C::OPER_BYTES >> 4);
           const uint32_t acc = (c2 > 0 || k > 0) ? 1u : 0u;
@@ -499,7 +504,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               } else {          // max(0, L); the MMA negates it
                 pk0[i] = pack_relu_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1]));
                 pk1[i] = pack_relu_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1]));
-                nzacc |= (pk0[i] | pk1[i]) & 0x7fff7fffu;   // -0 counts as zero
+                if (SKIP) nzacc |= (pk0[i] | pk1[i]) & 0x7fff7fffu;   // -0 counts as zero
               }
             }
             tmem_st16(lcol + jj * 32, pk0);
@@ -519,7 +524,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const float h0 = __uint_as_float(hp << 16), h1 = __uint_as_float(hp & 0xffff0000u);
                 ph[i] = hp;
                 pl[i] = pack_bf16x2(e0 - h0, e1 - h1);
-                if (EPI == 1) nzacc |= (ph[i] | pl[i]) & 0x7fff7fffu;   // -0 counts as zero
+                if (SKIP) nzacc |= (ph[i] | pl[i]) & 0x7fff7fffu;   // -0 counts as zero
               }
               tmem_st16(lcol + (2 * jj + h) * 32, ph);
               tmem_st16(lcol + (2 * jj + h) * 32 + 16, pl);
@@ -533,7 +538,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(b_lfree + 8 * lb);
         } else {
-          if (EPI == 1) {   // published before the arrive (release) that MMA2 acquires
+          if (SKIP) {   // published before the arrive (release) that MMA2 acquires
             const bool nz = __any_sync(0xffffffffu, nzacc != 0u);
             if (lane == 0) pflag[4 * lb + (warp & 3)] = nz ? 1u : 0u;
           }
@@ -656,7 +661,7 @@ bool tensor_map(const bf16* base, int64_t rows, int rp, int panel_w, int bn, CUt
   return true;
 }
 
-template <int RP, int EPI, bool SPLIT, bool LOSS>
+template <int RP, int EPI, bool SPLIT, bool LOSS, bool SKIP = false>
 nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, cudaStream_t s) {
   using C = Cfg<RP, SPLIT, LOSS>;
   CUtensorMap th, tl, tl2;
@@ -666,12 +671,12 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
   (void)fm;
   static bool attr_set = false;
   if (!attr_set) {
-    if (cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)C::SMEM) != cudaSuccess)
       return NMD_ERR_CUDA;
     attr_set = true;
   }
-  panel_tc_kernel<RP, EPI, SPLIT, LOSS><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u), kThreads, C::SMEM, s>>>(th, tl, tl2, p);
+  panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u), kThreads, C::SMEM, s>>>(th, tl, tl2, p);
   return NMD_OK;
 }
 
@@ -679,6 +684,10 @@ template <int RP, bool LOSS>
 nmd_status dispatch_rp(int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p, int grid,
                        cudaStream_t s) {
   if (LOSS) return split ? run<RP, 0, true, LOSS>(fm, fq, p, grid, s) : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
+  if (epilogue == NMD_EPI_DELTA && p.skip_on) {
+    if (split) return run<RP, 1, true, false, true>(fm, fq, p, grid, s);
+    return run<RP, 1, false, false, true>(fm, fq, p, grid, s);
+  }
   if (split)
     return epilogue == NMD_EPI_DELTA ? run<RP, 1, true, LOSS>(fm, fq, p, grid, s)
                                      : run<RP, 0, true, LOSS>(fm, fq, p, grid, s);
@@ -710,7 +719,7 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
                            int64_t* launches, float* Lout) {
   if (!tc_supported(a.rp, a.precision)) return NMD_ERR_UNSUPPORTED;
   TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout, nullptr, nullptr,
-             (unsigned long long*)counter};
+             (unsigned long long*)counter, a.skip_zero ? 1 : 0};
   // fewest CTAs that keep the same number of tile rounds: the SMs left over
   // run the side-stream kernels of the step
   const int64_t ntiles = (a.M + BM - 1) / BM;
@@ -725,7 +734,7 @@ nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts
                                 cudaStream_t s, int64_t* launches) {
   if (!tc_supported(h->rp, h->opt.precision)) return NMD_ERR_UNSUPPORTED;
   TcParams p{0, h->m, 0, h->n, h->W.hi, h->W.lo, nullptr, parts, status, nullptr, h->ws.rowptr, h->ws.col,
-             nullptr};
+             nullptr, 0};
   int64_t ntiles = (h->m + BM - 1) / BM;
   int grid = (int)(ntiles < h->num_sms ? ntiles : h->num_sms);
   if (grid > maxparts) grid = maxparts;

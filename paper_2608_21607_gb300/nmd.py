@@ -39,7 +39,7 @@ class nmd_options(C.Structure):
     _fields_ = [("block_rows", C.c_int64), ("block_cols", C.c_int64), ("schedule", C.c_int32),
                 ("order", C.c_int32), ("eta", C.c_double), ("gamma", C.c_double),
                 ("ridge", C.c_double), ("precision", C.c_int32), ("epilogue", C.c_int32),
-                ("seed", C.c_uint64)]
+                ("seed", C.c_uint64), ("skip_zero_chunks", C.c_int32)]
 
 
 class nmd_loss_out(C.Structure):
@@ -278,7 +278,7 @@ class Solver:
 
     def __init__(self, S, r: int, *, block_rows=4096, block_cols=4096, schedule=NMD_STOCH,
                  order=NMD_ALTERNATE, eta=1.0, gamma=0.9, ridge=0.0, precision=NMD_BF16,
-                 epilogue=NMD_EPI_Z, seed=0, stream=None, device=None):
+                 epilogue=NMD_EPI_Z, seed=0, skip_zero_chunks=False, stream=None, device=None):
         import torch
         self.m, self.n, self.r = int(S.m), int(S.n), int(r)
         o = nmd_default_options()
@@ -286,6 +286,7 @@ class Solver:
         o.schedule, o.order = int(schedule), int(order)
         o.eta, o.gamma, o.ridge = float(eta), float(gamma), float(ridge)
         o.precision, o.epilogue, o.seed = int(precision), int(epilogue), int(seed)
+        o.skip_zero_chunks = 1 if skip_zero_chunks else 0
         self.opts = o
         self.device = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
         nbytes = nmd_workspace_bytes(S, self.r, o)

@@ -248,11 +248,11 @@ def _planted_medium(seed=0, n=20000, r=32, block=2048, **kw):
                     1.0, 0.0, seed, {"tau": tau, "d": 32})
 
 
-def _connectome(seed=0, n=139255, r=64, block=4096, sweeps=10, **kw):
-    S = connectome(n, seed=seed)
+def _connectome(seed=0, n=139255, r=64, block=4096, sweeps=10, mean_degree=20.0, tag="", **kw):
+    S = connectome(n, mean_degree=mean_degree, seed=seed)
     W, H = init_factors(n, n, r, seed)
-    return Workload("connectome-%d-r%d" % (n, r), S, r, W, H, block, block, "stoch", sweeps,
-                    0.5, 0.9, seed, {})
+    return Workload("connectome%s-%d-r%d" % (tag, n, r), S, r, W, H, block, block, "stoch", sweeps,
+                    0.5, 0.9, seed, {"mean_degree": mean_degree})
 
 
 WORKLOADS = {
@@ -261,6 +261,10 @@ WORKLOADS = {
     "planted_medium": _planted_medium,
     "connectome_r64": lambda seed=0, **kw: _connectome(seed, r=64, block=4096, sweeps=10, **kw),
     "connectome_r256": lambda seed=0, **kw: _connectome(seed, r=256, block=8192, sweeps=5, **kw),
+    # the same generator at the density of Table 1's connectome
+    # (rho+ = 0.00102 of the n^2 entries: mean out-degree 142, ~19.8M nonzeros)
+    "connectome_dense_r64": lambda seed=0, **kw: _connectome(seed, r=64, block=4096, sweeps=10,
+                                                             mean_degree=0.00102 * 139254, tag="-dense", **kw),
 }
 
 

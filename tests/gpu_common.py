@@ -31,11 +31,11 @@ def rel(a, b):
 
 def make_pair(S, r, W, H, *, block_rows, block_cols, precision, epilogue=N.NMD_EPI_Z,
               schedule=N.NMD_STOCH, eta=0.5, gamma=0.9, seed=0, order=N.NMD_ALTERNATE, EW=None,
-              EH=None):
+              EH=None, skip_zero_chunks=False):
     """A GPU solver and an oracle state holding the same factors and momentum."""
     sol = N.Solver(S, r, block_rows=block_rows, block_cols=block_cols, schedule=schedule,
                    order=order, eta=eta, gamma=gamma, precision=precision, epilogue=epilogue,
-                   seed=seed)
+                   seed=seed, skip_zero_chunks=skip_zero_chunks)
     W = np.ascontiguousarray(W, np.float32)
     H = np.ascontiguousarray(H, np.float32)
     if EW is None:

@@ -51,7 +51,7 @@ def test_skipped_chunks_keep_the_result(r, n, b, prec):
     # all-negative L: every chunk but the first of each tile is skipped
     W, H = _signed_factors(n, r, seed=r)
     sol, orc = make_pair(S, r, W, H, block_rows=b, block_cols=b, precision=prec, epilogue=N.NMD_EPI_DELTA,
-                         eta=1.0, gamma=0.0)
+                         eta=1.0, gamma=0.0, skip_zero_chunks=True)
     sol.skip_count(reset=True)
     Rg, Ro = _step_terms(sol, orc, N.NMD_COL, block, N.NMD_STOCH)
     all_neg = sol.skip_count(reset=True)
@@ -64,7 +64,7 @@ def test_skipped_chunks_keep_the_result(r, n, b, prec):
     # computed, the others are still skipped
     W2, H2 = _signed_factors(n, r, seed=r, flip=np.arange(q0 + 128, min(q0 + 192, n)))
     sol2, orc2 = make_pair(S, r, W2, H2, block_rows=b, block_cols=b, precision=prec,
-                           epilogue=N.NMD_EPI_DELTA, eta=1.0, gamma=0.0)
+                           epilogue=N.NMD_EPI_DELTA, eta=1.0, gamma=0.0, skip_zero_chunks=True)
     sol2.skip_count(reset=True)
     Rg2, Ro2 = _step_terms(sol2, orc2, N.NMD_COL, block, N.NMD_STOCH)
     mixed = sol2.skip_count(reset=True)
@@ -78,11 +78,21 @@ def test_skipped_chunks_keep_the_result(r, n, b, prec):
     assert rel(Wg, orc2.A) <= TOL[prec]
 
 
+def test_skipping_is_off_by_default():
+    S = WL.connectome(1500, seed=6)
+    W, H = _signed_factors(1500, 32, seed=6)
+    sol, _ = make_pair(S, 32, W, H, block_rows=320, block_cols=320, precision=N.NMD_BF16,
+                       epilogue=N.NMD_EPI_DELTA, eta=1.0, gamma=0.0)
+    sol.skip_count(reset=True)
+    sol.block_update(N.NMD_COL, 1, N.NMD_STOCH)
+    assert sol.skip_count() == 0
+
+
 def test_z_form_never_skips():
     S = WL.connectome(1500, seed=5)
     W, H = _signed_factors(1500, 32, seed=5)
     sol, _ = make_pair(S, 32, W, H, block_rows=320, block_cols=320, precision=N.NMD_BF16,
-                       epilogue=N.NMD_EPI_Z, eta=1.0, gamma=0.0)
+                       epilogue=N.NMD_EPI_Z, eta=1.0, gamma=0.0, skip_zero_chunks=True)
     sol.skip_count(reset=True)
     sol.block_update(N.NMD_COL, 1, N.NMD_STOCH)
     assert sol.skip_count() == 0
