@@ -142,31 +142,35 @@ nmd_status build_sparse(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   return NMD_OK;
 }
 
-// Split every block's rows (ascending) into single rows (len <= kSeg) and
-// segments of kSeg entries for the longer rows.
+// Split every block's rows (ascending) into short rows (len <= kShort), whole
+// long rows (len <= kSeg) and kSeg slices of the longer rows.
 void finalize_panels(const std::vector<std::vector<PanelRow>>& per, PanelSet* P) {
   int64_t K = (int64_t)per.size();
   P->host.clear(); P->seg.clear(); P->multi.clear();
   P->row_ptr.assign(K + 1, 0);
   P->seg_ptr.assign(K + 1, 0);
   P->multi_ptr.assign(K + 1, 0);
+  P->segd.assign(K, 0);
   P->max_segments = 0;
   for (int64_t k = 0; k < K; ++k) {
     P->row_ptr[k] = (int64_t)P->host.size();
     P->seg_ptr[k] = (int64_t)P->seg.size();
     P->multi_ptr[k] = (int64_t)P->multi.size();
     for (const PanelRow& pr : per[k]) {
-      if (pr.len <= kSeg) {
-        P->host.push_back(pr);
-        continue;
-      }
-      int64_t first = (int64_t)P->seg.size() - P->seg_ptr[k];   // slot within the block
+      if (pr.len <= kShort) P->host.push_back(pr);
+      else if (pr.len <= kSeg) P->seg.push_back(pr);
+    }
+    P->segd[k] = (int64_t)P->seg.size() - P->seg_ptr[k];
+    const int64_t s0 = (int64_t)P->seg.size();
+    for (const PanelRow& pr : per[k]) {
+      if (pr.len <= kSeg) continue;
+      int64_t first = (int64_t)P->seg.size() - s0;   // slot within the block's slices
       int32_t nseg = 0;
       for (int64_t off = 0; off < pr.len; off += kSeg, ++nseg)
         P->seg.push_back(PanelRow{pr.row, (int32_t)std::min<int64_t>(kSeg, pr.len - off), pr.beg + off});
       P->multi.push_back(PanelRow{pr.row, nseg, first});
     }
-    P->max_segments = std::max<int64_t>(P->max_segments, (int64_t)P->seg.size() - P->seg_ptr[k]);
+    P->max_segments = std::max<int64_t>(P->max_segments, (int64_t)P->seg.size() - s0);
   }
   P->row_ptr[K] = (int64_t)P->host.size();
   P->seg_ptr[K] = (int64_t)P->seg.size();
@@ -514,13 +518,13 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   // sparse correction over the block's support
   const PanelSet& P = *ro.P;
   int64_t r0 = P.row_ptr[block], r1 = P.row_ptr[block + 1];
-  int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1];
+  int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1], gd = g0 + P.segd[block];
   int64_t u0 = P.multi_ptr[block], u1 = P.multi_ptr[block + 1];
   {
     TimedScope ts(h, NMD_K_SPARSE, h->side);
-    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, g1 - g0, P.d_multi + u0, u1 - u0, ro.qidx, ro.vals, Rs,
-                  h->ws.seg_partials, h->side);
-    h->launches += (r1 > r0) + 2 * (g1 > g0);
+    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, gd - g0, P.d_seg + gd, g1 - gd, P.d_multi + u0, u1 - u0,
+                  ro.qidx, ro.vals, Rs, h->ws.seg_partials, h->side);
+    h->launches += (r1 > r0) + (gd > g0) + 2 * (g1 > gd);
   }
   if ((st = after_launch(h, "sparse correction")) != NMD_OK) return st;
   CK(h, cudaEventRecord(h->ev_join, h->side));
@@ -937,11 +941,13 @@ nmd_status nmd_panel_traversal(const nmd_handle* h, int32_t side, int64_t block,
   // host mirrors of the index arrays are not kept; rebuild q from the device copy
   const PanelSet& P = *ro.P;
   std::vector<PanelRow> list(P.host.begin() + P.row_ptr[block], P.host.begin() + P.row_ptr[block + 1]);
+  const int64_t gs = P.seg_ptr[block] + P.segd[block];   // first slice of the split rows
+  list.insert(list.end(), P.seg.begin() + P.seg_ptr[block], P.seg.begin() + gs);
   for (int64_t u = P.multi_ptr[block]; u < P.multi_ptr[block + 1]; ++u) {
     const PanelRow& mr = P.multi[u];
-    const PanelRow& first = P.seg[P.seg_ptr[block] + mr.beg];
+    const PanelRow& first = P.seg[gs + mr.beg];
     int64_t len = 0;
-    for (int32_t q = 0; q < mr.len; ++q) len += P.seg[P.seg_ptr[block] + mr.beg + q].len;
+    for (int32_t q = 0; q < mr.len; ++q) len += P.seg[gs + mr.beg + q].len;
     list.push_back(PanelRow{mr.row, (int32_t)len, first.beg});
   }
   std::sort(list.begin(), list.end(), [](const PanelRow& a, const PanelRow& b) { return a.row < b.row; });

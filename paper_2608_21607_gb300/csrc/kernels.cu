@@ -344,6 +344,102 @@ __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __rest
   }
 }
 
+// Long rows (more than kShort entries in the panel): one warp per row or kSeg
+// slice with the lanes over the entries.  LPE = rp / 32 lanes share an entry
+// (lane sub = lane % LPE owns columns 32 sub ... 32 sub + 31; CPL = min(32, rp)
+// of them are real), so a warp takes EPW = 32 / LPE entries at a time.  The
+// q rows of those entries are first copied into a per-warp shared buffer with
+// coalesced loads (whole 128-byte lines), as 32 chunks of 32 columns padded to
+// 36 floats, chunk = lane that reads it, so that each lane's reads are free of
+// bank conflicts.  Each lane then forms its part of L_ik = m_i . q_k, the LPE
+// parts are added with shuffles, c = S_ik - min(0, L_ik), and the lane
+// accumulates c q_k over its own entries; at the end the EPW entry slots are
+// added with a butterfly (one reduction per row instead of one per entry).
+// The order of every sum is fixed, so results are the same on every run.
+template <int LPE, int CPL>
+__global__ void __launch_bounds__(256, 2) sparse_long_kernel(const PanelRow* __restrict__ segs, int64_t nseg,
+                                                          const float* __restrict__ Mop, int64_t m0,
+                                                          const float* __restrict__ Qop,
+                                                          const int32_t* __restrict__ qidx,
+                                                          const float* __restrict__ vals,
+                                                          float* __restrict__ R, float* __restrict__ partials,
+                                                          int rp) {
+  constexpr int EPW = 32 / LPE;
+  constexpr int CS = 36;                       // floats per staged chunk (32 + 4 padding)
+  constexpr int NPF = 4;                       // entry iterations whose indices are fetched together
+  __shared__ __align__(16) float stage[8][32 * CS];
+  const int lane = threadIdx.x & 31;
+  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
+  if (w >= nseg) return;
+  float* buf = stage[(threadIdx.x >> 5) & 7];
+  const PanelRow pr = segs[w];
+  const int sub = lane % LPE, slot = lane / LPE;
+  const int64_t i = pr.row;
+  float mv[CPL], acc[CPL];
+  {
+    const float4* m4 = (const float4*)(Mop + i * rp + 32 * sub);
+#pragma unroll
+    for (int c = 0; c < CPL / 4; ++c) {
+      const float4 v = __ldg(m4 + c);
+      mv[4 * c] = v.x; mv[4 * c + 1] = v.y; mv[4 * c + 2] = v.z; mv[4 * c + 3] = v.w;
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < CPL; ++c) acc[c] = 0.f;
+  for (int e00 = 0; e00 < pr.len; e00 += NPF * EPW) {
+    int kk[NPF];
+    float ss[NPF];
+#pragma unroll
+    for (int t = 0; t < NPF; ++t) {
+      const int e = e00 + t * EPW + slot;
+      const bool live = e < pr.len;
+      kk[t] = live ? __ldg(qidx + pr.beg + e) : -1;
+      ss[t] = live ? __ldg(vals + pr.beg + e) : 0.f;
+    }
+#pragma unroll
+    for (int t = 0; t < NPF; ++t) {
+      if (e00 + t * EPW >= pr.len) break;             // warp-uniform
+      // stage: float4 f = lane + 32 u (u < CPL / 4) of the 32 chunks; chunk
+      // f / 8 is columns 32 (chunk % LPE) ... of entry slot chunk / LPE
+#pragma unroll
+      for (int u = 0; u < CPL / 4; ++u) {
+        const int f = lane + 32 * u;
+        const int chunk = f / (CPL / 4), part = f % (CPL / 4);
+        const int ke = __shfl_sync(0xffffffffu, kk[t], (chunk / LPE) * LPE);
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (ke >= 0) v = __ldg((const float4*)(Qop + (int64_t)ke * rp + 32 * (chunk % LPE)) + part);
+        *(float4*)(buf + chunk * CS + 4 * part) = v;
+      }
+      __syncwarp();
+      float q[CPL];
+#pragma unroll
+      for (int c = 0; c < CPL / 4; ++c) {
+        const float4 v = *(const float4*)(buf + lane * CS + 4 * c);
+        q[4 * c] = v.x; q[4 * c + 1] = v.y; q[4 * c + 2] = v.z; q[4 * c + 3] = v.w;
+      }
+      __syncwarp();                                   // the buffer is refilled next iteration
+      float dot = 0.f;
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) dot = fmaf(mv[c], q[c], dot);
+#pragma unroll
+      for (int o = 1; o < LPE; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+      const float cval = ss[t] - fminf(0.f, dot);    // zero for the padding slots (s = 0, q = 0)
+#pragma unroll
+      for (int c = 0; c < CPL; ++c) acc[c] = fmaf(cval, q[c], acc[c]);
+    }
+  }
+#pragma unroll
+  for (int o = LPE; o < 32; o <<= 1)
+#pragma unroll
+    for (int c = 0; c < CPL; ++c) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
+  if (slot == 0) {
+    float* dst = (partials ? partials + w * rp : R + (i - m0) * rp) + 32 * sub;
+#pragma unroll
+    for (int c = 0; c < CPL / 4; ++c)
+      *(float4*)(dst + 4 * c) = make_float4(acc[4 * c], acc[4 * c + 1], acc[4 * c + 2], acc[4 * c + 3]);
+  }
+}
+
 // Rs_i = sum of the segment slots of row i.  One block per long row: thread
 // t handles column t % RP of the slots g, g + G, g + 2G, ... (g = t / RP,
 // G = 256 / RP groups) with eight loads in flight, and the G group sums are
@@ -768,31 +864,35 @@ static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* pa
   }
 }
 
-void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* seg, int64_t nseg,
-                   const PanelRow* multi, int64_t nmulti, const int32_t* qidx, const float* vals, float* R,
-                   float* partials, cudaStream_t s) {
+void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole, int64_t nwhole,
+                   const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
+                   const float* vals, float* R, float* partials, cudaStream_t s) {
   // The support correction always reads the fp32 masters, in every precision:
   // on rows with few support entries the term S_ik q_k dominates R_i and is
   // not averaged over many products, so rounding q_k to bf16 there would put
   // its full relative error (up to 2^-9) into the update.
   const float* Mop = a.fm->master;
   const float* Qop = a.fq->master;
-#define NMD_SP(V)                                                                                           \
-  do {                                                                                                      \
-    if (nrows > 0)                                                                                          \
+#define NMD_SP(V, LPE, CPL)                                                                                  \
+  do {                                                                                                       \
+    if (nrows > 0)                                                                                           \
       sparse_rows_kernel<V, 4><<<(unsigned)((nrows + 7) / 8), 256, 0, s>>>(rows, nrows, Mop, a.m0, Qop, qidx, \
-                                                                        vals, R, nullptr, a.rp);            \
-    if (nseg > 0) {                                                                                         \
-      sparse_rows_kernel<V, 8><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(seg, nseg, Mop, a.m0, Qop, qidx,  \
-                                                                       vals, R, partials, a.rp);            \
-      launch_reduce(multi, nmulti, partials, R, a.m0, a.rp, s);                                             \
-    }                                                                                                       \
+                                                                           vals, R, nullptr, a.rp);         \
+    if (nwhole > 0)                                                                                          \
+      sparse_long_kernel<LPE, CPL><<<(unsigned)((nwhole + 7) / 8), 256, 0, s>>>(whole, nwhole, Mop, a.m0, Qop, \
+                                                                                qidx, vals, R, nullptr, a.rp); \
+    if (nseg > 0) {                                                                                          \
+      sparse_long_kernel<LPE, CPL><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(seg, nseg, Mop, a.m0, Qop, qidx, \
+                                                                              vals, R, partials, a.rp);      \
+      launch_reduce(multi, nmulti, partials, R, a.m0, a.rp, s);                                              \
+    }                                                                                                        \
   } while (0)
   switch (a.rp) {
-    case 16: case 32: NMD_SP(1); break;
-    case 64: NMD_SP(2); break;
-    case 128: NMD_SP(4); break;
-    default: NMD_SP(8); break;
+    case 16: NMD_SP(1, 1, 16); break;
+    case 32: NMD_SP(1, 1, 32); break;
+    case 64: NMD_SP(2, 2, 32); break;
+    case 128: NMD_SP(4, 4, 32); break;
+    default: NMD_SP(8, 8, 32); break;
   }
 #undef NMD_SP
 }

@@ -23,18 +23,25 @@ struct PanelRow {
   int64_t beg;
 };
 
-// Panel rows with more entries than this are split into segments of at most
-// kSeg entries; each segment's partial sum goes to a scratch slot and the
-// slots of a row are added in a fixed order by a second pass.
-constexpr int kSeg = 32;
+// Panel rows of at most kShort entries are handled one warp per row with the
+// lanes over the r columns.  Longer rows go to a kernel that puts the lanes
+// over the entries, in segments of at most kSeg entries: a row of at most
+// kSeg entries is one segment that writes its result directly; a longer row
+// is split, each segment's partial sum goes to a scratch slot and the slots
+// of a row are added in a fixed order by a second pass.
+constexpr int kShort = 32;
+constexpr int kSeg = 128;
 
 // Per (side, kind): the panel lists of every block, concatenated.  For block k:
-//   single rows   [row_ptr[k], row_ptr[k+1])   of `host`/`d`   (len <= kSeg)
-//   segments      [seg_ptr[k], seg_ptr[k+1])   of `seg`        (one kSeg slice each)
-//   split rows    [multi_ptr[k], multi_ptr[k+1]) of `multi`    (row, #segments, first segment)
+//   short rows    [row_ptr[k], row_ptr[k+1])   of `host`/`d`   (len <= kShort)
+//   segments      [seg_ptr[k], seg_ptr[k+1])   of `seg`: first the segd[k]
+//                 whole rows of kShort < len <= kSeg, then the kSeg slices
+//                 of the longer rows
+//   split rows    [multi_ptr[k], multi_ptr[k+1]) of `multi`    (row, #segments,
+//                 first slice relative to the block's slices)
 // Rows are listed in ascending order.
 struct PanelSet {
-  std::vector<int64_t> row_ptr, seg_ptr, multi_ptr;
+  std::vector<int64_t> row_ptr, seg_ptr, multi_ptr, segd;
   std::vector<PanelRow> host, seg, multi;
   PanelRow* d = nullptr;
   PanelRow* d_seg = nullptr;
@@ -168,9 +175,11 @@ void launch_gram(const Factor& fq, int64_t q0, int64_t K, int r, int rp, float* 
                  int nparts, cudaStream_t s);
 void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge, float* G,
                      float* Ginv, float* scratch, int* status, cudaStream_t s);
-void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* seg,
-                   int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
-                   const float* vals, float* R, float* partials, cudaStream_t s);
+// rows: short rows; whole: the whole rows of the long-row kernel; seg: the
+// slices of the split rows, summed per row of `multi` into R
+void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole,
+                   int64_t nwhole, const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti,
+                   const int32_t* qidx, const float* vals, float* R, float* partials, cudaStream_t s);
 void launch_update(const StepArgs& a, const float* R, float* Rs, const float* Ginv, float eta,
                    float gamma, bool momentum, int* status, cudaStream_t s);
 void launch_combine(float* R, float* Rs, int64_t n, cudaStream_t s);
