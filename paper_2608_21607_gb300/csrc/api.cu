@@ -193,6 +193,14 @@ void build_stoch_panels(const std::vector<int64_t>& ptr, const std::vector<int32
     }
   }
   finalize_panels(per, P);
+  // every block's step updates all N rows
+  P->flag_off.assign(K + 1, 0);
+  P->flags.assign((size_t)K * N, 0);
+  for (int64_t k = 0; k < K; ++k) {
+    P->flag_off[k] = k * N;
+    for (const PanelRow& pr : per[k]) P->flags[(size_t)k * N + pr.row] = 1;
+  }
+  P->flag_off[K] = K * N;
 }
 
 // Exact panels: block k of rows [k b, (k+1) b) with their complete rows.
@@ -207,6 +215,14 @@ void build_exact_panels(const std::vector<int64_t>& ptr, int64_t N, int64_t b, P
     }
   }
   finalize_panels(per, P);
+  // block k's step updates its rows [k b, min(N, (k+1) b))
+  P->flag_off.assign(K + 1, 0);
+  P->flags.assign((size_t)N, 0);
+  for (int64_t k = 0; k < K; ++k) {
+    P->flag_off[k] = k * b;
+    for (const PanelRow& pr : per[k]) P->flags[pr.row] = 1;
+  }
+  P->flag_off[K] = N;
 }
 
 void build_panels(const HostSparse& S, const nmd_options& o, PanelSet P[2][2]) {
@@ -235,7 +251,7 @@ struct Carver {
 };
 
 void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanels, int64_t maxseg,
-            Workspace* w, Factor* W, Factor* B) {
+            int64_t nflags, Workspace* w, Factor* W, Factor* B) {
   w->rowptr = c.take<int64_t>(m + 1);
   w->col = c.take<int32_t>(nnz);
   w->val = c.take<float>(nnz);
@@ -263,6 +279,7 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->Ginv2 = c.take<float>((size_t)rp * rp);
   w->chol_scratch = c.take<float>((size_t)2 * rp * rp);
   w->seg_partials = c.take<float>((size_t)std::max<int64_t>(maxseg, 1) * rp);
+  w->flags = c.take<uint8_t>((size_t)std::max<int64_t>(nflags, 1));
   w->loss_part = c.take<double>((size_t)kLossParts * 8);
   w->loss_out = c.take<double>(8);
   w->status = c.take<int>(kStatusWords);
@@ -275,6 +292,13 @@ int64_t panel_total(PanelSet P[2][2]) {
   int64_t t = 0;
   for (int s = 0; s < 2; ++s)
     for (int k = 0; k < 2; ++k) t += (int64_t)(P[s][k].host.size() + P[s][k].seg.size() + P[s][k].multi.size());
+  return t;
+}
+
+int64_t flag_total(PanelSet P[2][2]) {
+  int64_t t = 0;
+  for (int s = 0; s < 2; ++s)
+    for (int k = 0; k < 2; ++k) t += (int64_t)P[s][k].flags.size();
   return t;
 }
 
@@ -464,14 +488,15 @@ struct NextUse {
 };
 
 nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro, float* R, float* Rs,
-                              const float* Ginv, int64_t lo, int64_t hi, bool momentum, cudaStream_t s) {
+                              const uint8_t* flags, const float* Ginv, int64_t lo, int64_t hi, bool momentum,
+                              cudaStream_t s) {
   if (hi <= lo) return NMD_OK;
   StepArgs sub = a;
   sub.m0 = ro.m0 + lo;
   sub.M = hi - lo;
   TimedScope ts(h, NMD_K_UPDATE, s);
-  launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, Ginv, (float)h->opt.eta, momentum ? (float)h->opt.gamma : 0.f,
-                momentum, h->ws.status, s);
+  launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, Ginv, (float)h->opt.eta,
+                momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, s);
   h->launches++;
   return NMD_OK;
 }
@@ -520,6 +545,8 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   int64_t r0 = P.row_ptr[block], r1 = P.row_ptr[block + 1];
   int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1], gd = g0 + P.segd[block];
   int64_t u0 = P.multi_ptr[block], u1 = P.multi_ptr[block + 1];
+  const uint8_t* flags = P.d_flags + P.flag_off[block];
+  h->cur_flags = flags;
   {
     TimedScope ts(h, NMD_K_SPARSE, h->side);
     launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, gd - g0, P.d_seg + gd, g1 - gd, P.d_multi + u0, u1 - u0,
@@ -554,12 +581,12 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
         hi = std::max(std::min(rn.q0 + rn.K - ro.m0, ro.M), lo);
       }
     }
-    if ((st = launch_update_rows(h, a, ro, R, Rs, Ginv, lo, hi, momentum, s)) != NMD_OK) return st;
+    if ((st = launch_update_rows(h, a, ro, R, Rs, flags, Ginv, lo, hi, momentum, s)) != NMD_OK) return st;
     if (lo > 0 || hi < ro.M) {
       CK(h, cudaEventRecord(h->ev_prio, s));
       CK(h, cudaStreamWaitEvent(h->aux, h->ev_prio, 0));
-      if ((st = launch_update_rows(h, a, ro, R, Rs, Ginv, 0, lo, momentum, h->aux)) != NMD_OK) return st;
-      if ((st = launch_update_rows(h, a, ro, R, Rs, Ginv, hi, ro.M, momentum, h->aux)) != NMD_OK) return st;
+      if ((st = launch_update_rows(h, a, ro, R, Rs, flags, Ginv, 0, lo, momentum, h->aux)) != NMD_OK) return st;
+      if ((st = launch_update_rows(h, a, ro, R, Rs, flags, Ginv, hi, ro.M, momentum, h->aux)) != NMD_OK) return st;
       nmd_handle::Pending& pm = h->pend[fm];
       CK(h, cudaEventRecord(pm.ev, h->aux));
       pm.active = true;
@@ -654,7 +681,7 @@ nmd_status nmd_workspace_bytes(int64_t m, int64_t n, int32_t r, const int64_t* r
   Carver c(nullptr);
   Workspace w;
   Factor W, B;
-  layout(c, m, n, (int64_t)S.col.size(), pad_rank(r), panel_total(P), max_segments(P), &w, &W, &B);
+  layout(c, m, n, (int64_t)S.col.size(), pad_rank(r), panel_total(P), max_segments(P), flag_total(P), &w, &W, &B);
   *bytes = w.bytes;
   return NMD_OK;
 }
@@ -682,7 +709,8 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   h->s_fro = S.s_fro;
   build_panels(S, h->opt, h->panels);
   Carver c(d_workspace);
-  layout(c, m, n, h->nnz, h->rp, panel_total(h->panels), max_segments(h->panels), &h->ws, &h->W, &h->B);
+  layout(c, m, n, h->nnz, h->rp, panel_total(h->panels), max_segments(h->panels), flag_total(h->panels), &h->ws,
+         &h->W, &h->B);
   auto bail = [&](nmd_status s, const std::string& w) {
     fprintf(stderr, "nmd_create: %s\n", w.c_str());
     delete h;
@@ -716,8 +744,16 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
       P.d_multi = h->ws.panels + all.size();
       all.insert(all.end(), P.multi.begin(), P.multi.end());
     }
+  std::vector<uint8_t> allf;
+  for (int s2 = 0; s2 < 2; ++s2)
+    for (int k = 0; k < 2; ++k) {
+      PanelSet& P = h->panels[s2][k];
+      P.d_flags = h->ws.flags + allf.size();
+      allf.insert(allf.end(), P.flags.begin(), P.flags.end());
+    }
   cudaStream_t s = h->stream;
   struct Cp { void* d; const void* src; size_t n; } cps[] = {
+      {h->ws.flags, allf.data(), allf.size()},
       {h->ws.rowptr, S.rowptr.data(), S.rowptr.size() * 8},
       {h->ws.col, S.col.data(), S.col.size() * 4},
       {h->ws.val, S.val.data(), S.val.size() * 4},
@@ -902,7 +938,7 @@ nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t k
   if (st != NMD_OK) return st;
   if ((st = run_step(h, side, block, kind, false)) != NMD_OK) return st;
   h->step_index--;
-  launch_combine(h->cur_R, h->cur_Rs, ro.M * h->rp, h->cur);
+  launch_combine(h->cur_R, h->cur_Rs, h->cur_flags, ro.M, h->rp, h->cur);
   h->launches++;
   if ((st = after_launch(h, "combine")) != NMD_OK) return st;
   if ((st = sync_and_check(h)) != NMD_OK) return st;

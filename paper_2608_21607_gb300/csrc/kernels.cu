@@ -514,7 +514,8 @@ template <int RP>
 __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
                                                      bf16* __restrict__ Mlo, bf16* __restrict__ Mlo2,
                                                      float* __restrict__ E, int64_t m0, int64_t rows,
-                                                     const float* __restrict__ R, float* __restrict__ Rs,
+                                                     const float* __restrict__ R, const float* __restrict__ Rs,
+                                                     const uint8_t* __restrict__ flags,
                                                      const float* __restrict__ Ginv, float eta,
                                                      float gamma, int momentum, int delta_form, int write_lo2,
                                                      int* __restrict__ status) {
@@ -551,13 +552,14 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
     if (t + gridDim.x < ntiles) issue(t + gridDim.x, buf ^ 1);
     cp_async_commit();
     const int64_t base = t * TR;
-    // the support term of this tile, taken from Rs (which is left zero)
+    // the support term of this tile: Rs on the rows flagged as having
+    // support in the step's panel (the other rows of Rs are stale)
     float4 sv[NV];
 #pragma unroll
     for (int u = 0; u < NV; ++u) {
       const int64_t o = base * RP + 4 * (threadIdx.x + 256 * u);
       sv[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (o < total) sv[u] = *(const float4*)(Rs + o);
+      if (o < total && __ldg(flags + o / RP)) sv[u] = *(const float4*)(Rs + o);
     }
     // this thread's M and E entries, in flight during the product
     float mo[4][CPT], eo[4][CPT];
@@ -590,8 +592,7 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
     }
     cp_async_wait_1();
     // add the support term to the entries this thread copied (its own copies
-    // have landed), clear Rs there (when one block covers all columns of the
-    // tile; otherwise the launcher clears it afterwards), then publish
+    // have landed), then publish the tile
 #pragma unroll
     for (int u = 0; u < NV; ++u) {
       const int e = threadIdx.x + 256 * u;
@@ -601,7 +602,6 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
         float4 v = *d;
         v.x += sv[u].x; v.y += sv[u].y; v.z += sv[u].z; v.w += sv[u].w;
         *d = v;
-        if (gridDim.y == 1) *(float4*)(Rs + o) = make_float4(0.f, 0.f, 0.f, 0.f);
       }
     }
     __syncthreads();
@@ -897,14 +897,9 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
 #undef NMD_SP
 }
 
-__global__ void zero_kernel(float4* __restrict__ p, int64_t n) {
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
-    p[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-}
-
 template <int RP>
-static void update_rp(const StepArgs& a, const float* R, float* Rs, const float* Ginv, float eta, float gamma,
-                      bool momentum, int* status, cudaStream_t s) {
+static void update_rp(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
+                      float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
   using C = UpdCfg<RP>;
   static int per_sm = 0;
   if (per_sm == 0) {
@@ -916,33 +911,32 @@ static void update_rp(const StepArgs& a, const float* R, float* Rs, const float*
   const int64_t tiles = (a.M + C::TR - 1) / C::TR;
   dim3 grid((unsigned)std::min<int64_t>(tiles, (int64_t)a.num_sms * per_sm), RP / C::CW);
   const Factor& f = *a.fm;
-  update_kernel<RP><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, Ginv, eta, gamma,
+  update_kernel<RP><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, flags, Ginv, eta,
+                                               gamma,
                                                momentum, a.epilogue == NMD_EPI_DELTA,
                                                a.precision == NMD_FP32, status);
-  if (RP / C::CW > 1) zero_kernel<<<grid_for(a.M * RP / 4, 256), 256, 0, s>>>((float4*)Rs, a.M * RP / 4);
 }
 
-void launch_update(const StepArgs& a, const float* R, float* Rs, const float* Ginv, float eta, float gamma,
-                   bool momentum, int* status, cudaStream_t s) {
+void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
+                   float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
   switch (a.rp) {
-    case 16: update_rp<16>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
-    case 32: update_rp<32>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
-    case 64: update_rp<64>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
-    case 128: update_rp<128>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
-    default: update_rp<256>(a, R, Rs, Ginv, eta, gamma, momentum, status, s); break;
+    case 16: update_rp<16>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
+    case 32: update_rp<32>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
+    case 64: update_rp<64>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
+    case 128: update_rp<128>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
+    default: update_rp<256>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
   }
 }
 
-// R += Rs, Rs = 0 over the first n floats (the terms of a step without update)
-__global__ void combine_kernel(float* __restrict__ R, float* __restrict__ Rs, int64_t n) {
-  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
-    R[i] += Rs[i];
-    Rs[i] = 0.f;
-  }
+// R += Rs on the flagged rows (the terms of a step without update)
+__global__ void combine_kernel(float* __restrict__ R, const float* __restrict__ Rs,
+                               const uint8_t* __restrict__ flags, int64_t n, int rp) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x)
+    if (flags[i / rp]) R[i] += Rs[i];
 }
 
-void launch_combine(float* R, float* Rs, int64_t n, cudaStream_t s) {
-  combine_kernel<<<grid_for(n, 256), 256, 0, s>>>(R, Rs, n);
+void launch_combine(float* R, const float* Rs, const uint8_t* flags, int64_t rows, int rp, cudaStream_t s) {
+  combine_kernel<<<grid_for(rows * rp, 256), 256, 0, s>>>(R, Rs, flags, rows * rp, rp);
 }
 
 void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s) {

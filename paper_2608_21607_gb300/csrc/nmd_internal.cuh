@@ -47,6 +47,11 @@ struct PanelSet {
   PanelRow* d_seg = nullptr;
   PanelRow* d_multi = nullptr;
   int64_t max_segments = 0;     // largest segment count of any block
+  // per block, one byte per M-side row of the step: 1 if the row has support
+  // entries in the panel (its row of Rs is written by the step), else 0
+  std::vector<int64_t> flag_off;
+  std::vector<uint8_t> flags;
+  uint8_t* d_flags = nullptr;
 };
 
 // Device status word (sticky): [0] = nmd_status code of the first error,
@@ -90,9 +95,9 @@ struct Workspace {
   // step t's update can still read its copy while step t + 1 runs
   float* R = nullptr;          // max(m, n) x rp fp32 right-hand side / staging
   float* R2 = nullptr;         // second copy of R
-  // the support term of R (sparse correction), kept zero outside the rows
-  // of the step in flight: written by the sparse kernels, added to R and
-  // cleared by the update; two copies like R
+  // the support term of R (sparse correction): written by the sparse kernels
+  // on the rows with support in the step's panel (the others are not read),
+  // added to R by the update; two copies like R
   float* Rs = nullptr;
   float* Rs2 = nullptr;
   float* gram_part = nullptr;  // kGramParts x rp x rp
@@ -106,6 +111,7 @@ struct Workspace {
   int* counters = nullptr;     // 64 ints; ints 0-1: skipped Delta-form chunks (u64)
   float* chol_scratch = nullptr;  // 2 x rp x rp (used when rp is too large for smem)
   float* seg_partials = nullptr;  // max segments x rp (sparse correction of long rows)
+  uint8_t* flags = nullptr;       // the panels' support-row flags, concatenated
 };
 
 constexpr int kGramParts = 64;
@@ -142,6 +148,7 @@ struct nmd_handle {
   } pend[2];
   float* cur_R = nullptr;      // the copies of R, Rs and G the last step used
   float* cur_Rs = nullptr;
+  const uint8_t* cur_flags = nullptr;   // the support-row flags of the last step
   float* cur_G = nullptr;
   nmd::Workspace ws;
   nmd::Factor W, B;            // A = W (m x r), B = H^T (n x r)
@@ -180,9 +187,11 @@ void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge,
 void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole,
                    int64_t nwhole, const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti,
                    const int32_t* qidx, const float* vals, float* R, float* partials, cudaStream_t s);
-void launch_update(const StepArgs& a, const float* R, float* Rs, const float* Ginv, float eta,
-                   float gamma, bool momentum, int* status, cudaStream_t s);
-void launch_combine(float* R, float* Rs, int64_t n, cudaStream_t s);
+// flags: one byte per row of the step (Rs is read only where it is nonzero)
+void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags,
+                   const float* Ginv, float eta, float gamma, bool momentum, int* status,
+                   cudaStream_t s);
+void launch_combine(float* R, const float* Rs, const uint8_t* flags, int64_t rows, int rp, cudaStream_t s);
 void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s);
 void launch_loss_final(const double* dense_parts, int ndense, const double* sparse_parts,
                        int nsparse, double* out, cudaStream_t s);
