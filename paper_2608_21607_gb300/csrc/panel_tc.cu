@@ -554,8 +554,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         fence_after();
         const int64_t li = t * BM + row;
         float* dst = p.R + li * RP + (C::RHALF ? (int64_t)blockIdx.y * C::NR : 0);
+        constexpr int NJ = (C::NR + 31) / 32;
 #pragma unroll 1
-        for (int j = wg; j < (C::NR + 31) / 32; j += 2) {
+        for (int j = wg; j < NJ; j += 2) {
+          // the warp's last TMEM read of the tile releases R (MMA2 may start
+          // the next tile) before the adds and global stores
+          const bool last = j + 2 >= NJ;
           uint32_t v[32];
           tmem_ld32(tmem + lane_base + C::COL_R + j * 32, v);   // RP = 16 reads 16 spare columns
           if (C::FUSEDN) {
@@ -563,6 +567,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_ld32(tmem + lane_base + C::COL_R + RP + j * 32, u);
             tmem_wait_ld(v);
             tmem_wait_ld(u);
+            if (last) {
+              fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(b_rempty);
+            }
             if (RP == 16) {   // the accumulators are 16 columns apart: u[i] = v[i + 16]
 #pragma unroll
               for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + __uint_as_float(v[i + 16]));
@@ -572,6 +581,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           tmem_wait_ld(v);
+          if (!C::FUSEDN && last) {
+            fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(b_rempty);
+          }
           if (li < p.M) {
 #pragma unroll
             for (int i = 0; i < 32; i += 4)
@@ -580,9 +594,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                                           __uint_as_float(v[i + 2]), __uint_as_float(v[i + 3]));
           }
         }
-        fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(b_rempty);
+        if (wg >= NJ) {   // no columns for this warpgroup (r_pad = 16): release at once
+          fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(b_rempty);
+        }
       }
       // refill this tile's W buffer with the tile NWB steps ahead
       const int64_t tn = t + (int64_t)NWB * gridDim.x;
