@@ -247,6 +247,16 @@ nmd_status nmd_profile_read(nmd_handle* h, int32_t kernel_class, double* ms, int
  * the Gram matrix of nmd_block_terms to fp32 rounding (summation order). */
 nmd_status nmd_gram_noalloc(const float* d_Q, int64_t K, int32_t r, int64_t ld, float* d_G, void* stream);
 
+/* Verification hook for failure detection: runs the bounded wait that every
+ * pipeline wait of the tensor-core kernels uses (mbarrier polling with a
+ * globaltimer limit, after which the kernel records NMD_ERR_TIMEOUT in the
+ * sticky status, raises its abort flag and returns) on a barrier that nothing
+ * arrives at, with a limit of limit_ns (1 us .. 1 s; the kernels use 2 s).
+ * Synchronises; returns NMD_ERR_TIMEOUT when the wait gave up as designed
+ * (the status is cleared, the handle stays usable), NMD_ERR_INVALID for a
+ * limit out of range. */
+nmd_status nmd_selftest_wait_timeout(nmd_handle* h, int64_t limit_ns);
+
 /* Number of kernel launches this handle has issued (for launch accounting). */
 int64_t nmd_launch_count(const nmd_handle* h);
 

@@ -656,6 +656,16 @@ const char* nmd_last_error(const nmd_handle* h) { return h ? h->last_error.c_str
 
 int64_t nmd_launch_count(const nmd_handle* h) { return h ? h->launches : 0; }
 
+nmd_status nmd_selftest_wait_timeout(nmd_handle* h, int64_t limit_ns) {
+  if (!h || limit_ns < 1000 || limit_ns > 1000000000) return NMD_ERR_INVALID;
+  nmd_status st = sync_and_check(h);
+  if (st != NMD_OK) return st;
+  launch_wait_selftest(h->ws.status, (uint64_t)limit_ns, h->stream);
+  h->launches++;
+  if ((st = after_launch(h, "wait self-test")) != NMD_OK) return st;
+  return sync_and_check(h);
+}
+
 nmd_status nmd_skip_count(nmd_handle* h, int64_t* skipped, int32_t reset) {
   if (!h || !skipped) return NMD_ERR_INVALID;
   nmd_status st = sync_and_check(h);

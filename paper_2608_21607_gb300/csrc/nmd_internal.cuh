@@ -192,6 +192,8 @@ void launch_update(const StepArgs& a, const float* R, const float* Rs, const uin
                    const float* Ginv, float eta, float gamma, bool momentum, int* status,
                    cudaStream_t s);
 void launch_combine(float* R, const float* Rs, const uint8_t* flags, int64_t rows, int rp, cudaStream_t s);
+// the bounded pipeline wait, run on a barrier that never completes
+void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);
 void launch_loss_sparse(const nmd_handle* h, double* parts, int nparts, cudaStream_t s);
 void launch_loss_final(const double* dense_parts, int ndense, const double* sparse_parts,
                        int nsparse, double* out, cudaStream_t s);

@@ -127,12 +127,12 @@ __device__ __forceinline__ void record(int* status, int code, int detail) {
 // The polls suspend in hardware until the phase completes (or 20 us pass), so
 // waiting warps do not take issue slots from the MMA and copy threads.
 __device__ __noinline__ bool wait_bar_slow(uint32_t bar, uint32_t parity, volatile int* abort_flag, int* status,
-                                           int where) {
+                                           int where, uint64_t limit_ns = kTimeoutNs) {
   const uint64_t t0 = globaltimer_ns();
   for (;;) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort_flag) return false;
-    if (globaltimer_ns() - t0 > kTimeoutNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
       *abort_flag = 1;
       record(status, NMD_ERR_TIMEOUT, where);
       return false;
@@ -631,6 +631,23 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kProducerWarp) tmem_dealloc(tmem, 512);
 }
 
+// Self-test of the bounded wait used by every pipeline wait above: thread 0
+// waits on a barrier that nothing arrives at; after limit_ns the wait gives
+// up, sets the abort flag and records NMD_ERR_TIMEOUT (detail 99) in the
+// status words, and the kernel returns normally.
+__global__ void wait_selftest_kernel(int* status, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(smem_u32(&bar), 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) wait_bar_slow(smem_u32(&bar), 0, &abort_flag, status, 99, limit_ns);
+  __syncthreads();
+}
+
 // ---------------------------------------------------------------------------
 // host side
 // ---------------------------------------------------------------------------
@@ -744,6 +761,10 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
   nmd_status st = dispatch<false>(a.rp, a.epilogue, a.precision == NMD_FP32, *a.fm, *a.fq, p, grid, s);
   if (st == NMD_OK) ++*launches;
   return st;
+}
+
+void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s) {
+  wait_selftest_kernel<<<1, 32, 0, s>>>(status, limit_ns);
 }
 
 nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts, int* status,

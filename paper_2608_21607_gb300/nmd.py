@@ -30,7 +30,7 @@ EXPORTS = [
     "nmd_version", "nmd_default_options", "nmd_workspace_bytes", "nmd_create", "nmd_set_factors",
     "nmd_get_factors", "nmd_block_update", "nmd_sweep", "nmd_block_order", "nmd_loss", "nmd_sync",
     "nmd_block_terms", "nmd_dense_products", "nmd_panel_traversal", "nmd_get_state", "nmd_set_state",
-    "nmd_launch_count", "nmd_skip_count", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
+    "nmd_launch_count", "nmd_skip_count", "nmd_selftest_wait_timeout", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
     "nmd_destroy", "nmd_gram_noalloc",
 ]
 
@@ -88,6 +88,7 @@ def lib() -> C.CDLL:
             "nmd_set_state": (C.c_int, [_P, _P, _P, _P, _P, C.c_int64]),
             "nmd_launch_count": (C.c_int64, [_P]),
             "nmd_skip_count": (C.c_int, [_P, C.POINTER(C.c_int64), C.c_int32]),
+            "nmd_selftest_wait_timeout": (C.c_int, [_P, C.c_int64]),
             "nmd_profile": (C.c_int, [_P, C.c_int]),
             "nmd_profile_read": (C.c_int, [_P, C.c_int32, C.POINTER(C.c_double), _i64p]),
             "nmd_status_string": (C.c_char_p, [C.c_int]),
@@ -235,6 +236,11 @@ def nmd_set_state(h, W, H, EW, EH, sweep_index: int):
 
 def nmd_launch_count(h) -> int:
     return lib().nmd_launch_count(h)
+
+
+def nmd_selftest_wait_timeout(h, limit_ns: int) -> int:
+    """Status of the bounded-wait self-test (NMD_ERR_TIMEOUT when it works)."""
+    return int(lib().nmd_selftest_wait_timeout(h, int(limit_ns)))
 
 
 def nmd_skip_count(h, reset: bool = False) -> int:
