@@ -153,6 +153,8 @@ def main():
     ap.add_argument("--epilogue", choices=["z", "delta"], default="z")
     ap.add_argument("--skip-zero-chunks", action="store_true",
                     help="Delta form: skip the second product of chunks whose rectified tile is zero")
+    ap.add_argument("--schedule", choices=["workload", "exact", "stoch"], default="workload",
+                    help="sweep kind: the workload's own, or exact / stochastic")
     ap.add_argument("--init", choices=["normal", "paper"], default="normal",
                     help="factor start: iid N(0, 0.01), or the sign-structured start W > 0, H < 0")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing on the host")
@@ -205,7 +207,7 @@ def main():
     wl = WLm.workload(gen, seed=0)
     prec = {"bf16": N.NMD_BF16, "fp32": N.NMD_FP32}[args.precision]
     epi = {"z": N.NMD_EPI_Z, "delta": N.NMD_EPI_DELTA}[args.epilogue]
-    exact = wl.schedule == "exact"
+    exact = wl.schedule == "exact" if args.schedule == "workload" else args.schedule == "exact"
     sol = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols,
                    schedule=N.NMD_EXACT if exact else N.NMD_STOCH,
                    eta=wl.eta, gamma=wl.gamma, precision=prec, epilogue=epi, seed=0,

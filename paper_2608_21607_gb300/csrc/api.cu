@@ -280,6 +280,7 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->chol_scratch = c.take<float>((size_t)2 * rp * rp);
   w->seg_partials = c.take<float>((size_t)std::max<int64_t>(maxseg, 1) * rp);
   w->flags = c.take<uint8_t>((size_t)std::max<int64_t>(nflags, 1));
+  w->rpart = c.take<float>((size_t)kRpartRows * rp);
   w->loss_part = c.take<double>((size_t)kLossParts * 8);
   w->loss_out = c.take<double>(8);
   w->status = c.take<int>(kStatusWords);
@@ -562,7 +563,8 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
       launch_panel_simt(a, R, s);
       h->launches++;
     } else {
-      st = launch_panel_tc(a, R, h->ws.status, h->ws.counters, h->num_sms, s, &h->launches);
+      st = launch_panel_tc(a, R, h->ws.status, h->ws.counters, h->num_sms, s, &h->launches, nullptr, h->ws.rpart,
+                           kRpartRows);
     }
   }
   if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");

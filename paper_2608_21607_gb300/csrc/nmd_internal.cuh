@@ -112,9 +112,11 @@ struct Workspace {
   float* chol_scratch = nullptr;  // 2 x rp x rp (used when rp is too large for smem)
   float* seg_partials = nullptr;  // max segments x rp (sparse correction of long rows)
   uint8_t* flags = nullptr;       // the panels' support-row flags, concatenated
+  float* rpart = nullptr;         // kRpartRows x rp: partial R's of split-K steps
 };
 
 constexpr int kGramParts = 64;
+constexpr int64_t kRpartRows = 256 * 128;   // splits x tiles x 128 rows never exceed 256 SMs' worth
 constexpr int kLossParts = 2048;
 
 }  // namespace nmd
@@ -205,8 +207,11 @@ int launch_loss_dense_simt(const nmd_handle* h, double* parts, int maxparts, cud
 // ---- dense contraction on the tcgen05 tensor cores (panel_tc.cu) ----
 // Returns NMD_OK, or NMD_ERR_UNSUPPORTED when no tensor-core kernel exists
 // for this rank; `launches` is incremented by the number of kernels issued.
+// rpart (rpart_rows x rp floats, or nullptr): scratch for the partial R's of
+// a step whose K is split because it has fewer tiles than SMs
 nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counter,
-                           int num_sms, cudaStream_t s, int64_t* launches, float* Lout = nullptr);
+                           int num_sms, cudaStream_t s, int64_t* launches, float* Lout = nullptr,
+                           float* rpart = nullptr, int64_t rpart_rows = 0);
 nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts,
                                 int* status, cudaStream_t s, int64_t* launches);
 bool tc_supported(int rp, int precision);

@@ -34,6 +34,7 @@
 // and copies are drained and TMEM is freed before the kernel returns.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <map>
 #include <mutex>
 #include <tuple>
@@ -117,6 +118,10 @@ struct TcParams {
   const int32_t* cidx;
   unsigned long long* skips;   // Delta form: count of chunks whose second product was skipped (or nullptr)
   int skip_on;                 // Delta form: skip chunks whose rectified tile is zero
+  // split K (steps with fewer tiles than SMs): CTA z takes Q-side rows
+  // [q0 + z ksplit, ...) and writes its partial R at R + z rstride
+  int64_t ksplit;              // 0: no split
+  int64_t rstride;
 };
 
 __device__ __forceinline__ void record(int* status, int code, int detail) {
@@ -233,7 +238,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t tmem = *tmem_slot;
 
   const int64_t ntiles = (p.M + BM - 1) / BM;
-  const int64_t nchunks = (p.K + BN - 1) / BN;
+  const int64_t kz = blockIdx.z;
+  const int64_t kq0 = p.ksplit ? p.q0 + kz * p.ksplit : p.q0;       // this CTA's Q-side rows
+  const int64_t kK = p.ksplit ? (p.K - kz * p.ksplit < p.ksplit ? p.K - kz * p.ksplit : p.ksplit) : p.K;
+  float* const Rout = p.ksplit ? p.R + kz * p.rstride : p.R;
+  const int64_t nchunks = (kK + BN - 1) / BN;
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
@@ -247,7 +256,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             break;
           mbar_expect_tx(b_full + 8 * s, C::STAGE_BYTES);
           const uint32_t dst = smem_u32(stages + (size_t)s * C::STAGE_BYTES);
-          const int y = (int)(p.q0 + c * BN);
+          const int y = (int)(kq0 + c * BN);
 #pragma unroll
           for (int pn = 0; pn < C::NPANEL; ++pn) {
             tma_load_2d(dst + pn * C::PANEL_BYTES, &tq_hi, b_full + 8 * s, pn * C::PANEL_W, y);
@@ -447,7 +456,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int lb = (int)(G % NB);
         if (!(ok = warp_wait(b_lfull + 8 * lb, (uint32_t)((G / NB) & 1), abort_flag, p.status, 7))) break;
         fence_after();
-        const int kv = (int)(p.K - c * BN < BN ? p.K - c * BN : BN);   // valid columns in this chunk
+        const int kv = (int)(kK - c * BN < BN ? kK - c * BN : BN);   // valid columns in this chunk
         const uint32_t lcol = tmem + lane_base + C::COL_L + lb * BN;
         float c2 = 0.f, c1 = 0.f;
         uint32_t nzacc = 0u;   // Delta form: OR of this thread's P words
@@ -553,7 +562,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (!(ok = warp_wait(b_rfull, (uint32_t)(tt & 1), abort_flag, p.status, 8))) break;
         fence_after();
         const int64_t li = t * BM + row;
-        float* dst = p.R + li * RP + (C::RHALF ? (int64_t)blockIdx.y * C::NR : 0);
+        float* dst = Rout + li * RP + (C::RHALF ? (int64_t)blockIdx.y * C::NR : 0);
         constexpr int NJ = (C::NR + 31) / 32;
 #pragma unroll 1
         for (int j = wg; j < NJ; j += 2) {
@@ -709,7 +718,9 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
       return NMD_ERR_CUDA;
     attr_set = true;
   }
-  panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u), kThreads, C::SMEM, s>>>(th, tl, tl2, p);
+  const unsigned gz = p.ksplit ? (unsigned)((p.K + p.ksplit - 1) / p.ksplit) : 1u;
+  panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u, gz), kThreads, C::SMEM, s>>>(
+      th, tl, tl2, p);
   return NMD_OK;
 }
 
@@ -748,19 +759,54 @@ bool tc_supported(int rp, int precision) {
   return rp == 16 || rp == 32 || rp == 64 || rp == 128 || rp == 256;
 }
 
+// R = sum over the splits of the partial R's, in split order
+__global__ void split_reduce_kernel(const float* __restrict__ part, int64_t stride, int splits,
+                                    float* __restrict__ R, int64_t n) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+    float v = part[i];
+    for (int z = 1; z < splits; ++z) v += part[z * stride + i];
+    R[i] = v;
+  }
+}
+
 nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counter, int num_sms, cudaStream_t s,
-                           int64_t* launches, float* Lout) {
+                           int64_t* launches, float* Lout, float* rpart, int64_t rpart_rows) {
   if (!tc_supported(a.rp, a.precision)) return NMD_ERR_UNSUPPORTED;
   TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout, nullptr, nullptr,
-             (unsigned long long*)counter, a.skip_zero ? 1 : 0};
-  // fewest CTAs that keep the same number of tile rounds: the SMs left over
-  // run the side-stream kernels of the step
+             (unsigned long long*)counter, a.skip_zero ? 1 : 0, 0, 0};
   const int64_t ntiles = (a.M + BM - 1) / BM;
-  const int64_t rounds = (ntiles + num_sms - 1) / num_sms;
-  const int grid = (int)((ntiles + rounds - 1) / rounds);
+  // a step with fewer tiles than SMs (the exact steps: b rows against all of
+  // the other factor) splits K so that tiles x splits fill the SMs, each split
+  // keeping at least 8 chunks; the partial R's are summed in split order
+  int64_t splits = 1;
+  if (Lout == nullptr && rpart != nullptr && ntiles < num_sms) {
+    splits = std::min<int64_t>({(int64_t)num_sms / ntiles, (a.K + 64 * 8 - 1) / (64 * 8), 16,
+                                rpart_rows / (ntiles * BM)});
+    if (splits < 2) splits = 1;
+  }
+  int grid;
+  if (splits > 1) {
+    p.ksplit = ((a.K + splits - 1) / splits + 127) / 128 * 128;   // whole chunks of 64 or 128 rows
+    splits = (a.K + p.ksplit - 1) / p.ksplit;
+    p.R = rpart;
+    p.rstride = a.M * a.rp;
+    grid = (int)ntiles;
+  } else {
+    // fewest CTAs that keep the same number of tile rounds: the SMs left over
+    // run the side-stream kernels of the step
+    const int64_t rounds = (ntiles + num_sms - 1) / num_sms;
+    grid = (int)((ntiles + rounds - 1) / rounds);
+  }
   nmd_status st = dispatch<false>(a.rp, a.epilogue, a.precision == NMD_FP32, *a.fm, *a.fq, p, grid, s);
-  if (st == NMD_OK) ++*launches;
-  return st;
+  if (st != NMD_OK) return st;
+  ++*launches;
+  if (splits > 1) {
+    const int64_t n = a.M * a.rp;
+    const int64_t blocks = std::min<int64_t>((n + 255) / 256, (int64_t)num_sms * 8);
+    split_reduce_kernel<<<(unsigned)blocks, 256, 0, s>>>(rpart, p.rstride, (int)splits, R, n);
+    ++*launches;
+  }
+  return NMD_OK;
 }
 
 void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s) {
@@ -771,7 +817,7 @@ nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts
                                 cudaStream_t s, int64_t* launches) {
   if (!tc_supported(h->rp, h->opt.precision)) return NMD_ERR_UNSUPPORTED;
   TcParams p{0, h->m, 0, h->n, h->W.hi, h->W.lo, nullptr, parts, status, nullptr, h->ws.rowptr, h->ws.col,
-             nullptr, 0};
+             nullptr, 0, 0, 0};
   int64_t ntiles = (h->m + BM - 1) / BM;
   int grid = (int)(ntiles < h->num_sms ? ntiles : h->num_sms);
   if (grid > maxparts) grid = maxparts;
