@@ -277,6 +277,8 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->Ginv = c.take<float>((size_t)rp * rp);
   w->G2 = c.take<float>((size_t)rp * rp);
   w->Ginv2 = c.take<float>((size_t)rp * rp);
+  w->Gc = c.take<float>((size_t)rp * rp);
+  w->Ginvc = c.take<float>((size_t)rp * rp);
   w->chol_scratch = c.take<float>((size_t)2 * rp * rp);
   w->seg_partials = c.take<float>((size_t)std::max<int64_t>(maxseg, 1) * rp);
   w->flags = c.take<uint8_t>((size_t)std::max<int64_t>(nflags, 1));
@@ -359,6 +361,7 @@ nmd_status sync_and_check(nmd_handle* h) {
   int st[kStatusWords];
   CK(h, cudaMemcpy(st, h->ws.status, sizeof st, cudaMemcpyDeviceToHost));
   if (st[0] != 0) {
+    h->gcache_f = -1;   // a failed step may have left the cached Gram unusable
     CK(h, cudaMemset(h->ws.status, 0, sizeof st));
     char b[192];
     snprintf(b, sizeof b, "%s (device detail %d, at block step %d)", status_name(st[0]), st[1], st[2]);
@@ -524,6 +527,16 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   float* Rs = par ? h->ws.Rs2 : h->ws.Rs;
   float* G = par ? h->ws.G2 : h->ws.G;
   float* Ginv = par ? h->ws.Ginv2 : h->ws.Ginv;
+  // an exact step's Q side is a whole factor: every block of a half-sweep has
+  // the same G, computed once and kept until that factor changes
+  bool need_gram = true;
+  if (kind == NMD_EXACT) {
+    G = h->ws.Gc;
+    Ginv = h->ws.Ginvc;
+    need_gram = !(h->gcache_f == fq && h->gcache_ver == h->fver[fq]);
+    h->gcache_f = fq;
+    h->gcache_ver = h->fver[fq];
+  }
   h->cur_R = R;
   h->cur_Rs = Rs;
   h->cur_G = G;
@@ -533,7 +546,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 127) / 128));
   CK(h, cudaEventRecord(h->ev_fork, s));
   CK(h, cudaStreamWaitEvent(h->side, h->ev_fork, 0));
-  {
+  if (need_gram) {
     TimedScope ts(h, NMD_K_GRAM, h->side);
     launch_gram(*ro.fq, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, h->side);
     launch_chol_inv(h->ws.gram_part, nparts, h->r, h->rp, (float)h->opt.ridge, G, Ginv, h->ws.chol_scratch,
@@ -600,6 +613,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
     }
     if ((st = after_launch(h, "update")) != NMD_OK) return st;
   }
+  if (do_update) h->fver[fm]++;
   h->step_index++;
   return NMD_OK;
 }
@@ -811,6 +825,8 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
 
 nmd_status nmd_set_factors(nmd_handle* h, const float* W, const float* H, int on_device) {
   if (!h || !W || !H) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_set_factors");
+  h->fver[0]++;
+  h->fver[1]++;
   cudaStream_t s = h->stream;
   cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
   // stage through R (max(m, n) x rp floats >= m x r and r x n)

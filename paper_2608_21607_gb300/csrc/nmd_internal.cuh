@@ -105,6 +105,8 @@ struct Workspace {
   float* Ginv = nullptr;       // rp x rp
   float* G2 = nullptr;
   float* Ginv2 = nullptr;
+  float* Gc = nullptr;         // G and G^{-1} of an exact step's Q side (all of one factor),
+  float* Ginvc = nullptr;      // kept while that factor is unchanged
   double* loss_part = nullptr; // kLossParts x 8
   double* loss_out = nullptr;  // 8
   int* status = nullptr;       // kStatusWords
@@ -148,6 +150,11 @@ struct nmd_handle {
     int64_t a0 = 0, a1 = 0, b0 = 0, b1 = 0;   // rows [a0, a1) and [b0, b1) in flight
     cudaEvent_t ev = nullptr;
   } pend[2];
+  // version of each factor (0 = W, 1 = B), advanced by every write to it, and
+  // the factor and version the cached exact-step Gram belongs to
+  int64_t fver[2] = {0, 0};
+  int gcache_f = -1;
+  int64_t gcache_ver = -1;
   float* cur_R = nullptr;      // the copies of R, Rs and G the last step used
   float* cur_Rs = nullptr;
   const uint8_t* cur_flags = nullptr;   // the support-row flags of the last step
