@@ -66,10 +66,18 @@ struct Cfg {
   static constexpr int NR = RHALF ? RP / 2 : RP;        // R columns of one CTA
   // TMEM columns of the R accumulator(s); the loss pass has none
   static constexpr int RCOLS = LOSS ? 0 : (FUSEDN ? 2 * RP : NR);
+  // bf16 mode, r_pad <= 128: the W tile is the first product's A operand
+  // from shared memory (loaded by TMA) instead of TMEM.  At r_pad <= 64 that
+  // leaves room for three L buffers of 128 columns: chunks of 128 Q rows
+  // halve the hand-offs (barrier waits and commits) per row and the first
+  // product's MMA count.  At r_pad = 128 it gives four L buffers of 64.
+  static constexpr bool WSMEM = FUSEDN;
   // Q rows per chunk.  64 where the TMEM budget would otherwise leave only
   // two L buffers: more chunks in flight hide the epilogue's latency.
-  static constexpr int BN = (RP == 256 || (SPLIT && RP == 128) || FUSEDN) ? 64 : 128;
-  static constexpr int WCOLS = SPLIT ? RP : RP / 2;    // TMEM columns of one W tile (hi [+ lo])
+  static constexpr int BN = WSMEM ? (RP == 128 ? 64 : 128) : ((RP == 256 || (SPLIT && RP == 128)) ? 64 : 128);
+  // TMEM columns of one W tile (hi [+ lo]); none when it sits in shared memory
+  static constexpr int WCOLS = WSMEM ? 0 : (SPLIT ? RP : RP / 2);
+  static constexpr int W_BYTES = WSMEM ? BM * RP * 2 : 0;   // one W tile in shared memory
   static constexpr int NWB = (RP == 256) ? 1 : 2;      // W tile buffers
   static constexpr int FREE = 512 - NWB * WCOLS - RCOLS;
   static constexpr int NB = FREE / BN >= 6 ? 6 : FREE / BN;  // L buffers
@@ -83,9 +91,13 @@ struct Cfg {
   // (first product only) needs hi (+ lo when split)
   static constexpr int NQ = LOSS ? (SPLIT ? 2 : 1) : (SPLIT ? 3 : 2);
   static constexpr int STAGE_BYTES = OPER_BYTES * NQ;
-  static constexpr int NSTAGE_RAW = (160 * 1024) / STAGE_BYTES;
+  static constexpr int NSTAGE_RAW = (WSMEM ? 192 * 1024 - NWB * W_BYTES : 160 * 1024) / STAGE_BYTES;
   static constexpr int NSTAGE = NSTAGE_RAW > 8 ? 8 : (NSTAGE_RAW < 2 ? 2 : NSTAGE_RAW);
   static constexpr uint32_t SWZ = PANEL_W == 64 ? SWZ_128B : (PANEL_W == 32 ? SWZ_64B : SWZ_32B);
+  // shared memory: stages, W tiles (WSMEM), barriers, TMEM slot + abort flag, ...
+  static constexpr size_t OFF_W = (size_t)NSTAGE * STAGE_BYTES;
+  static constexpr int W_PANEL_BYTES = BM * ROWB;     // one swizzle panel of a W tile
+  static constexpr size_t OFF_BARS = OFF_W + (size_t)NWB * W_BYTES;
   static constexpr int COL_L = 0;               // NB x BN columns
   static constexpr int COL_R = NB * BN;         // RP columns
   static constexpr int COL_W = COL_R + RCOLS;   // NWB x WCOLS columns
@@ -94,7 +106,7 @@ struct Cfg {
   static constexpr int NBAR = 2 * NSTAGE + 3 * NB + 8;
   // after the barriers: TMEM slot and abort flag (64 B), the loss reduction
   // (256 x 16 B), and 4 flags per L buffer (Delta form: P nonzero per warp)
-  static constexpr size_t SMEM_USED = 1024 + (size_t)NSTAGE * STAGE_BYTES + NBAR * 8 + 64 + 256 * 16 + NB * 16;
+  static constexpr size_t SMEM_USED = 1024 + OFF_BARS + NBAR * 8 + 64 + 256 * 16 + NB * 16;
   // at least 120 KB so that a second CTA (and its 512-column TMEM request)
   // never shares the SM
   static constexpr size_t SMEM = SMEM_USED > 120 * 1024 ? SMEM_USED : 120 * 1024;
@@ -177,16 +189,18 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 template <int RP, int EPI, bool SPLIT, bool LOSS, bool SKIP>
 __global__ void __launch_bounds__(kThreads, 1)
     panel_tc_kernel(const __grid_constant__ CUtensorMap tq_hi, const __grid_constant__ CUtensorMap tq_lo,
-                    const __grid_constant__ CUtensorMap tq_lo2, const TcParams p) {
+                    const __grid_constant__ CUtensorMap tq_lo2, const __grid_constant__ CUtensorMap tw,
+                    const TcParams p) {
   using C = Cfg<RP, SPLIT, LOSS>;
   constexpr int BN = C::BN, NB = C::NB, NSTAGE = C::NSTAGE, NWB = C::NWB;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* stages = smem;
-  uint64_t* bars = (uint64_t*)(smem + (size_t)NSTAGE * C::STAGE_BYTES);
+  const uint32_t wsm0 = smem_u32(smem + C::OFF_W);    // W tiles (WSMEM)
+  uint64_t* bars = (uint64_t*)(smem + C::OFF_BARS);
   uint32_t* tmem_slot = (uint32_t*)(bars + C::NBAR);
   volatile int* abort_flag = (volatile int*)(tmem_slot + 1);
-  double* red = (double*)(smem + (size_t)NSTAGE * C::STAGE_BYTES + C::NBAR * 8 + 64);
+  double* red = (double*)(smem + C::OFF_BARS + C::NBAR * 8 + 64);
   volatile uint32_t* pflag = (volatile uint32_t*)(red + 2 * kEpiThreads);   // [NB][4]
 
   const uint32_t b_full = smem_u32(bars);
@@ -215,7 +229,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(b_rfull, 1);
     mbar_init(b_rempty, kEpiThreads / 32);
     for (int i = 0; i < 2; ++i) {
-      mbar_init(b_wfull + 8 * i, kEpiThreads / 32);
+      mbar_init(b_wfull + 8 * i, C::WSMEM ? 1 : kEpiThreads / 32);   // TMA, or the epilogue warps
       mbar_init(b_wempty + 8 * i, 1);
     }
     mbar_init(b_drain, 1);
@@ -230,6 +244,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       prefetch_tmap(&tq_hi);
       if (C::NQ > 1) prefetch_tmap(&tq_lo);
       if (C::NQ > 2) prefetch_tmap(&tq_lo2);
+      if (C::WSMEM) prefetch_tmap(&tw);
     }
   }
   fence_before();
@@ -247,9 +262,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
-      int64_t G = 0;
+      int64_t G = 0, tt = 0;
       bool ok = true;
-      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++tt) {
+        if (C::WSMEM) {   // the tile's W rows into W buffer tt % NWB once MMA1 is done with it
+          const int wb = (int)(tt % NWB);
+          if (!(ok = wait_bar(b_wempty + 8 * wb, (uint32_t)((tt / NWB) & 1) ^ 1u, abort_flag, p.status, 10)))
+            break;
+          mbar_expect_tx(b_wfull + 8 * wb, C::W_BYTES);
+#pragma unroll
+          for (int pn = 0; pn < C::NPANEL; ++pn)
+            tma_load_2d(wsm0 + wb * C::W_BYTES + pn * C::W_PANEL_BYTES, &tw, b_wfull + 8 * wb, pn * C::PANEL_W,
+                        (int)(p.m0 + t * BM));
+        }
         for (int64_t c = 0; c < nchunks; ++c, ++G) {
           const int s = (int)(G % NSTAGE);
           if (!(ok = wait_bar(b_empty + 8 * s, (uint32_t)((G / NSTAGE) & 1) ^ 1u, abort_flag, p.status, 1)))
@@ -275,6 +300,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                  globaltimer_ns() - t0 < 100000000ull) {
           }
         }
+        // W loads: those of tiles [0, tt) were issued, only the last NWB can
+        // still be in flight
+        for (int64_t k = tt - NWB > 0 ? tt - NWB : 0; C::WSMEM && k < tt; ++k) {
+          uint64_t t0 = globaltimer_ns();
+          while (!mbar_try_wait(b_wfull + 8 * (int)(k % NWB), (uint32_t)((k / NWB) & 1)) &&
+                 globaltimer_ns() - t0 < 100000000ull) {
+          }
+        }
       }
     }
   } else if (warp == kMma1Warp) {
@@ -296,12 +329,18 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t wh = tmem + C::COL_W + wb1 * C::WCOLS;
       const uint32_t wl = wh + RP / 2;
       const uint64_t d1 = sdesc(stage0 + s1 * C::STAGE_BYTES, 16, 8 * C::ROWB, C::SWZ);
+      // WSMEM: the W tile in the same K-major swizzled panels as a chunk
+      const uint64_t a1 = sdesc(wsm0 + wb1 * C::W_BYTES, 16, 8 * C::ROWB, C::SWZ);
       const uint32_t d = tmem + C::COL_L + l1 * BN;
 #pragma unroll
       for (int k = 0; k < RP / 16; ++k) {
         const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
         const uint64_t bh = d1 + (off >> 4);
-        mma_ts_elect(d, wh + k * 8, bh, idesc1, k > 0);
+        if (C::WSMEM)
+          mma_ss_elect(d, a1 + (((k * 16 / C::PANEL_W) * C::W_PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2) >> 4), bh,
+                       idesc1, k > 0);
+        else
+          mma_ts_elect(d, wh + k * 8, bh, idesc1, k > 0);
         if (SPLIT) {
           const uint64_t bl = d1 + ((C::OPER_BYTES + off) >> 4);
           mma_ts_elect(d, wh + k * 8, bl, idesc1, 1);
@@ -408,6 +447,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     // load the W tile `tile` into W buffer wb: warpgroup g takes 8-word groups g, g+2, ...
     auto load_w = [&](int64_t tile, int wb) {
+      if constexpr (C::WSMEM) return;   // loaded by the producer's TMA
       const int64_t li = tile * BM + row;
       const bool valid = li < p.M;
       const uint4* src = (const uint4*)(p.Mhi + (p.m0 + (valid ? li : 0)) * RP);
@@ -611,7 +651,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // refill this tile's W buffer with the tile NWB steps ahead
       const int64_t tn = t + (int64_t)NWB * gridDim.x;
-      if (tn < ntiles) {
+      if (!C::WSMEM && tn < ntiles) {
         const int wb = (int)(tt % NWB);
         if (!(ok = warp_wait(b_wempty + 8 * wb, (uint32_t)((tt / NWB) & 1), abort_flag, p.status, 9))) break;
         fence_after();
@@ -710,7 +750,10 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
   if (!tensor_map(fq.hi, fq.rows, RP, C::PANEL_W, C::BN, &th)) return NMD_ERR_CUDA;
   if (!tensor_map(fq.lo, fq.rows, RP, C::PANEL_W, C::BN, &tl)) return NMD_ERR_CUDA;
   if (!tensor_map(fq.lo2, fq.rows, RP, C::PANEL_W, C::BN, &tl2)) return NMD_ERR_CUDA;
-  (void)fm;
+  // W tiles: the M-side rows [0, m0 + M) of the M factor's bf16 copy, so
+  // that the rows of a ragged last tile past the block read as zero
+  CUtensorMap tw = th;
+  if (C::WSMEM && !tensor_map(fm.hi, p.m0 + p.M, RP, C::PANEL_W, BM, &tw)) return NMD_ERR_CUDA;
   static bool attr_set = false;
   if (!attr_set) {
     if (cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -720,7 +763,7 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
   }
   const unsigned gz = p.ksplit ? (unsigned)((p.K + p.ksplit - 1) / p.ksplit) : 1u;
   panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u, gz), kThreads, C::SMEM, s>>>(
-      th, tl, tl2, p);
+      th, tl, tl2, tw, p);
   return NMD_OK;
 }
 
