@@ -91,7 +91,11 @@ struct Cfg {
   // (first product only) needs hi (+ lo when split)
   static constexpr int NQ = LOSS ? (SPLIT ? 2 : 1) : (SPLIT ? 3 : 2);
   static constexpr int STAGE_BYTES = OPER_BYTES * NQ;
-  static constexpr int NSTAGE_RAW = (WSMEM ? 160 * 1024 - NWB * W_BYTES : 160 * 1024) / STAGE_BYTES;
+  // stages within 160 KB with the W tiles (r_pad <= 64: 165 KB in all, so
+  // that an update block fits beside the CTA), 192 KB at r_pad = 128
+  static constexpr int NSTAGE_RAW =
+      ((WSMEM && RP <= 64) ? 160 * 1024 - NWB * W_BYTES : (WSMEM ? 192 * 1024 - NWB * W_BYTES : 160 * 1024)) /
+      STAGE_BYTES;
   static constexpr int NSTAGE = NSTAGE_RAW > 8 ? 8 : (NSTAGE_RAW < 2 ? 2 : NSTAGE_RAW);
   static constexpr uint32_t SWZ = PANEL_W == 64 ? SWZ_128B : (PANEL_W == 32 ? SWZ_64B : SWZ_32B);
   // shared memory: stages, W tiles (WSMEM), barriers, TMEM slot + abort flag, ...
