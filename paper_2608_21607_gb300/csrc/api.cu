@@ -355,6 +355,7 @@ const char* status_name(int s) {
 nmd_status sync_and_check(nmd_handle* h) {
   CK(h, cudaStreamSynchronize(h->stream));
   if (h->side) CK(h, cudaStreamSynchronize(h->side));
+  if (h->side2) CK(h, cudaStreamSynchronize(h->side2));
   if (h->aux) CK(h, cudaStreamSynchronize(h->aux));
   if (h->hp) CK(h, cudaStreamSynchronize(h->hp));
   h->pend[0].active = h->pend[1].active = false;
@@ -540,12 +541,14 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   h->cur_R = R;
   h->cur_Rs = Rs;
   h->cur_G = G;
-  // The side stream computes G = Q^T Q of the Q-side rows, G^{-1}, and the
-  // support term Rs of R; the main stream the dense term of R.  Neither reads
-  // what the other writes, so they overlap; the update joins them.
+  // The side stream computes G = Q^T Q of the Q-side rows and G^{-1}, the
+  // second side stream the support term Rs of R, the main stream the dense
+  // term of R.  None reads what another writes, so they overlap; the update
+  // joins them.
   int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 127) / 128));
   CK(h, cudaEventRecord(h->ev_fork, s));
   CK(h, cudaStreamWaitEvent(h->side, h->ev_fork, 0));
+  CK(h, cudaStreamWaitEvent(h->side2, h->ev_fork, 0));
   if (need_gram) {
     TimedScope ts(h, NMD_K_GRAM, h->side);
     launch_gram(*ro.fq, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, h->side);
@@ -562,13 +565,14 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   const uint8_t* flags = P.d_flags + P.flag_off[block];
   h->cur_flags = flags;
   {
-    TimedScope ts(h, NMD_K_SPARSE, h->side);
+    TimedScope ts(h, NMD_K_SPARSE, h->side2);
     launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, gd - g0, P.d_seg + gd, g1 - gd, P.d_multi + u0, u1 - u0,
-                  ro.qidx, ro.vals, Rs, h->ws.seg_partials, h->side);
+                  ro.qidx, ro.vals, Rs, h->ws.seg_partials, h->side2);
     h->launches += (r1 > r0) + (gd > g0) + 2 * (g1 > gd);
   }
   if ((st = after_launch(h, "sparse correction")) != NMD_OK) return st;
   CK(h, cudaEventRecord(h->ev_join, h->side));
+  CK(h, cudaEventRecord(h->ev_join2, h->side2));
   // dense Z-panel contraction R = P(L) Q over every (M-side, Q-side) pair
   {
     TimedScope ts(h, NMD_K_DENSE);
@@ -583,6 +587,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
   if ((st = after_launch(h, "dense panel")) != NMD_OK) return st;
   CK(h, cudaStreamWaitEvent(s, h->ev_join, 0));
+  CK(h, cudaStreamWaitEvent(s, h->ev_join2, 0));
   if (do_update) {
     const bool momentum = kind == NMD_STOCH;
     // rows [lo, hi) (relative to m0) are updated on the main stream; when the
@@ -622,6 +627,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
 
 nmd_handle::~nmd_handle() {
   if (side) cudaStreamSynchronize(side);
+  if (side2) cudaStreamSynchronize(side2);
   if (aux) cudaStreamSynchronize(aux);
   if (!timed.empty()) cudaStreamSynchronize(stream);
   for (auto& t : timed) {
@@ -631,7 +637,9 @@ nmd_handle::~nmd_handle() {
   for (cudaEvent_t e : event_pool) cudaEventDestroy(e);
   if (ev_fork) cudaEventDestroy(ev_fork);
   if (ev_join) cudaEventDestroy(ev_join);
+  if (ev_join2) cudaEventDestroy(ev_join2);
   if (side) cudaStreamDestroy(side);
+  if (side2) cudaStreamDestroy(side2);
   if (ev_prio) cudaEventDestroy(ev_prio);
   for (auto& p : pend)
     if (p.ev) cudaEventDestroy(p.ev);
@@ -803,10 +811,12 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   int least = 0, greatest = 0;
   e = cudaDeviceGetStreamPriorityRange(&least, &greatest);
   if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side, cudaStreamNonBlocking, greatest);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side2, cudaStreamNonBlocking, greatest);
   if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->hp, cudaStreamNonBlocking, greatest);
   if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->aux, cudaStreamNonBlocking, least);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_join2, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_in, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_out, cudaEventDisableTiming);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_prio, cudaEventDisableTiming);

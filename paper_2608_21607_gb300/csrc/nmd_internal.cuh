@@ -128,10 +128,11 @@ struct nmd_handle {
   int r = 0, rp = 0;
   nmd_options opt;
   cudaStream_t stream = nullptr;
-  // the Gram chain runs on a second stream, forked from and joined back into
-  // `stream` around the dense kernel of each step
-  cudaStream_t side = nullptr;
-  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // the Gram chain (G, G^{-1}) and the support term run on two more streams,
+  // forked from and joined back into `stream` around the dense kernel of
+  // each step
+  cudaStream_t side = nullptr, side2 = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr, ev_join2 = nullptr;
   // Within a sweep, the rows of a step's update that the next step does not
   // read are updated on `aux`, overlapping the next step.  pend[f] records,
   // for factor f (0 = W, 1 = B), the rows such an update may still be
