@@ -273,6 +273,66 @@ def test_identity_has_rank3_completion_omega():
     np.testing.assert_allclose(st.A @ st.B.T, Om, atol=1e-7)
 
 
+def _fixed_point_checks(D, W, H, block, stoch_block=None):
+    """The oracle at a zero-loss point of S = D: zero objective, and an exact
+    and a stochastic sweep (eta = 1) leave the model L = W H unchanged.  The
+    stochastic blocks must span the factor's column space (their Gram
+    matrices must be invertible)."""
+    S = WL.csr_from_dense(D, dtype=np.float64)
+    L0 = W @ H
+    for sched in (O.EXACT, O.STOCH):
+        b = block if sched == O.EXACT or stoch_block is None else stoch_block
+        st = O.State(S, W, H, O.Options(block_rows=b, block_cols=b, schedule=sched, eta=1.0,
+                                        gamma=0.9 if sched == O.STOCH else 0.0))
+        assert st.loss()["obj"] < 1e-12
+        st.sweep()
+        assert st.loss()["obj"] < 1e-10
+        np.testing.assert_allclose(st.A @ st.B.T, L0, atol=1e-9)
+
+
+@pytest.mark.parametrize("delta", [0.25, 0.5])
+def test_ring_graph_rank3_completion_is_fixed(delta):
+    """Prop. 'ring' (eqs. ring, ringvecs, tau, r2): with unit-spaced points on a
+    circle of radius r and the threshold tau, the thresholded similarities
+    reproduce the ring matrix (1 on the diagonal, delta between neighbours,
+    0 elsewhere) as max(0, L) with rank(L) = 3; the oracle must treat that
+    point as an exact, fixed completion."""
+    n = 40
+    phi = 2 * np.pi / n
+    tau = (np.cos(phi) - delta) / (1 - delta)
+    r2 = (1 - delta) / (1 - np.cos(phi))
+    th = phi * np.arange(n)
+    r = np.sqrt(r2)
+    W = np.stack([r * np.cos(th), r * np.sin(th), -tau * r2 * np.ones(n)], 1)
+    H = np.stack([r * np.cos(th), r * np.sin(th), np.ones(n)], 1).T
+    i, j = np.meshgrid(np.arange(n), np.arange(n), indexing="ij")
+    d = np.abs(i - j)
+    D = np.where(d == 0, 1.0, np.where((d == 1) | (d == n - 1), delta, 0.0))
+    np.testing.assert_allclose(np.maximum(0, W @ H), D, atol=1e-12)
+    assert np.linalg.matrix_rank(W @ H) == 3
+    _fixed_point_checks(D, W, H, 8)
+
+
+def test_hypercube_rank_d_plus_1_completion_is_fixed():
+    """Prop. 'hypercube' (eq. hypercube): with alpha_i = r v_i on the vertices
+    v_i of the d-cube, r^2 = (1 - delta) / 2 and tau = 1 - 2 / (d (1 - delta)),
+    max(0, L) is 1 on the diagonal, delta between vertices at distance 2 and 0
+    otherwise, with rank(L) <= d + 1."""
+    dim, delta = 5, 0.1
+    V = np.array([[1.0 if (k >> b) & 1 else -1.0 for b in range(dim)] for k in range(2 ** dim)])
+    r2 = (1 - delta) / 2
+    tau = 1 - 2 / (dim * (1 - delta))
+    W = np.hstack([np.sqrt(r2) * V, -tau * r2 * dim * np.ones((2 ** dim, 1))])
+    H = np.hstack([np.sqrt(r2) * V, np.ones((2 ** dim, 1))])
+    dist2 = ((V[:, None, :] - V[None, :, :]) ** 2).sum(-1)
+    D = np.where(dist2 == 0, 1.0, np.where(dist2 == 4, delta, 0.0))
+    np.testing.assert_allclose(np.maximum(0, W @ H.T), D, atol=1e-12)
+    assert np.linalg.matrix_rank(W @ H.T) == dim + 1
+    # a block of 8 or 16 consecutive vertices fixes the top coordinates, so its
+    # rows of [r v, 1] are rank deficient: stochastic blocks take the whole cube
+    _fixed_point_checks(D, W, H.T, 8, stoch_block=2 ** dim)
+
+
 def test_loss_of_all_zero_model_is_one():
     """Sec. 3.1: RMSE(S, 0) = WJD(S, 0) = 1; with L = 0, Z = S so the objective is 1 too."""
     S, _ = _rand_sparse(20, 30, 0.2, 6)
