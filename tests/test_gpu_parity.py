@@ -224,6 +224,32 @@ def test_identity_omega_point_is_fixed(prec):
     assert rel(W @ H, W0.astype(np.float64) @ H0) < 1e-3
 
 
+@pytest.mark.parametrize("prec", [N.NMD_SIMT, N.NMD_FP32], ids=lambda p: PREC_NAMES[p])
+def test_ring_point_is_fixed(prec):
+    """Prop. 'ring': the ring matrix (1 on the diagonal, delta = 1/2 between
+    neighbours) is max(0, L) for the rank-3 L of points on a circle of
+    radius r with threshold tau (eqs. tau, r2); support values other than 1
+    on the GPU path.  Products of size r^2 ~ 40 cancel to 0, 1/2 or 1, so
+    only the fp32-accurate paths are checked (as for eq. Omega)."""
+    n, delta = 48, 0.5
+    phi = 2 * np.pi / n
+    tau = (np.cos(phi) - delta) / (1 - delta)
+    r2 = (1 - delta) / (1 - np.cos(phi))
+    th = phi * np.arange(n)
+    r = np.sqrt(r2)
+    W0 = np.stack([r * np.cos(th), r * np.sin(th), -tau * r2 * np.ones(n)], 1).astype(np.float32)
+    H0 = np.stack([r * np.cos(th), r * np.sin(th), np.ones(n)], 0).astype(np.float32)
+    i, j = np.meshgrid(np.arange(n), np.arange(n), indexing="ij")
+    d = np.abs(i - j)
+    D = np.where(d == 0, 1.0, np.where((d == 1) | (d == n - 1), delta, 0.0))
+    sol = N.Solver(WL.csr_from_dense(D), 3, block_rows=16, block_cols=16, precision=prec, gamma=0.9)
+    sol.set_factors(W0, H0)
+    assert sol.loss()["obj"] < (1e-4 if prec == N.NMD_SIMT else 2e-3)
+    sol.sweep()
+    W, H = sol.get_factors()
+    assert rel(W @ H, W0.astype(np.float64) @ H0) < 1e-3
+
+
 def test_not_spd_is_reported_and_update_skipped():
     # 400 columns in blocks of 133: the last block has 1 column < r = 4
     S, _, _, _ = WL.planted(300, 400, 4, tau=0.5, seed=0)
