@@ -810,8 +810,9 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   }
   int least = 0, greatest = 0;
   e = cudaDeviceGetStreamPriorityRange(&least, &greatest);
-  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side, cudaStreamNonBlocking, greatest);
-  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side2, cudaStreamNonBlocking, greatest);
+  const int side_prio = greatest < least ? greatest + 1 : greatest;
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side, cudaStreamNonBlocking, side_prio);
+  if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->side2, cudaStreamNonBlocking, side_prio);
   if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->hp, cudaStreamNonBlocking, greatest);
   if (e == cudaSuccess) e = cudaStreamCreateWithPriority(&h->aux, cudaStreamNonBlocking, least);
   if (e == cudaSuccess) e = cudaEventCreateWithFlags(&h->ev_fork, cudaEventDisableTiming);
