@@ -142,6 +142,51 @@ def oracle_sample(wl, budget_s=20.0):
     return entries / t_used, len(done), t_used
 
 
+# The paper's kernel-throughput table (Sec. 4.2): the fused kernel on m =
+# 250000 rows against a block of n = 2500, TFLOP/s counted as 4 m n r
+# (both products), TF32 operands; H100 PCIe and RTX Pro 6000 figures.
+PAPER_KERNEL_TABLE = {16: (215.30, 191.72), 32: (283.73, 203.06), 64: (285.10, 206.11), 128: (279.19, 189.80)}
+
+
+def kernel_table(args):
+    """Each step here is one stochastic column step (all m rows of W against
+    a block of 2500 rows of B) run alone, synchronised after every step; the
+    dense kernel's own time comes from the library's CUDA-event profile."""
+    import numpy as np
+    import torch
+    from paper_2608_21607_gb300 import build as B
+    from paper_2608_21607_gb300 import nmd as N
+    from paper_2608_21607_gb300 import workloads as WLm
+    B.build()
+    m, nb = 250000, 2500
+    S = WLm.identity(m)
+    for prec_name, prec in (("bf16", N.NMD_BF16), ("fp32", N.NMD_FP32)):
+        for r in (16, 32, 64, 128):
+            W0, H0 = WLm.init_factors(m, m, r, 0)
+            sol = N.Solver(S, r, block_rows=nb, block_cols=nb, precision=prec, eta=0.5, gamma=0.0)
+            sol.set_factors(W0, H0)
+            for b in range(args.warmup):
+                sol.block_update(N.NMD_COL, b, N.NMD_STOCH)
+                sol.sync()
+            sol.profile(True)
+            for b in range(args.steps):
+                sol.block_update(N.NMD_COL, args.warmup + b, N.NMD_STOCH)
+                sol.sync()
+            ms, n = sol.profile_read(N.NMD_K_DENSE)
+            sol.profile(False)
+            us = 1e3 * ms / n
+            tf = 4.0 * m * nb * r / (us * 1e-6) / 1e12
+            h100, rtx = PAPER_KERNEL_TABLE[r]
+            print(json.dumps({"metric": "dense kernel TFLOP/s at the paper's kernel-table shape (4 m n r per launch)",
+                              "value": tf, "unit": "TFLOP/s", "higher_is_better": True, "r": r,
+                              "dtype": prec_name, "m": m, "block": nb, "launches": n, "us_per_launch": us,
+                              "paper_h100_tf32": h100, "paper_rtx_pro_6000_tf32": rtx,
+                              "data": "synthetic (identity S, N(0, 0.01) factors)"}))
+            del sol
+            torch.cuda.empty_cache()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -159,8 +204,13 @@ def main():
                     help="factor start: iid N(0, 0.01), or the sign-structured start W > 0, H < 0")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing on the host")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg (profiling runs)")
+    ap.add_argument("--kernel-table", action="store_true",
+                    help="dense kernel alone at the paper's kernel-table shape (m = 250000 rows against a "
+                         "block of 2500), one JSON line per rank and precision")
     args = ap.parse_args()
     assert args.warmup >= 3, "at least 3 warm-up steps"
+    if args.kernel_table:
+        return kernel_table(args)
 
     from paper_2608_21607_gb300.replicas import env as replica_env
     ws, rank, local = replica_env()
