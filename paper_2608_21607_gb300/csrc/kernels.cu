@@ -272,16 +272,15 @@ __global__ void __launch_bounds__(RP * 4) ginv_reg_kernel(const float* __restric
 // ---------------------------------------------------------------------------
 // Sparse correction: for every panel row i and entry (i, k) in the block,
 // L_ik = m_i . q_k, c = S_ik - min(0, L_ik), R_i += c q_k (fp32 masters).
-// One warp per panel row or per segment of at most kSeg entries; the lanes
-// first fetch the entries' indices and values (one per lane), then NE
-// entries at a time (4 for single rows, which are mostly short; 8 for the
-// full segments of long rows) are processed with their q rows in flight
-// together; the accumulation order over the entries stays ascending.
-// The result goes to Rs, the support term of R, which holds zeros on every
-// other row (the update consumes it and clears it): single rows write their
-// row of Rs directly (one writer per row); segments of long rows write a
-// partial sum to their slot and a second pass adds the slots of each row in
-// a fixed order and writes the sum.
+// This kernel takes the rows with at most kShort entries in the panel: one
+// warp per row; the lanes first fetch the entries' indices and values (one
+// per lane), then NE entries at a time are processed with their q rows in
+// flight together, lanes over the r columns; the accumulation order over
+// the entries stays ascending.  The result goes to Rs, the support term of
+// R, one writer per row (or to a partial slot when `partials` is given).
+// Rs is written only on the rows with support in the block's panel; a flag
+// byte per row tells the update which rows of Rs to add, so the other rows
+// are neither read nor cleared.  Longer rows: sparse_long_kernel below.
 // ---------------------------------------------------------------------------
 template <int VPL, int NE>
 __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __restrict__ rows, int64_t nrows,
