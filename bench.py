@@ -47,17 +47,23 @@ WORKLOADS = {
 # summarised in profiles/dense_panel_connectome_r64_bf16.md; valid only while
 # the kernel's sources hash to the digest recorded with it (else null)
 DENSE_TRAFFIC = {
-    # (workload, precision, epilogue): (bytes per launch, sha256 prefix of the kernel sources)
-    ("connectome-139255-r64", "bf16", "z"): (18920362, "403bf4da01ad07df"),
+    # (workload, precision, epilogue): (bytes per launch, dense_source_digest() of the code measured)
+    ("connectome-139255-r64", "bf16", "z"): (18920362, "2343bf0ed2467707"),
 }
 
 
 def dense_source_digest():
+    """Digest of the dense kernel's code (panel_tc.cu, tc_ptx.cuh) with line
+    comments and blank lines removed: a recorded DRAM-traffic figure stays
+    valid across comment edits and lapses when the code changes."""
     import hashlib
     h = hashlib.sha256()
     for f in ("panel_tc.cu", "tc_ptx.cuh"):
-        with open(os.path.join(ROOT, "paper_2608_21607_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2608_21607_gb300", "csrc", f), encoding="utf-8") as fh:
+            for line in fh:
+                code = line.split("//", 1)[0].rstrip()
+                if code:
+                    h.update(code.encode() + b"\n")
     return h.hexdigest()[:16]
 
 

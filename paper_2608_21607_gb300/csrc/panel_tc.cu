@@ -3,12 +3,14 @@
 // For M-side rows m_i (a tile of 128) and Q-side rows q_k (streamed in
 // chunks of BN), the panel kernel computes, without writing any tile of L or
 // Z to global memory (the fused kernel of Sec. 4.2, eq. "kernel"):
-//   L_ik = m_i . q_k                         MMA1: TMEM <- W tile (TMEM) x chunk^T
+//   L_ik = m_i . q_k                         MMA1: TMEM <- W tile x chunk^T
 //   P_ik = min(0, L_ik)      (Z form, eq. updateZ)   -- epilogue in registers,
 //        = -max(0, L_ik)     (Delta form, eq. updateD)  written back to TMEM
 //   R_i  = sum_k P_ik q_k                    MMA2: TMEM R += P (TMEM) x chunk
 // The same shared-memory copy of each chunk feeds both products: K-major for
-// MMA1 and MN-major for MMA2.  Every factor has bf16 pieces hi = bf16(x),
+// MMA1 and MN-major for MMA2.  The W tile is MMA1's A operand from shared
+// memory (bf16 mode, TMA-loaded with the chunk's swizzle) or from TMEM
+// (fp32-accurate mode, written by the epilogue warps).  Every factor has bf16 pieces hi = bf16(x),
 // lo = bf16(x - hi), lo2 = bf16(x - hi - lo).  bf16 mode: MMA1 uses hi only,
 // MMA2 uses q = hi + lo -- every row of R shares the same q_k, so a rounding
 // of q would be a coherent error that the Gram solve amplifies by its
@@ -23,7 +25,7 @@
 // Warp roles (352 threads, one CTA per SM, persistent over M tiles):
 //   warps 0-7  epilogue, two warpgroups taking alternate chunks; in each,
 //              thread t owns TMEM lane t = tile row t
-//   warp 8     TMA producer of Q chunks (+ TMEM allocation)
+//   warp 8     TMA producer of Q chunks and W tiles (+ TMEM allocation)
 //   warp 9     issues MMA1 (L = W Q^T) for every chunk
 //   warp 10    issues MMA2 (R += P Q) for every chunk
 // The two MMA warps run converged and predicate each tcgen05 operation on an
