@@ -288,6 +288,28 @@ def test_bad_block_index_rejected():
         sol.block_update(N.NMD_COL, -1, N.NMD_STOCH)
 
 
+@pytest.mark.parametrize("order", [N.NMD_ALTERNATE, N.NMD_PHASED], ids=["alternate", "phased"])
+@pytest.mark.parametrize("prec", [N.NMD_BF16, N.NMD_FP32], ids=lambda p: PREC_NAMES[p])
+def test_sweep_schedule_equals_serial_steps(prec, order):
+    """A sweep (four streams; the rows the next step does not read updated
+    beside it) gives bit for bit the factors and momentum of the same block
+    steps run one after another, in the oracle's order of the sweep."""
+    _, S, r, W, H, br, bc, _ = cases()["planted1500x1300_r32"]
+    a = N.Solver(S, r, block_rows=br, block_cols=bc, precision=prec, order=order)
+    b = N.Solver(S, r, block_rows=br, block_cols=bc, precision=prec, order=order)
+    a.set_factors(W, H)
+    b.set_factors(W, H)
+    orc = O.State(S, np.asarray(W, np.float64), np.asarray(H, np.float64),
+                  O.Options(block_rows=br, block_cols=bc, order=order))
+    a.sweep()
+    for side, block, kind in orc.sweep_steps(0):
+        b.block_update(side, block, kind)
+    a.sync()
+    b.sync()
+    for x, y in zip(a.get_state()[:4], b.get_state()[:4]):
+        assert np.array_equal(x, y)
+
+
 @pytest.mark.parametrize("prec", PRECISIONS, ids=lambda p: PREC_NAMES[p])
 def test_deterministic_and_resumable(prec):
     _, S, r, W, H, br, bc, _ = cases()["connectome4000_r64"]
