@@ -163,6 +163,11 @@ def kernel_table(args):
     from paper_2608_21607_gb300 import build as B
     from paper_2608_21607_gb300 import nmd as N
     from paper_2608_21607_gb300 import workloads as WLm
+    from paper_2608_21607_gb300.replicas import env as replica_env
+    _, rank, local = replica_env()
+    if rank != 0:
+        return 0
+    torch.cuda.set_device(local)
     B.build()
     m, nb = 250000, 2500
     S = WLm.identity(m)
@@ -212,7 +217,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg (profiling runs)")
     ap.add_argument("--kernel-table", action="store_true",
                     help="dense kernel alone at the paper's kernel-table shape (m = 250000 rows against a "
-                         "block of 2500), one JSON line per rank and precision")
+                         "block of 2500), one JSON line per factor rank r and precision (rank 0 only)")
     args = ap.parse_args()
     assert args.warmup >= 3, "at least 3 warm-up steps"
     if args.kernel_table:
