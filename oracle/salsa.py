@@ -70,18 +70,20 @@ class SplitMix64:
         return splitmix64_mix(self.state)
 
 
-def block_permutation(seed: int, sweep: int, side: int, K: int) -> list:
-    """Order in which the K blocks of one side are visited in sweep ``sweep``.
-
-    Generator state = mix(seed) xor mix((sweep << 1) | side); Fisher-Yates from
-    the top: for i = K-1 .. 1, j = next() mod (i+1), swap(i, j).
-    """
-    g = SplitMix64(splitmix64_mix(seed) ^ splitmix64_mix(((sweep << 1) | side) & _MASK))
+def fisher_yates(K: int, g: SplitMix64) -> list:
+    """Shuffle of [0, K) from the top: for i = K-1 .. 1, j = next() mod (i+1),
+    swap(i, j) (the modulo bias, below 2^-57 for K < 2^7, is part of the order)."""
     perm = list(range(K))
     for i in range(K - 1, 0, -1):
         j = g.next() % (i + 1)
         perm[i], perm[j] = perm[j], perm[i]
     return perm
+
+
+def block_permutation(seed: int, sweep: int, side: int, K: int) -> list:
+    """Order in which the K blocks of one side are visited in sweep ``sweep``:
+    Fisher-Yates driven by SplitMix64 with state mix(seed) xor mix((sweep << 1) | side)."""
+    return fisher_yates(K, SplitMix64(splitmix64_mix(seed) ^ splitmix64_mix(((sweep << 1) | side) & _MASK)))
 
 
 def num_blocks(N: int, b: int) -> int:

@@ -279,7 +279,8 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->Ginv2 = c.take<float>((size_t)rp * rp);
   w->Gc = c.take<float>((size_t)rp * rp);
   w->Ginvc = c.take<float>((size_t)rp * rp);
-  w->chol_scratch = c.take<float>((size_t)2 * rp * rp);
+  w->Gx = c.take<float>((size_t)rp * rp);
+  w->Tm = c.take<float>((size_t)rp * rp);
   w->seg_partials = c.take<float>((size_t)std::max<int64_t>(maxseg, 1) * rp);
   w->flags = c.take<uint8_t>((size_t)std::max<int64_t>(nflags, 1));
   w->rpart = c.take<float>((size_t)kRpartRows * rp);
@@ -311,6 +312,21 @@ int64_t max_segments(PanelSet P[2][2]) {
     for (int k = 0; k < 2; ++k) t = std::max(t, P[s][k].max_segments);
   return t;
 }
+
+// Every call that takes a handle runs with the handle's device current and
+// puts the caller's device back afterwards, so that kernels, per-device
+// kernel attributes and the handle's streams all belong to the same device.
+struct DeviceScope {
+  int prev = -1;
+  explicit DeviceScope(const nmd_handle* h) {
+    int cur = -1;
+    if (h && cudaGetDevice(&cur) == cudaSuccess && cur != h->device && cudaSetDevice(h->device) == cudaSuccess)
+      prev = cur;
+  }
+  ~DeviceScope() {
+    if (prev >= 0) cudaSetDevice(prev);
+  }
+};
 
 // ---------------------------------------------------------------------------
 // Error plumbing
@@ -494,14 +510,15 @@ struct NextUse {
 
 nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro, float* R, float* Rs,
                               const uint8_t* flags, const float* Ginv, int64_t lo, int64_t hi, bool momentum,
-                              cudaStream_t s) {
+                              cudaStream_t s, bool gram = false) {
   if (hi <= lo) return NMD_OK;
   StepArgs sub = a;
   sub.m0 = ro.m0 + lo;
   sub.M = hi - lo;
   TimedScope ts(h, NMD_K_UPDATE, s);
   launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, Ginv, (float)h->opt.eta,
-                momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, s);
+                momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, gram ? h->ws.gram_part : nullptr,
+                h->opt.precision == NMD_BF16, s);
   h->launches++;
   return NMD_OK;
 }
@@ -528,6 +545,13 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   float* Rs = par ? h->ws.Rs2 : h->ws.Rs;
   float* G = par ? h->ws.G2 : h->ws.G;
   float* Ginv = par ? h->ws.Ginv2 : h->ws.Ginv;
+  // bf16 mode: the step's least-squares problem is solved for the bf16 pieces
+  // of the factors throughout -- the dense term (tensor cores), the support
+  // term and the Gram matrix G = Qt^T Qt all read the rounded rows Qt (and
+  // Mt), so that the rounding of Q is not a coherent error between R and G
+  // that the solve would amplify by the condition number of G; the update
+  // is applied to the fp32 masters.  The other modes use the masters.
+  const bool rounded = h->opt.precision == NMD_BF16;
   // an exact step's Q side is a whole factor: every block of a half-sweep has
   // the same G, computed once and kept until that factor changes
   bool need_gram = true;
@@ -541,20 +565,30 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   h->cur_R = R;
   h->cur_Rs = Rs;
   h->cur_G = G;
+  h->cur_Ginv = Ginv;
   // The side stream computes G = Q^T Q of the Q-side rows and G^{-1}, the
   // second side stream the support term Rs of R, the main stream the dense
   // term of R.  None reads what another writes, so they overlap; the update
   // joins them.
-  int nparts = (int)std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 127) / 128));
+  // Gram partials over parts of 64 Q-side rows where there are at most
+  // kGramParts of them (then the previous step's update of exactly these rows
+  // may already have written them, with the same arithmetic), else over
+  // kGramParts equal parts
+  const bool rows64 = (ro.K + 63) / 64 <= kGramParts;
+  const int nparts = rows64 ? (int)((ro.K + 63) / 64) : kGramParts;
+  const int64_t chunk = rows64 ? 64 : ((ro.K + nparts - 1) / nparts + 31) / 32 * 32;
+  const bool pre = h->gpre.active && kind == NMD_STOCH && h->gpre.f == fq && h->gpre.q0 == ro.q0 &&
+                   h->gpre.K == ro.K && h->gpre.step == h->step_index;
+  h->gpre.active = false;
   CK(h, cudaEventRecord(h->ev_fork, s));
   CK(h, cudaStreamWaitEvent(h->side, h->ev_fork, 0));
   CK(h, cudaStreamWaitEvent(h->side2, h->ev_fork, 0));
   if (need_gram) {
     TimedScope ts(h, NMD_K_GRAM, h->side);
-    launch_gram(*ro.fq, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, h->side);
-    launch_chol_inv(h->ws.gram_part, nparts, h->r, h->rp, (float)h->opt.ridge, G, Ginv, h->ws.chol_scratch,
-                    h->ws.status, h->side);
-    h->launches += 2;
+    launch_gram(pre ? nullptr : ro.fq, rounded, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, chunk,
+                (float)h->opt.ridge, G, h->side);
+    launch_chol_inv(G, h->r, h->rp, Ginv, h->ws.status, h->side);
+    h->launches += pre ? 2 : 3;
   }
   if ((st = after_launch(h, "gram/cholesky")) != NMD_OK) return st;
   // sparse correction over the block's support
@@ -594,14 +628,27 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
     // next step reads only these rows of this factor and writes the other
     // factor, the rest are updated on the aux stream, overlapping it
     int64_t lo = 0, hi = ro.M;
+    // the next step's Q-side block is exactly these rows (an alternating
+    // stochastic sweep): their update also writes that step's Gram partials
+    bool gram_next = false;
     if (next) {
       Roles rn;
       if (roles(h, next->side, next->block, next->kind, &rn) == NMD_OK && rn.fq == ro.fm && rn.fm != ro.fm) {
         lo = std::min(std::max(rn.q0 - ro.m0, (int64_t)0), ro.M);
         hi = std::max(std::min(rn.q0 + rn.K - ro.m0, ro.M), lo);
+        gram_next = next->kind == NMD_STOCH && h->rp <= 64 && lo == rn.q0 - ro.m0 && hi - lo == rn.K &&
+                    (rn.K + 63) / 64 <= kGramParts;
       }
     }
-    if ((st = launch_update_rows(h, a, ro, R, Rs, flags, Ginv, lo, hi, momentum, s)) != NMD_OK) return st;
+    if ((st = launch_update_rows(h, a, ro, R, Rs, flags, Ginv, lo, hi, momentum, s, gram_next)) != NMD_OK)
+      return st;
+    if (gram_next) {
+      h->gpre.active = true;
+      h->gpre.f = fm;
+      h->gpre.q0 = ro.m0 + lo;
+      h->gpre.K = hi - lo;
+      h->gpre.step = h->step_index + 1;
+    }
     if (lo > 0 || hi < ro.M) {
       CK(h, cudaEventRecord(h->ev_prio, s));
       CK(h, cudaStreamWaitEvent(h->aux, h->ev_prio, 0));
@@ -682,6 +729,7 @@ int64_t nmd_launch_count(const nmd_handle* h) { return h ? h->launches : 0; }
 
 nmd_status nmd_selftest_wait_timeout(nmd_handle* h, int64_t limit_ns) {
   if (!h || limit_ns < 1000 || limit_ns > 1000000000) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   nmd_status st = sync_and_check(h);
   if (st != NMD_OK) return st;
   launch_wait_selftest(h->ws.status, (uint64_t)limit_ns, h->stream);
@@ -692,6 +740,7 @@ nmd_status nmd_selftest_wait_timeout(nmd_handle* h, int64_t limit_ns) {
 
 nmd_status nmd_skip_count(nmd_handle* h, int64_t* skipped, int32_t reset) {
   if (!h || !skipped) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   nmd_status st = sync_and_check(h);
   if (st != NMD_OK) return st;
   unsigned long long v = 0;
@@ -836,6 +885,7 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
 
 nmd_status nmd_set_factors(nmd_handle* h, const float* W, const float* H, int on_device) {
   if (!h || !W || !H) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_set_factors");
+  DeviceScope dg(h);
   h->fver[0]++;
   h->fver[1]++;
   cudaStream_t s = h->stream;
@@ -857,6 +907,7 @@ nmd_status nmd_set_factors(nmd_handle* h, const float* W, const float* H, int on
 
 nmd_status nmd_get_factors(nmd_handle* h, float* W, float* H, int on_device) {
   if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   nmd_status st = sync_and_check(h);
   cudaStream_t s = h->stream;
   cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost;
@@ -876,6 +927,7 @@ nmd_status nmd_get_factors(nmd_handle* h, float* W, float* H, int on_device) {
 
 nmd_status nmd_block_update(nmd_handle* h, int32_t side, int64_t block, int32_t kind) {
   if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   return run_step(h, side, block, kind, true);
 }
 
@@ -890,6 +942,7 @@ nmd_status nmd_block_order(const nmd_handle* h, int64_t sweep, int32_t side, int
 
 nmd_status nmd_sweep(nmd_handle* h) {
   if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   int64_t Kr = nblocks(h->m, h->opt.block_rows), Kc = nblocks(h->n, h->opt.block_cols);
   std::vector<int64_t> pr = permutation(h->opt.seed, h->sweep_index, NMD_ROW, Kr);
   std::vector<int64_t> pc = permutation(h->opt.seed, h->sweep_index, NMD_COL, Kc);
@@ -914,6 +967,7 @@ nmd_status nmd_sweep(nmd_handle* h) {
   for (size_t t = 0; t < steps.size() && st == NMD_OK; ++t)
     st = run_step(h, steps[t].side, steps[t].block, steps[t].kind, true,
                   t + 1 < steps.size() ? &steps[t + 1] : nullptr);
+  h->gpre.active = false;
   // `stream` continues after every kernel of the sweep, deferred ones included
   nmd_status st2 = wait_all_pending(h);
   h->cur = h->stream;
@@ -926,11 +980,13 @@ nmd_status nmd_sweep(nmd_handle* h) {
 
 nmd_status nmd_sync(nmd_handle* h) {
   if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   return sync_and_check(h);
 }
 
 nmd_status nmd_loss(nmd_handle* h, nmd_loss_out* out) {
   if (!h || !out) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_loss");
+  DeviceScope dg(h);
   nmd_status st = sync_and_check(h);
   if (st != NMD_OK) return st;
   cudaStream_t s = h->stream;
@@ -972,6 +1028,7 @@ nmd_status nmd_loss(nmd_handle* h, nmd_loss_out* out) {
 nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* R,
                            float* G, int64_t* rows) {
   if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   Roles ro;
   nmd_status st = roles(h, side, block, kind, &ro);
   if (st != NMD_OK) return st;
@@ -983,8 +1040,26 @@ nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t k
   if ((st = sync_and_check(h)) != NMD_OK) return st;
   if (rows) *rows = ro.M;
   cudaStream_t s = h->stream;
-  if (R) CK(h, cudaMemcpy2DAsync(R, h->r * 4, h->cur_R, h->rp * 4, h->r * 4, ro.M, cudaMemcpyDeviceToHost, s));
-  if (G) CK(h, cudaMemcpy2DAsync(G, h->r * 4, h->cur_G, h->rp * 4, h->r * 4, h->r, cudaMemcpyDeviceToHost, s));
+  const float* Rout = h->cur_R;
+  const float* Gout = h->cur_G;
+  if (h->opt.precision == NMD_BF16) {
+    // the bf16 mode solves X = R' Gt^{-1} for the rounded rows (R' = Z Qt,
+    // Gt = Qt^T Qt); report the exact G of the fp32 rows and the right-hand
+    // side that gives the same X with it: R' Gt^{-1} G
+    float* other = h->cur_R == h->ws.R ? h->ws.R2 : h->ws.R;
+    const int rp = h->rp;
+    const int64_t np = std::min<int64_t>(kGramParts, std::max<int64_t>(1, (ro.K + 63) / 64));
+    const int64_t ch = ((ro.K + np - 1) / np + 31) / 32 * 32;
+    launch_gram(ro.fq, false, ro.q0, ro.K, h->r, rp, h->ws.gram_part, (int)np, ch, (float)h->opt.ridge, h->ws.Gx, s);
+    launch_small_gemm(h->cur_Ginv, rp, h->ws.Gx, rp, h->ws.Tm, rp, rp, rp, rp, s);
+    launch_small_gemm(h->cur_R, rp, h->ws.Tm, rp, other, rp, ro.M, rp, rp, s);
+    h->launches += 4;
+    if ((st = after_launch(h, "equivalent right-hand side")) != NMD_OK) return st;
+    Rout = other;
+    Gout = h->ws.Gx;
+  }
+  if (R) CK(h, cudaMemcpy2DAsync(R, h->r * 4, Rout, h->rp * 4, h->r * 4, ro.M, cudaMemcpyDeviceToHost, s));
+  if (G) CK(h, cudaMemcpy2DAsync(G, h->r * 4, Gout, h->rp * 4, h->r * 4, h->r, cudaMemcpyDeviceToHost, s));
   CK(h, cudaStreamSynchronize(s));
   return NMD_OK;
 }
@@ -992,6 +1067,7 @@ nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t k
 nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* d_L,
                               int64_t* rows, int64_t* cols) {
   if (!h || !d_L) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_dense_products");
+  DeviceScope dg(h);
   Roles ro;
   nmd_status st = roles(h, side, block, kind, &ro);
   if (st != NMD_OK) return st;
@@ -1010,6 +1086,7 @@ nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_
 nmd_status nmd_panel_traversal(const nmd_handle* h, int32_t side, int64_t block, int32_t kind,
                                int64_t* rows_out, int64_t* q_out, int64_t cap, int64_t* count) {
   if (!h || !count) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   Roles ro;
   nmd_status st = roles(const_cast<nmd_handle*>(h), side, block, kind, &ro);
   if (st != NMD_OK) return st;
@@ -1046,6 +1123,7 @@ nmd_status nmd_panel_traversal(const nmd_handle* h, int32_t side, int64_t block,
 
 nmd_status nmd_get_state(nmd_handle* h, float* W, float* H, float* EW, float* EH, int64_t* sweep_index) {
   if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   nmd_status st = nmd_get_factors(h, W, H, 0);
   if (st != NMD_OK) return st;
   cudaStream_t s = h->stream;
@@ -1067,6 +1145,7 @@ nmd_status nmd_get_state(nmd_handle* h, float* W, float* H, float* EW, float* EH
 nmd_status nmd_set_state(nmd_handle* h, const float* W, const float* H, const float* EW, const float* EH,
                          int64_t sweep_index) {
   if (!h || !W || !H || !EW || !EH || sweep_index < 0) return fail(h, NMD_ERR_INVALID, "bad nmd_set_state argument");
+  DeviceScope dg(h);
   nmd_status st = nmd_set_factors(h, W, H, 0);
   if (st != NMD_OK) return st;
   cudaStream_t s = h->stream;
@@ -1088,6 +1167,7 @@ nmd_status nmd_set_state(nmd_handle* h, const float* W, const float* H, const fl
 
 nmd_status nmd_profile(nmd_handle* h, int on) {
   if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   CK(h, cudaStreamSynchronize(h->stream));
   collect_timing(h);
   for (int c = 0; c < 5; ++c) {
@@ -1100,6 +1180,7 @@ nmd_status nmd_profile(nmd_handle* h, int on) {
 
 nmd_status nmd_profile_read(nmd_handle* h, int32_t kernel_class, double* ms, int64_t* launches) {
   if (!h || kernel_class < 0 || kernel_class > 4) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
   CK(h, cudaStreamSynchronize(h->stream));
   collect_timing(h);
   if (ms) *ms = h->prof_ms[kernel_class];
@@ -1107,6 +1188,9 @@ nmd_status nmd_profile_read(nmd_handle* h, int32_t kernel_class, double* ms, int
   return NMD_OK;
 }
 
-void nmd_destroy(nmd_handle* h) { delete h; }
+void nmd_destroy(nmd_handle* h) {
+  DeviceScope dg(h);
+  delete h;
+}
 
 }  // extern "C"

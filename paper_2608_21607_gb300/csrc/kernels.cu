@@ -1,10 +1,12 @@
-// Small kernels of the block step: operand packing, Gram matrix, Gram
-// inverse, sparse support correction, least-squares/momentum update, and the
-// support part and final reduction of the loss.
+// Small kernels of the block step: operand packing, Gram matrix, Cholesky
+// factor and inverse of the Gram matrix, sparse support correction,
+// least-squares/momentum update, and the support part and final reduction of
+// the loss.
 #include <float.h>
 #include <math.h>
 
 #include <algorithm>
+#include <atomic>
 
 #include "nmd_internal.cuh"
 
@@ -68,13 +70,18 @@ __global__ void unpack_kernel(const float* __restrict__ master, int dst_is_rxN, 
 // Gram matrix G = Q^T Q over Q-side rows [q0, q0+K): grid (tiles, parts).
 // Tile (ta, tb), ta >= tb, of 64 x 64 entries; part p sums the rows
 // [p*chunk, (p+1)*chunk) in ascending order.  The partials are summed in a
-// fixed order by the inverse kernel, so the result is deterministic.
+// fixed order by gram_reduce_kernel, so the result is deterministic.  T is
+// the element type of the rows read: float (the fp32 masters) or bf16 (the
+// hi pieces, for the Gram matrix of the bf16-rounded rows).
 // ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ Q, int64_t q0, int64_t K,
-                                                   int rp, float* __restrict__ parts, int64_t chunk) {
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(bf16 x) { return __bfloat162float(x); }
+
+template <typename T>
+__global__ void __launch_bounds__(256, 4) gram_kernel(const T* __restrict__ Q, int64_t q0, int64_t K, int rp,
+                                                      float* __restrict__ parts, int64_t chunk) {
   __shared__ float Qa[32][65];
   __shared__ float Qb[32][65];
-  int nt = (rp + 63) / 64;
   int t = blockIdx.x, ta = 0;
   while (t >= ta + 1) { t -= ta + 1; ++ta; }
   int tb = t;
@@ -88,8 +95,8 @@ __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ Q, 
       int rr = e / 64, cc = e % 64;
       int64_t k = kb + rr;
       bool ok = k < k1;
-      Qa[rr][cc] = (ok && cc < wa) ? Q[(q0 + k) * rp + ta * 64 + cc] : 0.f;
-      if (ta != tb) Qb[rr][cc] = (ok && cc < wb) ? Q[(q0 + k) * rp + tb * 64 + cc] : 0.f;
+      Qa[rr][cc] = (ok && cc < wa) ? to_f(Q[(q0 + k) * rp + ta * 64 + cc]) : 0.f;
+      if (ta != tb) Qb[rr][cc] = (ok && cc < wb) ? to_f(Q[(q0 + k) * rp + tb * 64 + cc]) : 0.f;
     }
     __syncthreads();
     const float(*Qs)[65] = ta != tb ? Qb : Qa;   // a diagonal tile reads one copy
@@ -107,7 +114,6 @@ __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ Q, 
     }
     __syncthreads();
   }
-  (void)nt;
   float* out = parts + (size_t)p * rp * rp;
   for (int i = 0; i < 4; ++i)
     for (int j = 0; j < 4; ++j) {
@@ -116,157 +122,412 @@ __global__ void __launch_bounds__(256) gram_kernel(const float* __restrict__ Q, 
     }
 }
 
-// ---------------------------------------------------------------------------
-// G^{-1} by the symmetric sweep operator (Gauss-Jordan without pivoting, valid
-// for symmetric positive definite G): sweeping pivot k maps
-//   a_kk -> -1/a_kk, a_ik -> a_ik/a_kk, a_kj -> a_kj/a_kk,
-//   a_ij -> a_ij - a_ik a_kj / a_kk  (i, j != k);
-// after all r pivots the matrix holds -G^{-1}.  The pivots are the Schur
-// complements (the squared Cholesky pivots); one that is not positive
-// relative to the diagonal marks G as not positive definite.
-// One thread block; the r x r matrix lives in shared memory when it fits.
-// ---------------------------------------------------------------------------
-// Thread (ty, tx) of a T x T block owns the entries (ty + T a, tx + T b).
-template <int T>
-__global__ void __launch_bounds__(T * T) ginv_kernel(const float* __restrict__ parts, int nparts, int r, int rp,
-                                                     float ridge, float* __restrict__ Gout,
-                                                     float* __restrict__ Ginv, float* __restrict__ scratch,
-                                                     int* __restrict__ status, int use_smem) {
-  extern __shared__ float sm[];
-  float* A = use_smem ? sm : scratch;             // r x r
-  __shared__ float rowk[256];
-  __shared__ float diag0[256];
-  __shared__ int bad;
-  const int tx = threadIdx.x % T, ty = threadIdx.x / T;
-  if (threadIdx.x == 0) bad = 0;
-  for (int i = ty; i < r; i += T)
-    for (int j = tx; j < r; j += T) {
-      const int a = max(i, j), b = min(i, j);     // the partials hold the lower triangle
-      const float* src = parts + (size_t)a * rp + b;
-      float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      int p = 0;
-      for (; p + 8 <= nparts; p += 8)
+// G = the partials summed in part order (eight interleaved sums, added in a
+// fixed tree), + ridge on the diagonal, written to both triangles from the
+// lower one (the partials hold every entry whose 64-row tile is at or below
+// its 64-column tile); pad rows and columns (>= r) are zero.  One thread per
+// entry.
+__global__ void __launch_bounds__(256) gram_reduce_kernel(const float* __restrict__ parts, int nparts, int r,
+                                                          int rp, float ridge, float* __restrict__ G) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e >= rp * rp) return;
+  const int i = e / rp, j = e - (e / rp) * rp;
+  if (j > i) return;
+  float sum = 0.f;
+  if (i < r) {
+    const float* src = parts + (size_t)i * rp + j;
+    float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    int p = 0;
+    for (; p + 8 <= nparts; p += 8)
 #pragma unroll
-        for (int q = 0; q < 8; ++q) acc[q] += __ldg(src + (size_t)(p + q) * rp * rp);
-      for (; p < nparts; ++p) acc[0] += __ldg(src + (size_t)p * rp * rp);
-      float sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
-      if (i == j) {
-        sum += ridge;
-        diag0[i] = sum;
-      }
-      A[i * r + j] = sum;
+      for (int q = 0; q < 8; ++q) acc[q] += __ldg(src + (size_t)(p + q) * rp * rp);
+    for (; p < nparts; ++p) acc[0] += __ldg(src + (size_t)p * rp * rp);
+    sum = ((acc[0] + acc[1]) + (acc[2] + acc[3])) + ((acc[4] + acc[5]) + (acc[6] + acc[7]));
+    if (i == j) sum += ridge;
+  }
+  G[(size_t)i * rp + j] = sum;
+  G[(size_t)j * rp + i] = sum;
+}
+
+// C (M x N) = A (M x K) B (K x N), row-major fp32 with leading dimensions,
+// for the small products of the Gram chain (T = G^{-1} Gt and Q' = Q T, both
+// with N, K <= 256).  64 x 64 output tile per block of 16 x 16 threads, 4 x 4
+// per thread, K in slices of 16 staged in shared memory; the order of every
+// sum is fixed.
+__global__ void __launch_bounds__(256) small_gemm_kernel(const float* __restrict__ A, int64_t lda,
+                                                         const float* __restrict__ B, int64_t ldb,
+                                                         float* __restrict__ Cm, int64_t ldc, int64_t M, int N,
+                                                         int K) {
+  __shared__ float As[16][64 + 4];
+  __shared__ float Bs[16][64];
+  const int tx = threadIdx.x % 16, ty = threadIdx.x / 16;
+  const int64_t m0 = (int64_t)blockIdx.x * 64;
+  const int n0 = blockIdx.y * 64;
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+  for (int k0 = 0; k0 < K; k0 += 16) {
+    for (int e = threadIdx.x; e < 64 * 16; e += 256) {
+      const int rr = e / 16, kk = e % 16;
+      const int64_t row = m0 + rr;
+      As[kk][rr] = (row < M && k0 + kk < K) ? A[row * lda + k0 + kk] : 0.f;
+      const int kb = e / 64, cc = e % 64;
+      Bs[kb][cc] = (k0 + kb < K && n0 + cc < N) ? B[(int64_t)(k0 + kb) * ldb + n0 + cc] : 0.f;
     }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < 16; ++kk) {
+      float a[4], b[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int64_t row = m0 + ty * 4 + i;
+    if (row >= M) break;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int col = n0 + tx * 4 + j;
+      if (col < N) Cm[row * ldc + col] = acc[i][j];
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// G^{-1} through the Cholesky factorisation of G (the normal equations of
+// eqs. lsqA/lsqB, Sec. 3.2), in its square-root-free form G = L D L^T (L unit
+// lower triangular, D diagonal; the Cholesky factor is L D^{1/2}), then
+// Y = L^{-1} and G^{-1} = Y^T D^{-1} Y.  One thread block of T x T threads.
+// The lower triangle lives in
+// shared memory in packed row-major form (row i starts at i (i + 1) / 2);
+// thread (ty, tx) takes rows ty, ty + T, ... and within a row the columns
+// tx, tx + T, ..., so the lanes of a warp touch consecutive entries of a row.
+//  1. Right-looking factorisation, one column per step and one barrier per
+//     step: the pivot d_k = a_kk is the Schur complement (the square of the
+//     Cholesky pivot); d_k <= 4 r eps g_kk or a non-finite d_k marks G as not
+//     positive definite (NMD_ERR_NOT_SPD, detail k) and leaves G^{-1} = 0.
+//     Otherwise a_ij -= a_ik a_jk / d_k for k < j <= i; column k keeps
+//     a_ik = l_ik d_k.  Column k is read from a copy that the previous step
+//     wrote (two copies alternate), so no step reads what it writes.
+//  2. Y = L^{-1} (unit lower; its diagonal is implicit), column step k: row k
+//     of Y is final, and every row i > k subtracts l_ik Y[k, 0..k].  With
+//     room for a second triangle (r_pad <= 128, SEPY) Y has its own;
+//     otherwise (r_pad = 256) Y takes the place of L, and each warp reads
+//     l_ik before any of its lanes writes Y[i, k] over it (a warp is one row
+//     group there).  One barrier per step.
+//  3. G^{-1}[a][b] = sum over k >= max(a, b) of Y[k][a] Y[k][b] / d_k, each
+//     thread a 4 x 4 block of the lower triangle, written to both triangles
+//     so that the result is exactly symmetric.
+// ---------------------------------------------------------------------------
+__host__ __device__ __forceinline__ int tri(int i) { return (i * (i + 1)) >> 1; }
+
+inline size_t chol_smem_bytes(int r, int rp, bool sepy) {
+  return ((size_t)(sepy ? 2 : 1) * (size_t)((tri(r) + 3) & ~3) + 4 * (size_t)rp) * sizeof(float);
+}
+
+template <int T, bool SEPY>
+__global__ void __launch_bounds__(T * T) chol_inv_kernel(const float* __restrict__ G, int r, int rp,
+                                                         float* __restrict__ Ginv, int* __restrict__ status) {
+  static_assert(SEPY || T == 32, "in-place inverse needs one warp per row group");
+  extern __shared__ __align__(16) float sm[];
+  const int ntri = (tri(r) + 3) & ~3;
+  float* A = sm;                                   // the factor
+  float* Y = SEPY ? sm + ntri : sm;                // L^{-1}
+  float* colk = sm + (SEPY ? 2 : 1) * ntri;        // 2 x rp: column k of the factor, alternating
+  float* invd = colk + 2 * rp;                     // rp: 1 / d_k
+  float* diag0 = invd + rp;                        // rp: the diagonal of G
+  constexpr int NT = T * T;
+  const int tx = threadIdx.x % T, ty = threadIdx.x / T;
+  for (int i = ty; i < r; i += T)
+    for (int j = tx; j <= i; j += T) {
+      const float g = G[(size_t)i * rp + j];
+      A[tri(i) + j] = g;
+      if (j == 0) colk[i] = g;
+      if (i == j) diag0[i] = g;
+    }
+  for (int e = threadIdx.x; e < rp * rp; e += NT)
+    if (e / rp >= r || e % rp >= r) Ginv[e] = 0.f;
   __syncthreads();
-  for (int i = ty; i < rp; i += T)
-    for (int j = tx; j < rp; j += T) Gout[i * rp + j] = (i < r && j < r) ? A[i * r + j] : 0.f;
+  // 1. G = L D L^T
   const float tol = 4.0f * (float)r * FLT_EPSILON;
   for (int k = 0; k < r; ++k) {
-    const float d = A[k * r + k];
-    if (!(d > tol * diag0[k]) || !isfinite(d)) {
-      if (threadIdx.x == 0) {
-        bad = 1;
-        set_status(status, NMD_ERR_NOT_SPD, k, 0);
-      }
-      break;   // uniform: every thread read the same d
+    const float* ck = colk + (k & 1) * rp;
+    float* cn = colk + ((k + 1) & 1) * rp;
+    const float d = ck[k];
+    if (!(d > tol * diag0[k]) || !isfinite(d)) {   // uniform: every thread read the same d
+      if (threadIdx.x == 0) set_status(status, NMD_ERR_NOT_SPD, k, 0);
+      for (int e = threadIdx.x; e < rp * rp; e += NT) Ginv[e] = 0.f;
+      return;
     }
-    for (int j = threadIdx.x; j < r; j += T * T) rowk[j] = A[k * r + j];
-    __syncthreads();
     const float inv = 1.0f / d;
-    for (int i = ty; i < r; i += T) {
-      const float ri = rowk[i] * inv;
-      for (int j = tx; j < r; j += T) {
-        float v;
-        if (i == k && j == k) v = -inv;
-        else if (i == k) v = rowk[j] * inv;
-        else if (j == k) v = ri;                  // symmetric: a_ik = a_ki
-        else v = A[i * r + j] - ri * rowk[j];
-        A[i * r + j] = v;
+    if (threadIdx.x == 0) invd[k] = inv;
+    for (int i = k + 1 + ty; i < r; i += T) {
+      const float ci = ck[i];
+      float* row = A + tri(i);
+      for (int j = k + 1 + tx; j <= i; j += T) {
+        const float v = fmaf(-(ci * ck[j]), inv, row[j]);
+        row[j] = v;
+        if (j == k + 1) cn[i] = v;                  // column k + 1 for the next step
       }
     }
     __syncthreads();
   }
-  __syncthreads();
-  for (int i = ty; i < rp; i += T)
-    for (int j = tx; j < rp; j += T) {
-      float v = 0.f;
-      if (!bad && i < r && j < r) v = -0.5f * (A[i * r + j] + A[j * r + i]);   // symmetrise
-      Ginv[i * rp + j] = v;
+  // 2. Y = L^{-1}, l_ik = a_ik / d_k
+  for (int k = 0; k + 1 < r; ++k) {
+    const float* yk = Y + tri(k);
+    const float ik = invd[k];
+    for (int i = k + 1 + ty; i < r; i += T) {
+      const float lik = A[tri(i) + k] * ik;
+      if (!SEPY) __syncwarp();                     // every lane has l_ik before Y[i, k] replaces it
+      float* row = Y + tri(i);
+      for (int j = tx; j <= k; j += T) row[j] = j == k ? -lik : fmaf(-lik, yk[j], row[j]);
     }
+    __syncthreads();
+  }
+  // 3. G^{-1} = Y^T D^{-1} Y
+  const int n4 = (r + 3) / 4;
+  for (int t = threadIdx.x; t < tri(n4); t += NT) {
+    int ta = (int)((sqrtf(8.f * (float)t + 1.f) - 1.f) * 0.5f);
+    while (tri(ta + 1) <= t) ++ta;
+    while (tri(ta) > t) --ta;
+    const int tb = t - tri(ta);
+    const int a0 = 4 * ta, b0 = 4 * tb;
+    float acc[4][4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int v = 0; v < 4; ++v) acc[u][v] = 0.f;
+    for (int k = a0; k < r; ++k) {
+      const float* yk = Y + tri(k);
+      const float w = invd[k];
+      float ya[4], yb[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        ya[u] = w * (a0 + u < k ? yk[a0 + u] : (a0 + u == k ? 1.f : 0.f));
+        yb[u] = b0 + u < k ? yk[b0 + u] : (b0 + u == k ? 1.f : 0.f);
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(ya[u], yb[v], acc[u][v]);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const int a = a0 + u, b = b0 + v;
+        if (a < r && b <= a) {
+          Ginv[(size_t)a * rp + b] = acc[u][v];
+          Ginv[(size_t)b * rp + a] = acc[u][v];
+        }
+      }
+  }
 }
 
-// Register-resident variant for rp <= 128: thread t owns row t / 4 and the
-// rp / 4 contiguous columns (t % 4) rp / 4 ... of it.  Before pivot k the
-// owners of row k publish it to shared memory (two alternating buffers, one
-// barrier per pivot); every thread then updates its own entries from that
-// row alone, using the symmetry a_ik = a_ki.  Each update is written so that
-// (i, j) and (j, i) round identically (the product a_ik a_kj is formed
-// before the division), so the matrix stays exactly symmetric.  The partial
-// Gram matrices are summed in part order first.
+// Register-resident, blocked form of the same factorisation for r_pad <= 128
+// (the pad rows and columns >= r get a unit diagonal, so the padded matrix
+// diag(G, I) is factored and inverted; its pad part is dropped at the end).
+// Thread t owns row i = t / 4 and the CPT = r_pad / 4 contiguous columns
+// c0 = (t % 4) CPT ... of it in registers; a warp holds 8 whole rows.  The
+// columns are taken in panels of PB = min(8, CPT):
+//  1. The PB x PB diagonal block lies in one warp: its rows factor it in
+//     their registers, reading each other's entries by shuffles (pivot test
+//     as above), and publish it.
+//     Every row below then eliminates its own PB panel values against the
+//     block (no communication) and publishes them; after a barrier every
+//     row applies the rank-PB update a_ij -= sum_k a_ik a_jk / d_k to its
+//     columns right of the panel.  Two barriers per panel.
+//  2. Y = L^{-1} by panels of PB rows: inside the block's warp, forward
+//     substitution with shuffles; the block's rows of Y go to shared memory
+//     (two buffers) and every row below subtracts sum_k l_ik Y[k, :].  One
+//     barrier per panel.
+//  3. G^{-1} = Y^T D^{-1} Y from shared memory.
 template <int RP>
-__global__ void __launch_bounds__(RP * 4) ginv_reg_kernel(const float* __restrict__ parts, int nparts, int r,
-                                                          float ridge, float* __restrict__ Gout,
-                                                          float* __restrict__ Ginv, int* __restrict__ status) {
-  constexpr int CPT = RP / 4;
-  __shared__ __align__(16) float rk[2][RP];
-  __shared__ float diag0[RP];
-  const int i = threadIdx.x / 4, c0 = (threadIdx.x % 4) * CPT;
-  // the partials hold the entries whose 64-row tile is >= their 64-column tile
-  const bool direct = (i / 64) >= (c0 / 64);
+__global__ void __launch_bounds__(RP * 4) ldlt_inv_reg_kernel(const float* __restrict__ G, int r,
+                                                              float* __restrict__ Ginv, int* __restrict__ status) {
+  constexpr int CPT = RP / 4, PB = CPT < 8 ? CPT : 8, LD = RP + 1;
+  extern __shared__ __align__(16) float smr[];
+  float* invd = smr;                 // RP: 1 / d_k
+  float* diag0 = invd + RP;          // RP: the diagonal of G
+  float* DB = diag0 + RP;            // PB x PB: the diagonal block being factored (64 floats)
+  float* Pn = DB + 64;               // RP x PB: the panel's columns / 2 x PB x RP: rows of Y
+  float* F = Pn + 2 * PB * RP;       // RP x LD: the factor, then Y
+  __shared__ int bad;
+  const int i = threadIdx.x / 4, s = threadIdx.x % 4, c0 = s * CPT, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) bad = 0;
   float a[CPT];
 #pragma unroll
-  for (int j = 0; j < CPT; ++j) a[j] = 0.f;
-#pragma unroll 4
-  for (int p = 0; p < nparts; ++p) {
-    const float* src = parts + (size_t)p * RP * RP;
-    if (direct) {
-#pragma unroll
-      for (int j = 0; j < CPT; j += 4) {
-        const float4 v = __ldg((const float4*)(src + i * RP + c0 + j));
-        a[j] += v.x; a[j + 1] += v.y; a[j + 2] += v.z; a[j + 3] += v.w;
-      }
-    } else {
-#pragma unroll
-      for (int j = 0; j < CPT; ++j) a[j] += __ldg(src + (c0 + j) * RP + i);
-    }
+  for (int j = 0; j < CPT; j += 4) {
+    const float4 v = *(const float4*)(G + (size_t)i * RP + c0 + j);
+    a[j] = v.x; a[j + 1] = v.y; a[j + 2] = v.z; a[j + 3] = v.w;
   }
 #pragma unroll
   for (int j = 0; j < CPT; ++j)
-    if (c0 + j == i && i < r) {
-      a[j] += ridge;
+    if (c0 + j == i) {
+      if (i >= r) a[j] = 1.f;
       diag0[i] = a[j];
     }
-#pragma unroll
-  for (int j = 0; j < CPT; ++j) Gout[i * RP + c0 + j] = (i < r && c0 + j < r) ? a[j] : 0.f;
+  __syncthreads();
   const float tol = 4.0f * (float)r * FLT_EPSILON;
-  bool bad = false;
-  for (int k = 0; k < r; ++k) {
-    float* rb = rk[k & 1];
-    if (i == k) {
+  // 1. G = L D L^T, a[] keeping a_ij = l_ij d_j (j < i) and d_i (j == i)
 #pragma unroll
-      for (int j = 0; j < CPT; j += 4) *(float4*)(rb + c0 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
+  for (int kb = 0; kb < RP; kb += PB) {
+    const int sp = kb / CPT, jp = kb - (kb / CPT) * CPT;   // segment and offset of the panel's columns
+    const bool in_block = i >= kb && i < kb + PB;
+    if ((threadIdx.x >> 5) == (kb >> 3)) {
+      // the block's rows kb + q are lanes 4 ((kb + q) % 8) + sp of this warp:
+      // factor the block in their registers, one shuffle per entry read
+      const bool mine = in_block && s == sp;
+      const int qo = i - kb;
+      float blk[PB];
+#pragma unroll
+      for (int k = 0; k < PB; ++k) blk[k] = a[jp + k];
+#pragma unroll
+      for (int k = 0; k < PB; ++k) {
+        const int lk = ((kb + k) & 7) * 4 + sp;
+        const float d = __shfl_sync(0xffffffffu, blk[k], lk);
+        const float inv = 1.0f / d;
+        if (lane == lk) {
+          const int kk = kb + k;
+          if (kk < r && (!(d > tol * diag0[kk]) || !isfinite(d))) {
+            if (!bad) set_status(status, NMD_ERR_NOT_SPD, kk, 0);
+            bad = 1;
+          }
+          invd[kk] = inv;
+        }
+        const float ajk = blk[k] * inv;
+#pragma unroll
+        for (int q = k + 1; q < PB; ++q) {
+          const float aqk = __shfl_sync(0xffffffffu, blk[k], ((kb + q) & 7) * 4 + sp);
+          if (mine && qo > k && q <= qo) blk[q] = fmaf(-ajk, aqk, blk[q]);
+        }
+      }
+      if (mine)
+#pragma unroll
+        for (int k = 0; k < PB; ++k) {
+          a[jp + k] = blk[k];
+          DB[qo * PB + k] = blk[k];
+        }
     }
     __syncthreads();
-    const float d = rb[k];
-    if (!(d > tol * diag0[k]) || !isfinite(d)) {   // uniform: every thread read the same d
-      bad = true;
-      if (threadIdx.x == 0) set_status(status, NMD_ERR_NOT_SPD, k, 0);
-      break;
+    if (bad) {   // uniform: every thread reads the flag after the barrier
+#pragma unroll
+      for (int j = 0; j < CPT; ++j) Ginv[(size_t)i * RP + c0 + j] = 0.f;
+      return;
     }
-    const float inv = 1.0f / d;
-    if (i == k) {
+    if (s == sp && i >= kb) {
+      if (!in_block) {
 #pragma unroll
-      for (int j = 0; j < CPT; ++j) a[j] = (c0 + j == k) ? -inv : a[j] * inv;
-    } else {
-      const float ri = rb[i];
+        for (int k = 0; k < PB; ++k) {
+          const float u = a[jp + k] * invd[kb + k];
 #pragma unroll
-      for (int j = 0; j < CPT; ++j) {
-        const float rj = rb[c0 + j];
-        a[j] = (c0 + j == k) ? ri * inv : fmaf(-(ri * rj), inv, a[j]);
+          for (int q = k + 1; q < PB; ++q) a[jp + q] = fmaf(-u, DB[q * PB + k], a[jp + q]);
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < PB; k += 4)
+        *(float4*)(Pn + i * PB + k) = make_float4(a[jp + k], a[jp + k + 1], a[jp + k + 2], a[jp + k + 3]);
+    }
+    __syncthreads();
+    if (i >= kb + PB) {
+      float u[PB];
+#pragma unroll
+      for (int k = 0; k < PB; k += 4) {
+        const float4 v = *(const float4*)(Pn + i * PB + k);
+        u[k] = v.x * invd[kb + k]; u[k + 1] = v.y * invd[kb + k + 1];
+        u[k + 2] = v.z * invd[kb + k + 2]; u[k + 3] = v.w * invd[kb + k + 3];
+      }
+#pragma unroll
+      for (int jj = 0; jj < CPT; ++jj) {
+        if (c0 + jj >= kb + PB) {
+          float acc = a[jj];
+#pragma unroll
+          for (int k = 0; k < PB; k += 4) {
+            const float4 v = *(const float4*)(Pn + (c0 + jj) * PB + k);
+            acc = fmaf(-u[k], v.x, acc); acc = fmaf(-u[k + 1], v.y, acc);
+            acc = fmaf(-u[k + 2], v.z, acc); acc = fmaf(-u[k + 3], v.w, acc);
+          }
+          a[jj] = acc;
+        }
       }
     }
   }
 #pragma unroll
-  for (int j = 0; j < CPT; ++j) Ginv[i * RP + c0 + j] = (!bad && i < r && c0 + j < r) ? -a[j] : 0.f;
+  for (int j = 0; j < CPT; ++j) F[i * LD + c0 + j] = a[j];
+  __syncthreads();
+  // 2. Y = L^{-1} (a[] now holds row i of Y), l_ik = a_ik / d_k
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) a[j] = c0 + j == i ? 1.f : 0.f;
+#pragma unroll
+  for (int kb = 0; kb < RP; kb += PB) {
+    float* YP = Pn + ((kb / PB) & 1) * PB * RP;
+    if ((threadIdx.x >> 5) == (kb >> 3)) {
+      const int rl = i - kb;   // row within the block (outside [0, PB) for the warp's other rows)
+#pragma unroll
+      for (int k = 0; k + 1 < PB; ++k) {
+        const int src = ((kb + k) & 7) * 4 + s;
+        const float l = (rl > k && rl < PB) ? F[i * LD + kb + k] * invd[kb + k] : 0.f;
+#pragma unroll
+        for (int jj = 0; jj < CPT; ++jj) {
+          const float yk = __shfl_sync(0xffffffffu, a[jj], src);
+          a[jj] = fmaf(-l, yk, a[jj]);
+        }
+      }
+      if (rl >= 0 && rl < PB)
+#pragma unroll
+        for (int jj = 0; jj < CPT; jj += 4)
+          *(float4*)(YP + rl * RP + c0 + jj) = make_float4(a[jj], a[jj + 1], a[jj + 2], a[jj + 3]);
+    }
+    __syncthreads();
+    if (i >= kb + PB) {
+      float l[PB];
+#pragma unroll
+      for (int k = 0; k < PB; ++k) l[k] = F[i * LD + kb + k] * invd[kb + k];
+#pragma unroll
+      for (int jj = 0; jj < CPT; jj += 4) {
+        float4 acc = make_float4(a[jj], a[jj + 1], a[jj + 2], a[jj + 3]);
+#pragma unroll
+        for (int k = 0; k < PB; ++k) {
+          const float4 v = *(const float4*)(YP + k * RP + c0 + jj);
+          acc.x = fmaf(-l[k], v.x, acc.x); acc.y = fmaf(-l[k], v.y, acc.y);
+          acc.z = fmaf(-l[k], v.z, acc.z); acc.w = fmaf(-l[k], v.w, acc.w);
+        }
+        a[jj] = acc.x; a[jj + 1] = acc.y; a[jj + 2] = acc.z; a[jj + 3] = acc.w;
+      }
+    }
+  }
+  __syncthreads();   // every read of the factor is done
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) F[i * LD + c0 + j] = a[j];
+  __syncthreads();
+  // 3. G^{-1}[i][j] = sum over k of Y[k][i] Y[k][j] / d_k (Y[k][j] = 0 for j > k)
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) a[j] = 0.f;
+  for (int k = i > c0 ? i : c0; k < RP; ++k) {
+    const float w = F[k * LD + i] * invd[k];
+#pragma unroll
+    for (int j = 0; j < CPT; ++j) a[j] = fmaf(w, F[k * LD + c0 + j], a[j]);
+  }
+#pragma unroll
+  for (int j = 0; j < CPT; ++j) a[j] = (i < r && c0 + j < r) ? a[j] : 0.f;
+#pragma unroll
+  for (int j = 0; j < CPT; j += 4)
+    *(float4*)(Ginv + (size_t)i * RP + c0 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
+}
+
+inline size_t ldlt_reg_smem_bytes(int rp) {
+  const size_t pb = rp / 4 < 8 ? rp / 4 : 8;
+  return ((size_t)2 * rp + 64 + 2 * pb * rp + (size_t)rp * (rp + 1)) * sizeof(float);
 }
 
 // ---------------------------------------------------------------------------
@@ -282,10 +543,13 @@ __global__ void __launch_bounds__(RP * 4) ginv_reg_kernel(const float* __restric
 // byte per row tells the update which rows of Rs to add, so the other rows
 // are neither read nor cleared.  Longer rows: sparse_long_kernel below.
 // ---------------------------------------------------------------------------
-template <int VPL, int NE>
+__device__ __forceinline__ float ldv(const float* p) { return __ldg(p); }
+__device__ __forceinline__ float ldv(const bf16* p) { return __bfloat162float(__ldg(p)); }
+
+template <int VPL, int NE, typename T>
 __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __restrict__ rows, int64_t nrows,
-                                                          const float* __restrict__ Mop, int64_t m0,
-                                                          const float* __restrict__ Qop,
+                                                          const T* __restrict__ Mop, int64_t m0,
+                                                          const T* __restrict__ Qop,
                                                           const int32_t* __restrict__ qidx,
                                                           const float* __restrict__ vals,
                                                           float* __restrict__ R, float* __restrict__ partials,
@@ -305,7 +569,7 @@ __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __rest
 #pragma unroll
   for (int v = 0; v < VPL; ++v) {
     const int c = lane + 32 * v;
-    mv[v] = c < rp ? __ldg(Mop + i * rp + c) : 0.f;
+    mv[v] = c < rp ? ldv(Mop + i * rp + c) : 0.f;
     acc[v] = 0.f;
   }
   for (int e = 0; e < pr.len; e += NE) {
@@ -320,7 +584,7 @@ __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __rest
 #pragma unroll
       for (int v = 0; v < VPL; ++v) {
         const int c = lane + 32 * v;
-        qv[j][v] = (live && c < rp) ? __ldg(Qop + (int64_t)k * rp + c) : 0.f;
+        qv[j][v] = (live && c < rp) ? ldv(Qop + (int64_t)k * rp + c) : 0.f;
         part[j] = fmaf(mv[v], qv[j][v], part[j]);
       }
     }
@@ -355,10 +619,28 @@ __global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __rest
 // accumulates c q_k over its own entries; at the end the EPW entry slots are
 // added with a butterfly (one reduction per row instead of one per entry).
 // The order of every sum is fixed, so results are the same on every run.
-template <int LPE, int CPL>
+// Stage 32 columns (one chunk) of a q row into 32 floats of shared memory,
+// 16 bytes per load: 4 fp32 or 8 bf16 values.
+__device__ __forceinline__ void stage16(float* dst, const float* src) {
+  *(float4*)dst = __ldg((const float4*)src);
+}
+__device__ __forceinline__ void stage16(float* dst, const bf16* src) {
+  const uint4 u = __ldg((const uint4*)src);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+  float f[8];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    f[2 * q] = __uint_as_float(w[q] << 16);
+    f[2 * q + 1] = __uint_as_float(w[q] & 0xffff0000u);
+  }
+  *(float4*)dst = make_float4(f[0], f[1], f[2], f[3]);
+  *(float4*)(dst + 4) = make_float4(f[4], f[5], f[6], f[7]);
+}
+
+template <int LPE, int CPL, typename T>
 __global__ void __launch_bounds__(256, 2) sparse_long_kernel(const PanelRow* __restrict__ segs, int64_t nseg,
-                                                          const float* __restrict__ Mop, int64_t m0,
-                                                          const float* __restrict__ Qop,
+                                                          const T* __restrict__ Mop, int64_t m0,
+                                                          const T* __restrict__ Qop,
                                                           const int32_t* __restrict__ qidx,
                                                           const float* __restrict__ vals,
                                                           float* __restrict__ R, float* __restrict__ partials,
@@ -366,6 +648,8 @@ __global__ void __launch_bounds__(256, 2) sparse_long_kernel(const PanelRow* __r
   constexpr int EPW = 32 / LPE;
   constexpr int CS = 36;                       // floats per staged chunk (32 + 4 padding)
   constexpr int NPF = 4;                       // entry iterations whose indices are fetched together
+  constexpr int VEC = 16 / (int)sizeof(T);     // elements per 16-byte load
+  constexpr int LPC = CPL / VEC;               // 16-byte loads per 32-column chunk
   __shared__ __align__(16) float stage[8][32 * CS];
   const int lane = threadIdx.x & 31;
   const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
@@ -375,14 +659,8 @@ __global__ void __launch_bounds__(256, 2) sparse_long_kernel(const PanelRow* __r
   const int sub = lane % LPE, slot = lane / LPE;
   const int64_t i = pr.row;
   float mv[CPL], acc[CPL];
-  {
-    const float4* m4 = (const float4*)(Mop + i * rp + 32 * sub);
 #pragma unroll
-    for (int c = 0; c < CPL / 4; ++c) {
-      const float4 v = __ldg(m4 + c);
-      mv[4 * c] = v.x; mv[4 * c + 1] = v.y; mv[4 * c + 2] = v.z; mv[4 * c + 3] = v.w;
-    }
-  }
+  for (int c = 0; c < CPL; ++c) mv[c] = ldv(Mop + i * rp + 32 * sub + c);
 #pragma unroll
   for (int c = 0; c < CPL; ++c) acc[c] = 0.f;
   for (int e00 = 0; e00 < pr.len; e00 += NPF * EPW) {
@@ -398,16 +676,20 @@ __global__ void __launch_bounds__(256, 2) sparse_long_kernel(const PanelRow* __r
 #pragma unroll
     for (int t = 0; t < NPF; ++t) {
       if (e00 + t * EPW >= pr.len) break;             // warp-uniform
-      // stage: float4 f = lane + 32 u (u < CPL / 4) of the 32 chunks; chunk
-      // f / 8 is columns 32 (chunk % LPE) ... of entry slot chunk / LPE
+      // stage: load f = lane + 32 u (u < LPC) of the 32 chunks; chunk f / LPC
+      // is columns 32 (chunk % LPE) ... of entry slot chunk / LPE
 #pragma unroll
-      for (int u = 0; u < CPL / 4; ++u) {
+      for (int u = 0; u < LPC; ++u) {
         const int f = lane + 32 * u;
-        const int chunk = f / (CPL / 4), part = f % (CPL / 4);
+        const int chunk = f / LPC, part = f % LPC;
         const int ke = __shfl_sync(0xffffffffu, kk[t], (chunk / LPE) * LPE);
-        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (ke >= 0) v = __ldg((const float4*)(Qop + (int64_t)ke * rp + 32 * (chunk % LPE)) + part);
-        *(float4*)(buf + chunk * CS + 4 * part) = v;
+        float* dst = buf + chunk * CS + VEC * part;
+        if (ke >= 0) {
+          stage16(dst, Qop + (int64_t)ke * rp + 32 * (chunk % LPE) + VEC * part);
+        } else {
+#pragma unroll
+          for (int q = 0; q < VEC; q += 4) *(float4*)(dst + q) = make_float4(0.f, 0.f, 0.f, 0.f);
+        }
       }
       __syncwarp();
       float q[CPL];
@@ -473,7 +755,10 @@ __global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __re
 //   Z form:     U = eta (X - M)      (eqs. lsqA/lsqB with step size)
 //   Delta form: U = eta X            (eqs. spLsqA/spLsqB)
 // then E = U + gamma E (stochastic steps) and M += E, refreshing the bf16
-// pieces (the third piece only where the fp32-accurate mode reads it).
+// pieces: hi always, lo and lo2 only in the fp32-accurate mode (the only
+// one whose dense kernel reads them).
+// In the bf16 mode R and Ginv belong to the bf16-rounded Q-side rows (R = Z Qt,
+// Ginv = (Qt^T Qt)^{-1}), so X is the least-squares solution for them.
 // Skipped entirely while a sticky error is set.
 // X = R G^{-1} is a small GEMM per tile of TR rows.  A block keeps CW columns
 // of G^{-1} in shared memory; the tile's R rows (contiguous in global memory)
@@ -516,8 +801,9 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
                                                      const float* __restrict__ R, const float* __restrict__ Rs,
                                                      const uint8_t* __restrict__ flags,
                                                      const float* __restrict__ Ginv, float eta,
-                                                     float gamma, int momentum, int delta_form, int write_lo2,
-                                                     int* __restrict__ status) {
+                                                     float gamma, int momentum, int delta_form, int write_lo,
+                                                     int* __restrict__ status, float* __restrict__ gpart,
+                                                     int gram_round) {
   using C = UpdCfg<RP>;
   constexpr int NV = C::TR * RP / 4 / 256;   // float4 of a tile per thread
   constexpr int CW = C::CW, TR = C::TR, TX = C::TX, CPT = C::CPT;
@@ -637,10 +923,22 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
         }
       }
     }
+    // Gram partials of the new rows (r_pad <= 64, one block column): the
+    // tile's R staging buffer receives the new rows once every thread is done
+    // with it (rows past the end read as zero)
+    constexpr bool GRAM_OK = RP <= 64 && CW == RP && TR == 64;
+    const bool gram = GRAM_OK && gpart != nullptr;
+    float* Ms = Rb + buf * TR * RP;
+    if (gram) __syncthreads();
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int64_t li = base + 4 * ty + i;
-      if (li >= rows) break;
+      if (li >= rows) {
+        if (gram)
+#pragma unroll
+          for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * RP + upd_col<CPT, TX>(tx, j)] = 0.f;
+        continue;
+      }
       const int64_t g = (m0 + li) * RP + cw0;
       bool finite = true;
       float nv[CPT], ev[CPT];
@@ -668,9 +966,10 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
           *(float4*)(M + g + c) = make_float4(nv[j], nv[j + 1], nv[j + 2], nv[j + 3]);
           if (momentum) *(float4*)(E + g + c) = make_float4(ev[j], ev[j + 1], ev[j + 2], ev[j + 3]);
           *(uint2*)(Mhi + g + c) = make_uint2(hw[j] | (hw[j + 1] << 16), hw[j + 2] | (hw[j + 3] << 16));
-          *(uint2*)(Mlo + g + c) = make_uint2(lw[j] | (lw[j + 1] << 16), lw[j + 2] | (lw[j + 3] << 16));
-          if (write_lo2)
+          if (write_lo) {
+            *(uint2*)(Mlo + g + c) = make_uint2(lw[j] | (lw[j + 1] << 16), lw[j + 2] | (lw[j + 3] << 16));
             *(uint2*)(Mlo2 + g + c) = make_uint2(l2w[j] | (l2w[j + 1] << 16), l2w[j + 2] | (l2w[j + 3] << 16));
+          }
         }
       } else {
 #pragma unroll
@@ -679,11 +978,54 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
           M[g + c] = nv[j];
           if (momentum) E[g + c] = ev[j];
           Mhi[g + c] = __ushort_as_bfloat16((unsigned short)hw[j]);
-          Mlo[g + c] = __ushort_as_bfloat16((unsigned short)lw[j]);
-          if (write_lo2) Mlo2[g + c] = __ushort_as_bfloat16((unsigned short)l2w[j]);
+          if (write_lo) {
+            Mlo[g + c] = __ushort_as_bfloat16((unsigned short)lw[j]);
+            Mlo2[g + c] = __ushort_as_bfloat16((unsigned short)l2w[j]);
+          }
         }
       }
       if (!finite) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
+      if (gram)
+#pragma unroll
+        for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * RP + upd_col<CPT, TX>(tx, j)] = nv[j];
+    }
+    if constexpr (GRAM_OK) {
+      if (gram) {
+        // partial t of the Gram matrix of the new rows (gram_round: of their
+        // bf16 rounding, the hi pieces just written): every entry summed over
+        // the tile's 64 rows in ascending order with fmaf, the same operations
+        // as gram_kernel on a part of 64 rows, so that a step gets the same G
+        // whichever kernel formed its partials
+        __syncthreads();
+        constexpr int GA = RP / 16;
+        const int a0 = (threadIdx.x / 16) * GA, b0 = (threadIdx.x % 16) * GA;
+        float g1[GA][GA];
+#pragma unroll
+        for (int u = 0; u < GA; ++u)
+#pragma unroll
+          for (int v = 0; v < GA; ++v) g1[u][v] = 0.f;
+        for (int rr = 0; rr < TR; ++rr) {
+          float av[GA], bv[GA];
+#pragma unroll
+          for (int u = 0; u < GA; ++u) {
+            av[u] = Ms[rr * RP + a0 + u];
+            bv[u] = Ms[rr * RP + b0 + u];
+            if (gram_round) {
+              av[u] = __bfloat162float(__float2bfloat16_rn(av[u]));
+              bv[u] = __bfloat162float(__float2bfloat16_rn(bv[u]));
+            }
+          }
+#pragma unroll
+          for (int u = 0; u < GA; ++u)
+#pragma unroll
+            for (int v = 0; v < GA; ++v) g1[u][v] = fmaf(av[u], bv[v], g1[u][v]);
+        }
+        float* o1 = gpart + (size_t)t * RP * RP;
+#pragma unroll
+        for (int u = 0; u < GA; ++u)
+#pragma unroll
+          for (int v = 0; v < GA; ++v) o1[(a0 + u) * RP + b0 + v] = g1[u][v];
+      }
     }
     __syncthreads();   // the buffer read above is refilled by the next iteration's copy
   }
@@ -819,36 +1161,50 @@ void launch_unpack(const float* master, bool dst_is_rxN, int64_t N, int r, int r
   unpack_kernel<<<grid_for(N * r, 256), 256, 0, s>>>(master, dst_is_rxN, N, r, rp, dst);
 }
 
-void launch_gram(const Factor& fq, int64_t q0, int64_t K, int r, int rp, float* parts, int nparts,
-                 cudaStream_t s) {
-  (void)r;
-  int nt = (rp + 63) / 64;
-  int64_t chunk = (K + nparts - 1) / nparts;
-  chunk = (chunk + 31) / 32 * 32;
-  dim3 grid(nt * (nt + 1) / 2, nparts);
-  gram_kernel<<<grid, 256, 0, s>>>(fq.master, q0, K, rp, parts, chunk);
+void launch_gram(const Factor* fq, bool rounded, int64_t q0, int64_t K, int r, int rp, float* parts, int nparts,
+                 int64_t chunk, float ridge, float* G, cudaStream_t s) {
+  if (fq) {
+    int nt = (rp + 63) / 64;
+    dim3 grid(nt * (nt + 1) / 2, nparts);
+    if (rounded)
+      gram_kernel<bf16><<<grid, 256, 0, s>>>(fq->hi, q0, K, rp, parts, chunk);
+    else
+      gram_kernel<float><<<grid, 256, 0, s>>>(fq->master, q0, K, rp, parts, chunk);
+  }
+  gram_reduce_kernel<<<(unsigned)((rp * rp + 255) / 256), 256, 0, s>>>(parts, nparts, r, rp, ridge, G);
 }
 
-void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge, float* G, float* Ginv,
-                     float* scratch, int* status, cudaStream_t s) {
-  const size_t smem = (size_t)r * r * sizeof(float);
-  const int use_smem = smem <= 200 * 1024;
+void launch_small_gemm(const float* A, int64_t lda, const float* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
+                       int N, int K, cudaStream_t s) {
+  if (M <= 0) return;
+  dim3 grid((unsigned)((M + 63) / 64), (unsigned)((N + 63) / 64));
+  small_gemm_kernel<<<grid, 256, 0, s>>>(A, lda, B, ldb, C, ldc, M, N, K);
+}
+
+void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cudaStream_t s) {
   if (rp <= 128) {
+    const size_t smem = ldlt_reg_smem_bytes(rp);
     switch (rp) {
-      case 16: ginv_reg_kernel<16><<<1, 64, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
-      case 32: ginv_reg_kernel<32><<<1, 128, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
-      case 64: ginv_reg_kernel<64><<<1, 256, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
-      default: ginv_reg_kernel<128><<<1, 512, 0, s>>>(parts, nparts, r, ridge, G, Ginv, status); break;
+      case 16: ldlt_inv_reg_kernel<16><<<1, 64, smem, s>>>(G, r, Ginv, status); break;
+      case 32: ldlt_inv_reg_kernel<32><<<1, 128, smem, s>>>(G, r, Ginv, status); break;
+      case 64: ldlt_inv_reg_kernel<64><<<1, 256, smem, s>>>(G, r, Ginv, status); break;
+      default: {
+        static std::atomic<int> attr[kMaxDevices];
+        per_device(attr, [] {
+          return cudaFuncSetAttribute(ldlt_inv_reg_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                      (int)ldlt_reg_smem_bytes(128)) == cudaSuccess ? 1 : 0;
+        });
+        ldlt_inv_reg_kernel<128><<<1, 512, smem, s>>>(G, r, Ginv, status);
+      }
     }
-  } else {
-    static bool attr = false;
-    if (!attr) {
-      cudaFuncSetAttribute(ginv_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
-      attr = true;
-    }
-    ginv_kernel<32><<<1, 1024, use_smem ? smem : 0, s>>>(parts, nparts, r, rp, ridge, G, Ginv, scratch, status,
-                                                         use_smem);
+    return;
   }
+  static std::atomic<int> attr[kMaxDevices];
+  per_device(attr, [] {
+    return cudaFuncSetAttribute(chol_inv_kernel<32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)chol_smem_bytes(256, 256, false)) == cudaSuccess ? 1 : 0;
+  });
+  chol_inv_kernel<32, false><<<1, 1024, chol_smem_bytes(r, rp, false), s>>>(G, r, rp, Ginv, status);
 }
 
 static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* partials, float* R, int64_t m0, int rp,
@@ -866,64 +1222,74 @@ static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* pa
 void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole, int64_t nwhole,
                    const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
                    const float* vals, float* R, float* partials, cudaStream_t s) {
-  // The support correction always reads the fp32 masters, in every precision:
-  // on rows with few support entries the term S_ik q_k dominates R_i and is
-  // not averaged over many products, so rounding q_k to bf16 there would put
-  // its full relative error (up to 2^-9) into the update.
-  const float* Mop = a.fm->master;
-  const float* Qop = a.fq->master;
-#define NMD_SP(V, LPE, CPL)                                                                                  \
+  // The support term reads the same factor values as the rest of the step's
+  // least-squares problem: the bf16 pieces in the bf16 mode (whose dense term
+  // and Gram matrix are formed from them), the fp32 masters otherwise.
+#define NMD_SP(V, LPE, CPL, TT, MOP, QOP)                                                                    \
   do {                                                                                                       \
     if (nrows > 0)                                                                                           \
-      sparse_rows_kernel<V, 4><<<(unsigned)((nrows + 7) / 8), 256, 0, s>>>(rows, nrows, Mop, a.m0, Qop, qidx, \
-                                                                           vals, R, nullptr, a.rp);         \
+      sparse_rows_kernel<V, 4, TT><<<(unsigned)((nrows + 7) / 8), 256, 0, s>>>(rows, nrows, MOP, a.m0, QOP, qidx, \
+                                                                               vals, R, nullptr, a.rp);     \
     if (nwhole > 0)                                                                                          \
-      sparse_long_kernel<LPE, CPL><<<(unsigned)((nwhole + 7) / 8), 256, 0, s>>>(whole, nwhole, Mop, a.m0, Qop, \
-                                                                                qidx, vals, R, nullptr, a.rp); \
+      sparse_long_kernel<LPE, CPL, TT><<<(unsigned)((nwhole + 7) / 8), 256, 0, s>>>(                          \
+          whole, nwhole, MOP, a.m0, QOP, qidx, vals, R, nullptr, a.rp);                                      \
     if (nseg > 0) {                                                                                          \
-      sparse_long_kernel<LPE, CPL><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(seg, nseg, Mop, a.m0, Qop, qidx, \
-                                                                              vals, R, partials, a.rp);      \
+      sparse_long_kernel<LPE, CPL, TT><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(                            \
+          seg, nseg, MOP, a.m0, QOP, qidx, vals, R, partials, a.rp);                                         \
       launch_reduce(multi, nmulti, partials, R, a.m0, a.rp, s);                                              \
     }                                                                                                        \
   } while (0)
+#define NMD_SP2(V, LPE, CPL)                                                                \
+  do {                                                                                      \
+    if (a.precision == NMD_BF16) NMD_SP(V, LPE, CPL, bf16, a.fm->hi, a.fq->hi);             \
+    else NMD_SP(V, LPE, CPL, float, a.fm->master, a.fq->master);                            \
+  } while (0)
   switch (a.rp) {
-    case 16: NMD_SP(1, 1, 16); break;
-    case 32: NMD_SP(1, 1, 32); break;
-    case 64: NMD_SP(2, 2, 32); break;
-    case 128: NMD_SP(4, 4, 32); break;
-    default: NMD_SP(8, 8, 32); break;
+    case 16: NMD_SP2(1, 1, 16); break;
+    case 32: NMD_SP2(1, 1, 32); break;
+    case 64: NMD_SP2(2, 2, 32); break;
+    case 128: NMD_SP2(4, 4, 32); break;
+    default: NMD_SP2(8, 8, 32); break;
   }
+#undef NMD_SP2
 #undef NMD_SP
 }
 
 template <int RP>
 static void update_rp(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
-                      float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
+                      float eta, float gamma, bool momentum, int* status, float* gpart, bool gram_round,
+                      cudaStream_t s) {
   using C = UpdCfg<RP>;
-  static int per_sm = 0;
-  if (per_sm == 0) {
+  // the attribute and the occupancy belong to the current device
+  static std::atomic<int> cache[kMaxDevices];
+  const int per_sm = per_device(cache, [] {
+    int n = 0;
     cudaFuncSetAttribute(update_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, update_kernel<RP>, 256, C::SMEM) != cudaSuccess ||
-        per_sm < 1)
-      per_sm = 1;
-  }
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, update_kernel<RP>, 256, C::SMEM) != cudaSuccess || n < 1)
+      n = 1;
+    return n;
+  });
+  // one tile per block: blocks retire every few microseconds, so that the
+  // higher-priority streams' kernels (the next step's Gram chain and support
+  // term) get SM slots while a deferred update runs beside the dense kernel;
+  // per_sm only bounds the grid when the tiles exceed 65,535 waves' worth
   const int64_t tiles = (a.M + C::TR - 1) / C::TR;
-  dim3 grid((unsigned)std::min<int64_t>(tiles, (int64_t)a.num_sms * per_sm), RP / C::CW);
+  dim3 grid((unsigned)std::min<int64_t>(tiles, (int64_t)a.num_sms * per_sm * 65535), RP / C::CW);
   const Factor& f = *a.fm;
   update_kernel<RP><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, flags, Ginv, eta,
                                                gamma,
                                                momentum, a.epilogue == NMD_EPI_DELTA,
-                                               a.precision == NMD_FP32, status);
+                                               a.precision == NMD_FP32, status, gpart, gram_round ? 1 : 0);
 }
 
 void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
-                   float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
+                   float eta, float gamma, bool momentum, int* status, float* gpart, bool gram_round, cudaStream_t s) {
   switch (a.rp) {
-    case 16: update_rp<16>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
-    case 32: update_rp<32>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
-    case 64: update_rp<64>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
-    case 128: update_rp<128>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
-    default: update_rp<256>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, s); break;
+    case 16: update_rp<16>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, gpart, gram_round, s); break;
+    case 32: update_rp<32>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, gpart, gram_round, s); break;
+    case 64: update_rp<64>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, gpart, gram_round, s); break;
+    case 128: update_rp<128>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, nullptr, false, s); break;
+    default: update_rp<256>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, nullptr, false, s); break;
   }
 }
 

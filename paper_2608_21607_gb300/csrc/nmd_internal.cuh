@@ -5,6 +5,7 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include <atomic>
 #include <string>
 #include <vector>
 
@@ -13,6 +14,23 @@
 namespace nmd {
 
 typedef __nv_bfloat16 bf16;
+
+// Kernel attributes (cudaFuncSetAttribute) and occupancy figures belong to a
+// device, so the host code caches them per device ordinal: slot[d] holds the
+// value f() returned with device d current (0 = not yet computed; f returns
+// a positive value, or 0 when it failed and should run again next time).
+constexpr int kMaxDevices = 64;
+template <class F>
+int per_device(std::atomic<int> (&slot)[kMaxDevices], F f) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return f();
+  int v = slot[dev].load(std::memory_order_acquire);
+  if (v == 0) {
+    v = f();
+    if (v > 0) slot[dev].store(v, std::memory_order_release);
+  }
+  return v;
+}
 
 // One row of a block's sparse panel: entries [beg, beg + len) of the CSR (or
 // CSC) arrays, all belonging to M-side row `row` and lying in the block's
@@ -107,11 +125,12 @@ struct Workspace {
   float* Ginv2 = nullptr;
   float* Gc = nullptr;         // G and G^{-1} of an exact step's Q side (all of one factor),
   float* Ginvc = nullptr;      // kept while that factor is unchanged
+  float* Gx = nullptr;         // rp x rp: the exact G of a bf16-mode step (verification hook)
+  float* Tm = nullptr;         // rp x rp: scratch of the verification hook
   double* loss_part = nullptr; // kLossParts x 8
   double* loss_out = nullptr;  // 8
   int* status = nullptr;       // kStatusWords
   int* counters = nullptr;     // 64 ints; ints 0-1: skipped Delta-form chunks (u64)
-  float* chol_scratch = nullptr;  // 2 x rp x rp (used when rp is too large for smem)
   float* seg_partials = nullptr;  // max segments x rp (sparse correction of long rows)
   uint8_t* flags = nullptr;       // the panels' support-row flags, concatenated
   float* rpart = nullptr;         // kRpartRows x rp: partial R's of split-K steps
@@ -160,6 +179,14 @@ struct nmd_handle {
   float* cur_Rs = nullptr;
   const uint8_t* cur_flags = nullptr;   // the support-row flags of the last step
   float* cur_G = nullptr;
+  float* cur_Ginv = nullptr;   // the inverse the last step's update applied
+  // Gram partials of the next step's Q-side block, written by this step's
+  // update of exactly those rows (see run_step); valid for step `step` only
+  struct GramPre {
+    bool active = false;
+    int f = -1;
+    int64_t q0 = 0, K = 0, step = -1;
+  } gpre;
   nmd::Workspace ws;
   nmd::Factor W, B;            // A = W (m x r), B = H^T (n x r)
   nmd::PanelSet panels[2][2];  // [side][kind]
@@ -188,19 +215,31 @@ void launch_pack(const float* src, bool src_is_rxN, int64_t N, int r, int rp, Fa
                  cudaStream_t s);
 void launch_unpack(const float* master, bool dst_is_rxN, int64_t N, int r, int rp, float* dst,
                    cudaStream_t s);
-void launch_gram(const Factor& fq, int64_t q0, int64_t K, int r, int rp, float* parts,
-                 int nparts, cudaStream_t s);
-void launch_chol_inv(const float* parts, int nparts, int r, int rp, float ridge, float* G,
-                     float* Ginv, float* scratch, int* status, cudaStream_t s);
+// G = Q^T Q of the Q-side rows [q0, q0 + K) (+ ridge on the diagonal) via
+// nparts fixed-order partials of `chunk` rows; rounded: of their bf16 pieces
+// (hi) instead of the fp32 masters.  fq == nullptr: the partials are already
+// there (written by launch_update's gpart) and only the reduction runs.
+void launch_gram(const Factor* fq, bool rounded, int64_t q0, int64_t K, int r, int rp, float* parts, int nparts,
+                 int64_t chunk, float ridge, float* G, cudaStream_t s);
+// Ginv = G^{-1} through the Cholesky (L D L^T) factorisation; NMD_ERR_NOT_SPD
+// in the status words on failure
+void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cudaStream_t s);
+// C = A B (row-major fp32, M x K times K x N, N and K <= 256)
+void launch_small_gemm(const float* A, int64_t lda, const float* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
+                       int N, int K, cudaStream_t s);
 // rows: short rows; whole: the whole rows of the long-row kernel; seg: the
 // slices of the split rows, summed per row of `multi` into R
+// (bf16 mode: the factors' hi pieces, else the fp32 masters)
 void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole,
                    int64_t nwhole, const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti,
                    const int32_t* qidx, const float* vals, float* R, float* partials, cudaStream_t s);
 // flags: one byte per row of the step (Rs is read only where it is nonzero)
+// gpart, when not nullptr and r_pad <= 64: also write the Gram partials of the
+// new rows, one per 64-row tile (gram_round: of their bf16 rounding), exactly
+// as launch_gram would with parts of 64 rows
 void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags,
-                   const float* Ginv, float eta, float gamma, bool momentum, int* status,
-                   cudaStream_t s);
+                   const float* Ginv, float eta, float gamma, bool momentum, int* status, float* gpart,
+                   bool gram_round, cudaStream_t s);
 void launch_combine(float* R, const float* Rs, const uint8_t* flags, int64_t rows, int rp, cudaStream_t s);
 // the bounded pipeline wait, run on a barrier that never completes
 void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);

@@ -57,26 +57,28 @@ constexpr uint64_t kTimeoutNs = 2000000000ull;
 
 template <int RP, bool SPLIT, bool LOSS>
 struct Cfg {
-  // bf16 mode with r_pad <= 128: MMA2 multiplies P by [q_hi | q_lo] as one
-  // product of width 2 r_pad (two accumulators side by side, summed at
-  // readout): half the MMA instructions of two separate products
-  static constexpr bool FUSEDN = !SPLIT && !LOSS && RP <= 128;
   // fp32-accurate mode at r_pad = 256: W hi + lo take 256 TMEM columns, so a
   // CTA accumulates one 128-column half of R (blockIdx.y selects it) and the
   // first product is formed once per half
   static constexpr bool RHALF = SPLIT && !LOSS && RP == 256;
   static constexpr int NR = RHALF ? RP / 2 : RP;        // R columns of one CTA
-  // TMEM columns of the R accumulator(s); the loss pass has none
-  static constexpr int RCOLS = LOSS ? 0 : (FUSEDN ? 2 * RP : NR);
+  // TMEM columns of the R accumulator; the loss pass has none.  In the bf16
+  // mode the second product multiplies P by q_hi alone: the update pairs
+  // this term with the Gram matrix of q_hi, so the rounding of q cancels
+  // (see update_kernel), and R needs one accumulator of r_pad columns.
+  static constexpr int RCOLS = LOSS ? 0 : NR;
   // bf16 mode, r_pad <= 128: the W tile is the first product's A operand
-  // from shared memory (loaded by TMA) instead of TMEM.  At r_pad <= 64 that
-  // leaves room for three L buffers of 128 columns: chunks of 128 Q rows
-  // halve the hand-offs (barrier waits and commits) per row and the first
-  // product's MMA count.  At r_pad = 128 it gives four L buffers of 64.
-  static constexpr bool WSMEM = FUSEDN;
-  // Q rows per chunk.  64 where the TMEM budget would otherwise leave only
-  // two L buffers: more chunks in flight hide the epilogue's latency.
-  static constexpr int BN = WSMEM ? (RP == 128 ? 64 : 128) : ((RP == 256 || (SPLIT && RP == 128)) ? 64 : 128);
+  // from shared memory (loaded by TMA) instead of TMEM, which leaves TMEM
+  // to the L buffers.
+  static constexpr bool WSMEM = !SPLIT && !LOSS && RP <= 128;
+  // Q rows per chunk (the N of the first product and the K of the second):
+  // as many L buffers as fit in the TMEM left over, so that the chunks in
+  // flight hide the round trip MMA1 -> epilogue -> MMA2 of each buffer.
+#ifndef NMD_BN_BF16_64
+#define NMD_BN_BF16_64 128
+#endif
+  static constexpr int BN = WSMEM ? (RP == 128 ? 64 : NMD_BN_BF16_64)
+                                  : ((RP == 256 || (SPLIT && RP == 128)) ? 64 : 128);
   // TMEM columns of one W tile (hi [+ lo]); none when it sits in shared memory
   static constexpr int WCOLS = WSMEM ? 0 : (SPLIT ? RP : RP / 2);
   static constexpr int W_BYTES = WSMEM ? BM * RP * 2 : 0;   // one W tile in shared memory
@@ -88,10 +90,9 @@ struct Cfg {
   static constexpr int PANEL_BYTES = BN * ROWB;
   static constexpr int NPANEL = RP / PANEL_W;
   static constexpr int OPER_BYTES = BN * RP * 2;       // one bf16 piece of a chunk
-  // bf16 pieces of each chunk in shared memory: the second product always
-  // uses q = hi + lo (three pieces in the fp32-accurate mode); the loss pass
-  // (first product only) needs hi (+ lo when split)
-  static constexpr int NQ = LOSS ? (SPLIT ? 2 : 1) : (SPLIT ? 3 : 2);
+  // bf16 pieces of each chunk in shared memory: hi in the bf16 mode, hi, lo
+  // and lo2 in the fp32-accurate mode (hi and lo in its loss pass)
+  static constexpr int NQ = SPLIT ? (LOSS ? 2 : 3) : 1;
   static constexpr int STAGE_BYTES = OPER_BYTES * NQ;
   // stages within 160 KB with the W tiles (r_pad <= 64: 165 KB in all, so
   // that an update block fits beside the CTA), 192 KB at r_pad = 128
@@ -376,7 +377,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // R += P[lb] x chunk for every chunk once its P is in TMEM; frees the
     // shared-memory stage and the L buffer, and hands R over per tile.
     if (!LOSS) {
-      constexpr uint32_t idesc2 = idesc_bf16(BM, C::FUSEDN ? 2 * RP : C::NR, true, EPI == 1 && !SPLIT);   // Q MN-major
+      constexpr uint32_t idesc2 = idesc_bf16(BM, C::NR, true, EPI == 1 && !SPLIT);   // Q MN-major
       // R columns [hcol, hcol + NR) of Q: their panels start hcol / PANEL_W panels in
       const uint32_t hpan = C::RHALF ? (uint32_t)blockIdx.y * (C::NR / C::PANEL_W) * C::PANEL_BYTES : 0u;
       const int64_t my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
@@ -403,14 +404,11 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int k = 0; k < BN / 16 && !(SKIP && skip); ++k) {
           const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
-          const uint64_t bl = bh + (C::OPER_BYTES >> 4);
           const uint32_t acc = (c2 > 0 || k > 0) ? 1u : 0u;
-          if (C::FUSEDN) {          // P [q_hi | q_lo] into two accumulators side by side
+          if (!SPLIT) {             // P q_hi
             mma_ts_elect(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
-          } else if (!SPLIT) {      // P (q_hi + q_lo)
-            mma_ts_elect(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
-            mma_ts_elect(tmem + C::COL_R, pl + k * 8, bl, idesc2, 1);
           } else {                  // P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
+            const uint64_t bl = bh + (C::OPER_BYTES >> 4);
             const uint64_t bl2 = bh + ((2 * C::OPER_BYTES) >> 4);
             const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
             mma_ts_elect(tmem + C::COL_R, ph, bh, idesc2, acc);
@@ -506,85 +504,88 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t lcol = tmem + lane_base + C::COL_L + lb * BN;
         float c2 = 0.f, c1 = 0.f;
         uint32_t nzacc = 0u;   // Delta form: OR of this thread's P words
-#pragma unroll 1
-        for (int jj = 0; jj < BN / 64; ++jj) {
-          uint32_t v0[32], v1[32];
-          tmem_ld32(lcol + jj * 64, v0);
-          tmem_ld32(lcol + jj * 64 + 32, v1);
-          tmem_wait_ld(v0);
-          tmem_wait_ld(v1);
+        // one group of 32 columns of L (TMEM columns [32 g, 32 g + 32) of the
+        // buffer): mask the columns past the block, then the loss sums or P
+        // (bf16, 16 TMEM columns at 16 g; fp32-accurate: hi and lo, 32 at 32 g,
+        // so P never overwrites L columns that are still to be read)
+        auto group = [&](uint32_t(&v)[32], int g) {
           if (kv < BN) {   // last chunk: columns past the block end contribute nothing
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              if (jj * 64 + i >= kv) v0[i] = LOSS ? 0u : (EPI == 0 ? 0u : 0xff800000u);   // -inf -> relu 0
-              if (jj * 64 + 32 + i >= kv) v1[i] = LOSS ? 0u : (EPI == 0 ? 0u : 0xff800000u);
-            }
+            for (int i = 0; i < 32; ++i)
+              if (g * 32 + i >= kv) v[i] = LOSS ? 0u : (EPI == 0 ? 0u : 0xff800000u);   // -inf -> relu 0
           }
           if (p.Lout != nullptr) {
             const int64_t li = t * BM + row;
             if (li < p.M) {
 #pragma unroll
-              for (int i = 0; i < 32; ++i) {
-                if (jj * 64 + i < kv) p.Lout[li * p.K + c * BN + jj * 64 + i] = __uint_as_float(v0[i]);
-                if (jj * 64 + 32 + i < kv) p.Lout[li * p.K + c * BN + jj * 64 + 32 + i] = __uint_as_float(v1[i]);
-              }
+              for (int i = 0; i < 32; ++i)
+                if (g * 32 + i < kv) p.Lout[li * p.K + c * BN + g * 32 + i] = __uint_as_float(v[i]);
             }
           }
           if (LOSS) {
-            const int64_t cb = c * BN + jj * 64;
-            if (snext < cb + 64) {   // support columns in this group: zero them
+            const int64_t cb = c * BN + g * 32;
+            if (snext < cb + 32) {   // support columns in this group: zero them
 #pragma unroll
-              for (int i = 0; i < 64; ++i) {
+              for (int i = 0; i < 32; ++i) {
                 if (cb + i == snext) {
-                  if (i < 32) v0[i] = 0u; else v1[i - 32] = 0u;
+                  v[i] = 0u;
                   ++se;
                   snext = se < send ? p.cidx[se] : INT64_MAX;
                 }
               }
             }
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float x0 = fmaxf(0.f, __uint_as_float(v0[i])), x1 = fmaxf(0.f, __uint_as_float(v1[i]));
+            for (int i = 0; i < 32; i += 2) {
+              const float x0 = fmaxf(0.f, __uint_as_float(v[i])), x1 = fmaxf(0.f, __uint_as_float(v[i + 1]));
               c2 = fmaf(x0, x0, c2);
               c2 = fmaf(x1, x1, c2);
               c1 += x0 + x1;
             }
           } else if (!SPLIT) {
-            uint32_t pk0[16], pk1[16];
+            uint32_t pk[16];
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
               if (EPI == 0) {   // min(0, L)
-                pk0[i] = min0_bf16x2(pack_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1])));
-                pk1[i] = min0_bf16x2(pack_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1])));
+                pk[i] = min0_bf16x2(pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])));
               } else {          // max(0, L); the MMA negates it
-                pk0[i] = pack_relu_bf16x2(__uint_as_float(v0[2 * i]), __uint_as_float(v0[2 * i + 1]));
-                pk1[i] = pack_relu_bf16x2(__uint_as_float(v1[2 * i]), __uint_as_float(v1[2 * i + 1]));
-                if (SKIP) nzacc |= (pk0[i] | pk1[i]) & 0x7fff7fffu;   // -0 counts as zero
+                pk[i] = pack_relu_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+                if (SKIP) nzacc |= pk[i] & 0x7fff7fffu;   // -0 counts as zero
               }
             }
-            tmem_st16(lcol + jj * 32, pk0);
-            tmem_st16(lcol + jj * 32 + 16, pk1);
+            tmem_st16(lcol + g * 16, pk);
           } else {
-            // fp32-accurate: P = hi + lo, hi at columns [32j, 32j+16), lo at [32j+16, 32j+32)
+            // fp32-accurate: P = hi + lo, hi at columns [32 g, 32 g + 16), lo at [32 g + 16, 32 g + 32)
+            uint32_t ph[16], pl[16];
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              uint32_t(&v)[32] = h == 0 ? v0 : v1;
-              uint32_t ph[16], pl[16];
-#pragma unroll
-              for (int i = 0; i < 16; ++i) {
-                const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
-                const float e0 = EPI == 0 ? fminf(0.f, x0) : fminf(0.f, -x0);
-                const float e1 = EPI == 0 ? fminf(0.f, x1) : fminf(0.f, -x1);
-                const uint32_t hp = pack_bf16x2(e0, e1);
-                const float h0 = __uint_as_float(hp << 16), h1 = __uint_as_float(hp & 0xffff0000u);
-                ph[i] = hp;
-                pl[i] = pack_bf16x2(e0 - h0, e1 - h1);
-                if (SKIP) nzacc |= (ph[i] | pl[i]) & 0x7fff7fffu;   // -0 counts as zero
-              }
-              tmem_st16(lcol + (2 * jj + h) * 32, ph);
-              tmem_st16(lcol + (2 * jj + h) * 32 + 16, pl);
+            for (int i = 0; i < 16; ++i) {
+              const float x0 = __uint_as_float(v[2 * i]), x1 = __uint_as_float(v[2 * i + 1]);
+              const float e0 = EPI == 0 ? fminf(0.f, x0) : fminf(0.f, -x0);
+              const float e1 = EPI == 0 ? fminf(0.f, x1) : fminf(0.f, -x1);
+              const uint32_t hp = pack_bf16x2(e0, e1);
+              const float h0 = __uint_as_float(hp << 16), h1 = __uint_as_float(hp & 0xffff0000u);
+              ph[i] = hp;
+              pl[i] = pack_bf16x2(e0 - h0, e1 - h1);
+              if (SKIP) nzacc |= (ph[i] | pl[i]) & 0x7fff7fffu;   // -0 counts as zero
             }
+            tmem_st16(lcol + g * 32, ph);
+            tmem_st16(lcol + g * 32 + 16, pl);
           }
+        };
+#pragma unroll 1
+        for (int jj = 0; jj < BN / 64; ++jj) {   // two groups per pass, both loads in flight
+          uint32_t v0[32], v1[32];
+          tmem_ld32(lcol + jj * 64, v0);
+          tmem_ld32(lcol + jj * 64 + 32, v1);
+          tmem_wait_ld(v0);
+          tmem_wait_ld(v1);
+          group(v0, 2 * jj);
+          group(v1, 2 * jj + 1);
+        }
+        if (BN % 64 != 0) {   // a last group of 32 columns
+          uint32_t v0[32];
+          tmem_ld32(lcol + (BN / 64) * 64, v0);
+          tmem_wait_ld(v0);
+          group(v0, BN / 32 - 1);
         }
         if (LOSS) {
           s2 += (double)c2;
@@ -616,27 +617,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           // the next tile) before the adds and global stores
           const bool last = j + 2 >= NJ;
           uint32_t v[32];
-          tmem_ld32(tmem + lane_base + C::COL_R + j * 32, v);   // RP = 16 reads 16 spare columns
-          if (C::FUSEDN) {
-            uint32_t u[32];
-            tmem_ld32(tmem + lane_base + C::COL_R + RP + j * 32, u);
-            tmem_wait_ld(v);
-            tmem_wait_ld(u);
-            if (last) {
-              fence_before();
-              __syncwarp();
-              if (lane == 0) mbar_arrive(b_rempty);
-            }
-            if (RP == 16) {   // the accumulators are 16 columns apart: u[i] = v[i + 16]
-#pragma unroll
-              for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + __uint_as_float(v[i + 16]));
-            } else {
-#pragma unroll
-              for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + __uint_as_float(u[i]));
-            }
-          }
+          tmem_ld32(tmem + lane_base + C::COL_R + j * 32, v);   // RP = 16 reads 16 columns past R
           tmem_wait_ld(v);
-          if (!C::FUSEDN && last) {
+          if (last) {
             fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(b_rempty);
@@ -760,13 +743,13 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
   // that the rows of a ragged last tile past the block read as zero
   CUtensorMap tw = th;
   if (C::WSMEM && !tensor_map(fm.hi, p.m0 + p.M, RP, C::PANEL_W, BM, &tw)) return NMD_ERR_CUDA;
-  static bool attr_set = false;
-  if (!attr_set) {
-    if (cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)C::SMEM) != cudaSuccess)
-      return NMD_ERR_CUDA;
-    attr_set = true;
-  }
+  // the shared-memory attribute belongs to the current device
+  static std::atomic<int> attr_set[kMaxDevices];
+  if (!per_device(attr_set, [] {
+        return cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) == cudaSuccess ? 1 : 0;
+      }))
+    return NMD_ERR_CUDA;
   const unsigned gz = p.ksplit ? (unsigned)((p.K + p.ksplit - 1) / p.ksplit) : 1u;
   panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u, gz), kThreads, C::SMEM, s>>>(
       th, tl, tl2, tw, p);

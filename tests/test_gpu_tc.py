@@ -2,7 +2,10 @@
 
 MMA1 (L = M Q^T) through the nmd_dense_products hook against the same
 product of the rounded operands in fp64; MMA2 (R = P(L) Q plus the sparse
-correction) against a CPU restatement fed with the kernel's own L.  Covers
+correction) against a CPU restatement fed with the kernel's own L (in the
+bf16 mode the whole step uses the bf16 rows q_hi: P q_hi plus the support
+term on q_hi, paired with the Gram matrix of q_hi, reported by the hook as
+the equivalent right-hand side under the exact G).  Covers
 every padded rank (16, 32, 64, 128, 256), both epilogues, both tensor-core
 precisions, ragged M and K tails.
 """
@@ -101,18 +104,26 @@ def test_second_product_R(r, n, b, epi, precision):
         P = np.minimum(0, L) if epi == N.NMD_EPI_Z else -np.maximum(0, L)
         Qf = Q.astype(np.float32)
         qh, ql, ql2 = pieces(Qf)
-        if precision == N.NMD_BF16:       # P (q_hi + q_lo)
+        Qd = Qf.astype(np.float64)
+        Sd = src.dense_panel(m0, m1, c0, c1)
+        sup = Sd > 0
+        if precision == N.NMD_BF16:
+            # the whole step on the bf16 rows: R' = P q_hi + c q_hi with
+            # c = S - min(0, m_hi . q_hi) on the support, solved with
+            # Gt = q_hi^T q_hi; the hook reports the right-hand side with the
+            # same solution under the exact G: R' Gt^{-1} G
             Pb = bf16_round(P.astype(np.float32))
-            want = Pb @ (qh + ql)
+            mh = pieces(M[m0:m1].astype(np.float32))[0]
+            Lb = (mh @ qh.T).astype(np.float32).astype(np.float64)
+            corr = np.where(sup, Sd - np.minimum(0, Lb), 0.0)
+            want = (Pb @ qh + corr @ qh) @ np.linalg.solve(qh.T @ qh, Qd.T @ Qd)
         else:                             # P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
             ph = bf16_round(P.astype(np.float32))
             pl = bf16_round((P - ph).astype(np.float32))
             want = ph @ (qh + ql + ql2) + pl @ qh
-        Sd = src.dense_panel(m0, m1, c0, c1)
-        sup = Sd > 0
-        # the support correction uses fp32 L and q: c = S - min(0, L) on the support
-        Lf = (M[m0:m1].astype(np.float32) @ Qf.T).astype(np.float64)
-        corr = np.where(sup, Sd - np.minimum(0, Lf), 0.0)
-        want = want + corr @ Qf.astype(np.float64)
+            # the support correction uses fp32 L and q: c = S - min(0, L) on the support
+            Lf = (M[m0:m1].astype(np.float32) @ Qf.T).astype(np.float64)
+            corr = np.where(sup, Sd - np.minimum(0, Lf), 0.0)
+            want = want + corr @ Qd
         got, _ = sol.block_terms(side, block, kind)
         assert rel(got, want) <= 1e-5, (side, kind, block, rel(got, want))

@@ -60,14 +60,74 @@ def test_block_permutation_golden():
         assert O.block_permutation(seed, sweep, side, K) == row[4:]
 
 
-def test_fisher_yates_uniform_small():
-    """All 3! orders of 3 blocks appear with roughly equal frequency."""
+_SM64 = [row[0] for row in _read_numbers("splitmix64_seed1234567.txt")]
+_GOLDEN_GAMMA = 0x9E3779B97F4A7C15
+
+
+def test_fisher_yates_hand_derived_from_published_vector():
+    """Shuffle of 6 blocks driven by SplitMix64 from state 1234567, derived by
+    hand from the published outputs v1..v5 (tests/golden/splitmix64_seed1234567.txt):
+      i=5: j = v1 mod 6 = 3 -> [0 1 2 5 4 3]
+      i=4: j = v2 mod 5 = 3 -> [0 1 2 4 5 3]
+      i=3: j = v3 mod 4 = 3 -> [0 1 2 4 5 3]
+      i=2: j = v4 mod 3 = 1 -> [0 2 1 4 5 3]
+      i=1: j = v5 mod 2 = 1 -> [0 2 1 4 5 3]"""
+    assert [_SM64[0] % 6, _SM64[1] % 5, _SM64[2] % 4, _SM64[3] % 3, _SM64[4] % 2] == [3, 3, 3, 1, 1]
+    assert O.fisher_yates(6, O.SplitMix64(1234567)) == [0, 2, 1, 4, 5, 3]
+
+
+def test_block_order_state_derivation_from_published_vector():
+    """state = mix(seed) xor mix((sweep << 1) | side), with both mixes taken
+    from the published vector: mix(x) is the first output of a generator
+    started at x - 0x9E3779B97F4A7C15, so mix(1234567 + g) = v1 and
+    mix(1234567 + 2 g) = v2 (g = the golden gamma)."""
+    mask = (1 << 64) - 1
+    x1 = (1234567 + _GOLDEN_GAMMA) & mask
+    x2 = (1234567 + 2 * _GOLDEN_GAMMA) & mask
+    assert O.splitmix64_mix(x1) == _SM64[0] and O.splitmix64_mix(x2) == _SM64[1]
+    seed, sweep, side = x1, x2 >> 1, x2 & 1
+    state = _SM64[0] ^ _SM64[1]
+    for K in (2, 5, 34):
+        assert O.block_permutation(seed, sweep, side, K) == O.fisher_yates(K, O.SplitMix64(state))
+    # swapping the roles of seed and (sweep, side) changes the order
+    assert O.block_permutation(seed, sweep, 1 - side, 34) != O.block_permutation(seed, sweep, side, 34)
+
+
+def _chi2_orders(perm_fn, K=4, samples=24000):
     counts = {}
-    for s in range(6000):
-        p = tuple(O.block_permutation(7, s, 0, 3))
+    for s in range(samples):
+        p = tuple(perm_fn(s))
         counts[p] = counts.get(p, 0) + 1
-    assert len(counts) == 6
-    assert min(counts.values()) > 850 and max(counts.values()) < 1150
+    cells = math.factorial(K)
+    e = samples / cells
+    return len(counts), sum((counts.get(p, 0) - e) ** 2 / e for p in counts) + (cells - len(counts)) * e
+
+
+# chi-square with 23 degrees of freedom: mean 23, sd 6.8; P(chi2 > 60) ~ 4e-5
+_CHI2_23_BOUND = 60.0
+
+
+def test_fisher_yates_uniform_chi_square():
+    """All 4! orders of 4 blocks are equally likely over 24,000 sweeps (chi-square
+    with 23 degrees of freedom below 60)."""
+    seen, chi2 = _chi2_orders(lambda s: O.block_permutation(7, s, 0, 4))
+    assert seen == 24
+    assert chi2 < _CHI2_23_BOUND, chi2
+
+
+def test_chi_square_rejects_the_naive_shuffle():
+    """The same statistic on the classic slip j = next() mod K (a swap with any
+    position at every step: 4^4 = 256 equally likely paths over 24 orders) is
+    far above the bound, so the uniformity test above can tell them apart."""
+    def naive(s):
+        g = O.SplitMix64(O.splitmix64_mix(7) ^ O.splitmix64_mix(s << 1))
+        p = list(range(4))
+        for i in range(3, -1, -1):
+            j = g.next() % 4
+            p[i], p[j] = p[j], p[i]
+        return p
+    _, chi2 = _chi2_orders(naive)
+    assert chi2 > 10 * _CHI2_23_BOUND, chi2
 
 
 # --------------------------------------------------------------------------
