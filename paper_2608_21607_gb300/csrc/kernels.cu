@@ -1032,13 +1032,6 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
   asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
-template <typename T>
-__device__ __forceinline__ float ld(const T* p);
-template <>
-__device__ __forceinline__ float ld<float>(const float* p) { return __ldg(p); }
-template <>
-__device__ __forceinline__ float ld<bf16>(const bf16* p) { return __bfloat162float(*p); }
-
 // ---------------------------------------------------------------------------
 // Loss, support part: for every stored (i, j), with L = w_i . b_j and
 // Shat = max(0, L):
@@ -1270,8 +1263,9 @@ static void update_rp(const StepArgs& a, const float* R, const float* Rs, const 
     return n;
   });
   // one tile per block: blocks retire every few microseconds, so that the
-  // higher-priority streams' kernels (the next step's Gram chain and support
-  // term) get SM slots while a deferred update runs beside the dense kernel;
+  // higher-priority streams' kernels (the dense kernel, the next step's Gram
+  // chain and support term) get SM slots while a deferred update runs.  (One
+  // persistent block per SM instead slowed the dense kernel beside it.)
   // per_sm only bounds the grid when the tiles exceed 65,535 waves' worth
   const int64_t tiles = (a.M + C::TR - 1) / C::TR;
   dim3 grid((unsigned)std::min<int64_t>(tiles, (int64_t)a.num_sms * per_sm * 65535), RP / C::CW);

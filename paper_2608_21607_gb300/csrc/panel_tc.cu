@@ -72,13 +72,10 @@ struct Cfg {
   // to the L buffers.
   static constexpr bool WSMEM = !SPLIT && !LOSS && RP <= 128;
   // Q rows per chunk (the N of the first product and the K of the second):
-  // as many L buffers as fit in the TMEM left over, so that the chunks in
-  // flight hide the round trip MMA1 -> epilogue -> MMA2 of each buffer.
-#ifndef NMD_BN_BF16_64
-#define NMD_BN_BF16_64 128
-#endif
-  static constexpr int BN = WSMEM ? (RP == 128 ? 64 : NMD_BN_BF16_64)
-                                  : ((RP == 256 || (SPLIT && RP == 128)) ? 64 : 128);
+  // 128 where three L buffers of 128 columns fit beside R (bf16 mode at
+  // r_pad <= 64: 3 x 128 + r_pad <= 512); 64 where that would leave fewer
+  // than three.  (Four buffers of 96 rows were slower at r_pad = 64.)
+  static constexpr int BN = WSMEM ? (RP == 128 ? 64 : 128) : ((RP == 256 || (SPLIT && RP == 128)) ? 64 : 128);
   // TMEM columns of one W tile (hi [+ lo]); none when it sits in shared memory
   static constexpr int WCOLS = WSMEM ? 0 : (SPLIT ? RP : RP / 2);
   static constexpr int W_BYTES = WSMEM ? BM * RP * 2 : 0;   // one W tile in shared memory
