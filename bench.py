@@ -43,9 +43,9 @@ WORKLOADS = {
 }
 
 
-# DRAM bytes (read + write) of one dense-kernel launch, from the ncu capture
-# summarised in profiles/dense_panel_connectome_r64_bf16.md; valid only while
-# the kernel's sources hash to the digest recorded with it (else null)
+# DRAM bytes (read + write) of one dense-kernel launch, from an ncu capture of
+# the same workload (dram__bytes_read.sum + dram__bytes_write.sum); valid only
+# while the kernel's sources hash to the digest recorded with it (else null)
 DENSE_TRAFFIC = {
     # (workload, precision, epilogue): (bytes per launch, dense_source_digest() of the code measured)
     ("connectome-139255-r64", "bf16", "z"): (18920362, "2343bf0ed2467707"),
@@ -65,6 +65,52 @@ def dense_source_digest():
                 if code:
                     h.update(code.encode() + b"\n")
     return h.hexdigest()[:16]
+
+
+def support_bytes_per_sweep(wl, elem_bytes):
+    """Algorithmic bytes of the support term over one sweep (each step once):
+    per support entry its index and value (8 B) and the q row (r elements);
+    per M-side row with support in the step's panel its m row (r elements)
+    and its row of Rs (r fp32 values, written).  Every nonzero is in one
+    column step and one row step; the panel rows are counted per step."""
+    import numpy as np
+    S = wl.S
+    rows = np.repeat(np.arange(S.m, dtype=np.int64), np.diff(S.row_ptr))
+    cols = np.asarray(S.col_idx, np.int64)
+    # column steps: (row, column block) pairs; row steps: (column, row block) pairs
+    col_pairs = np.unique(rows * (-(-S.n // wl.block_cols)) + cols // wl.block_cols).size
+    row_pairs = np.unique(cols * (-(-S.m // wl.block_rows)) + rows // wl.block_rows).size
+    nnz = int(S.row_ptr[-1])
+    return 2 * nnz * (8 + elem_bytes * wl.r) + (col_pairs + row_pairs) * (elem_bytes * wl.r + 4 * wl.r)
+
+
+def measure_support(sol, wl, N):
+    """The support-term kernels alone (nmd_support_term, no other work on the
+    GPU) over every step of one sweep, timed with CUDA events on the solver's
+    stream: ms for the sweep's steps."""
+    import torch
+    pr, pc = sol.block_order(0, N.NMD_ROW), sol.block_order(0, N.NMD_COL)
+    if wl.schedule == "exact":
+        order = [(N.NMD_ROW, b, N.NMD_EXACT) for b in pr] + [(N.NMD_COL, b, N.NMD_EXACT) for b in pc]
+    else:   # alternating stochastic sweep
+        order = []
+        for t in range(max(len(pr), len(pc))):
+            if t < len(pc):
+                order.append((N.NMD_COL, int(pc[t]), N.NMD_STOCH))
+            if t < len(pr):
+                order.append((N.NMD_ROW, int(pr[t]), N.NMD_STOCH))
+    buf = torch.empty(max(wl.m, wl.n) * sol.r_pad, dtype=torch.float32, device=sol.device)
+    st = sol.stream
+    for side, block, kind in order[:4]:
+        sol.support_term(side, block, kind, buf)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sol.sync()
+    e0.record(st)
+    for side, block, kind in order:
+        sol.support_term(side, block, kind, buf)
+    e1.record(st)
+    sol.sync()
+    return e0.elapsed_time(e1), len(order)
 
 
 def peaks():
@@ -215,6 +261,7 @@ def main():
                     help="factor start: iid N(0, 0.01), or the sign-structured start W > 0, H < 0")
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing on the host")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg (profiling runs)")
+    ap.add_argument("--no-modes", action="store_true", help="skip the fp32-accurate mode's sweep timing")
     ap.add_argument("--kernel-table", action="store_true",
                     help="dense kernel alone at the paper's kernel-table shape (m = 250000 rows against a "
                          "block of 2500), one JSON line per factor rank r and precision (rank 0 only)")
@@ -339,6 +386,7 @@ def main():
     flops_per_launch = flops_sweep / launches_per_sweep
     pk, pk_kind = peaks()
     peak = pk.get("bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])
+    burst = pk.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
     achieved = flops_sweep * args.steps / (dense_ms / 1e3) / 1e12 if dense_ms > 0 else None
     traffic = None
     rec = DENSE_TRAFFIC.get((wl.name, args.precision, args.epilogue))
@@ -346,15 +394,67 @@ def main():
         traffic = rec[0]
     roofline = {"bound": "tensor", "kernel": "panel_tc_kernel (fused Z-panel, tcgen05)",
                 "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
-                "frac": (achieved / peak) if achieved else None, "traffic": traffic,
+                "frac": (achieved / peak) if achieved else None,
+                "frac_of_burst": (achieved / burst) if achieved else None, "traffic": traffic,
                 "traffic_unit": "bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum)",
                 "peak_kind": "%s bf16 dense, sustained" % pk_kind,
                 "flops_per_launch": flops_per_launch, "launches": dense_n,
                 "avg_launch_us": 1e3 * dense_ms / max(dense_n, 1),
                 "share_of_step": dense_ms / ms_total if ms_total > 0 else None,
-                "other_kernels_ms": {k: v[0] for k, v in other.items()}}
+                "other_kernels_ms_per_sweep": {k: v[0] / args.steps for k, v in other.items()}}
     if prec == N.NMD_FP32:
         roofline["note"] = "fp32-accurate mode issues 3 bf16 MMAs per product; flops counted once"
+
+    # support term alone (HBM roofline by algorithmic bytes)
+    hbm = pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+    sp_ms, sp_steps = measure_support(sol, wl, N)
+    sp_bytes = support_bytes_per_sweep(wl, 2 if prec == N.NMD_BF16 else 4)
+    sp_gbs = sp_bytes / (sp_ms / 1e3) / 1e9
+    roofline_sparse = {"bound": "hbm", "kernel": "support term (sparse_rows_kernel, sparse_long_kernel, "
+                                                 "sparse_reduce_kernel), alone",
+                       "achieved": sp_gbs, "peak": hbm, "unit": "GB/s", "frac": sp_gbs / hbm,
+                       "traffic": None, "peak_kind": "%s copy bandwidth" % pk_kind,
+                       "bytes_per_sweep": sp_bytes, "ms_per_sweep": sp_ms, "steps": sp_steps,
+                       "bytes_rule": "per support entry 8 B + r operand elements; per panel row r operand "
+                                     "elements + 4 r B (Rs); operands bf16 in the bf16 mode"}
+
+    # the fp32-accurate mode on the same workload and start, same run
+    modes = None
+    if prec == N.NMD_BF16 and not args.no_modes:
+        sol2 = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols,
+                        schedule=N.NMD_EXACT if exact else N.NMD_STOCH, eta=wl.eta, gamma=wl.gamma,
+                        precision=N.NMD_FP32, epilogue=epi, seed=0)
+        sol2.set_factors(W0, H0)
+        for _ in range(args.warmup):
+            sol2.sweep()
+        sol2.sync()
+        k2 = min(args.steps, 5)
+        clocks2 = ClockSampler(local)
+        clocks2.start()
+        sol2.profile(True)
+        f0, f1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ms2 = 0.0
+        for _ in range(k2):
+            if flush:
+                with torch.cuda.stream(sol2.stream):
+                    scratch.fill_(1)
+            f0.record(sol2.stream)
+            sol2.sweep()
+            f1.record(sol2.stream)
+            sol2.sync()
+            ms2 += f0.elapsed_time(f1)
+        d2_ms, d2_n = sol2.profile_read(N.NMD_K_DENSE)
+        sol2.profile(False)
+        clk2 = clocks2.stop()
+        ach2 = flops_sweep * k2 / (d2_ms / 1e3) / 1e12 if d2_ms > 0 else None
+        modes = {"fp32": {"ms_per_sweep": ms2 / k2, "value": entries * k2 / (ms2 / 1e3), "unit": "Z entries/s",
+                          "sweeps": k2, "dense_tflops_algorithmic": ach2,
+                          "dense_frac_of_burst": (ach2 / burst) if ach2 else None,
+                          "dense_avg_launch_us": 1e3 * d2_ms / max(d2_n, 1), "clocks": clk2,
+                          "note": "fp32-accurate mode (three bf16 pieces per factor; the tensor cores run 3 "
+                                  "MMAs per first product and 4 per second); flops counted once"}}
+        del sol2
+        torch.cuda.empty_cache()
 
     # ---------------- end to end through the public API, host buffers -------
     Wh = torch.from_numpy(np.ascontiguousarray(W0, np.float32)).pin_memory()
@@ -406,7 +506,8 @@ def main():
                            "workspace_mb": round(ws_bytes / 2**20, 1),
                            "l2": ("workspace smaller than L2: L2 flushed (512 MB write) before each timed sweep"
                                   if flush else "workspace larger than L2 (%.0f MB): no flush" % (ws_bytes / 2**20))},
-                "e2e": e2e, "roofline": roofline, "cpu_baseline": cpu, "clocks": clk,
+                "e2e": e2e, "roofline": roofline, "roofline_sparse": roofline_sparse, "modes": modes,
+                "cpu_baseline": cpu, "clocks": clk,
                 "gpu_launches": launches}
         print(json.dumps(line))
     rep.close()

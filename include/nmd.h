@@ -61,15 +61,22 @@ typedef enum { NMD_ROW = 0, NMD_COL = 1 } nmd_side;
 typedef enum { NMD_EXACT = 0, NMD_STOCH = 1 } nmd_kind;
 typedef enum { NMD_ALTERNATE = 0, NMD_PHASED = 1 } nmd_order;
 
-/* Arithmetic of the dense Z-panel contraction and of the loss:
- *   NMD_BF16 -- operands rounded to bf16 (round to nearest even), products on
- *               the tcgen05 tensor cores with fp32 accumulation;
- *   NMD_FP32 -- fp32-accurate: every operand x is split as x = hi + lo with
- *               hi = bf16(x), lo = bf16(x - hi) and each product is formed as
- *               hi*hi + hi*lo + lo*hi on the tensor cores (3 MMAs, fp32 accumulate);
+/* Arithmetic of a block step's least-squares problem (each factor is kept as
+ * fp32 masters plus bf16 pieces hi = bf16(x), lo = bf16(x - hi),
+ * lo2 = bf16(x - hi - lo), all rounded to nearest even):
+ *   NMD_BF16 -- the step is set up on the bf16-rounded rows: the dense term
+ *               (L = M_hi Q_hi^T and R = P Q_hi on the tcgen05 tensor cores,
+ *               fp32 accumulation), the support term (on the hi pieces) and
+ *               the Gram matrix G = Q_hi^T Q_hi all use them, so the rounding
+ *               is not a coherent error between R and G; the update itself is
+ *               applied to the fp32 masters;
+ *   NMD_FP32 -- fp32-accurate: L = M_hi Q_hi^T + M_hi Q_lo^T + M_lo Q_hi^T,
+ *               P = P_hi + P_lo (two bf16 pieces), R = P_hi (Q_hi + Q_lo +
+ *               Q_lo2) + P_lo Q_hi on the tensor cores; the support term and
+ *               G from the fp32 masters;
  *   NMD_SIMT -- plain fp32 FMA on the CUDA cores (slow; reference path).
- * Gram matrices, Cholesky, solves and updates are fp32 in every mode;
- * loss reductions are fp64. */
+ * Gram matrices are formed in fp32, factored in fp32 (L D L^T Cholesky form),
+ * updates are fp32; loss reductions are fp64. */
 typedef enum { NMD_BF16 = 0, NMD_FP32 = 1, NMD_SIMT = 2 } nmd_precision;
 
 /* Form of the dense contraction (both give the same update, Sec. 3.2):
@@ -113,7 +120,9 @@ const char* nmd_version(void);
 void nmd_default_options(nmd_options* opts);
 
 /* Device workspace (bytes) nmd_create needs for this problem.  Validates the
- * CSR exactly as nmd_create does.  The workspace must be 256-byte aligned. */
+ * CSR exactly as nmd_create does (the number of nonzeros is row_ptr[m]; the
+ * size depends on the block panels, so the CSR itself is an argument).  The
+ * workspace must be 256-byte aligned. */
 nmd_status nmd_workspace_bytes(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
                                const int32_t* col_idx, const float* vals,
                                const nmd_options* opts, size_t* bytes);
@@ -196,6 +205,19 @@ nmd_status nmd_block_terms(nmd_handle* h, int32_t side, int64_t block, int32_t k
  * NMD_SIMT.  Synchronises. */
 nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* d_L,
                               int64_t* rows, int64_t* cols);
+
+/* Verification and timing hook: the support term of one block update alone
+ * (the sparse correction of eqs. updateZ/updateD, Sec. 3.2): for every M-side
+ * row i with support in the block's panel,
+ *   Rs_i = sum over the panel's entries (i, k) of (S_ik - min(0, L_ik)) q_k,
+ * with L_ik = m_i . q_k, and Rs_i = 0 on the other rows.  The step's own
+ * operands are used: the bf16 pieces of both factors in the NMD_BF16 mode,
+ * the fp32 masters otherwise.  d_R: caller-owned device memory of rows x
+ * r_pad floats, row-major, r_pad = r rounded up to 16, 32, 64, 128 or 256;
+ * *rows (if not NULL) receives the number of M-side rows.  Asynchronous on
+ * the handle's stream (it first waits for any deferred update of a sweep),
+ * so the caller can time it with events. */
+nmd_status nmd_support_term(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* d_R, int64_t* rows);
 
 /* Verification hook: the sparse traversal of one block update -- for every
  * M-side row with support in the block's panel, ascending, its entries in

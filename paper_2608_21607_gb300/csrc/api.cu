@@ -1083,6 +1083,32 @@ nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_
   return NMD_OK;
 }
 
+nmd_status nmd_support_term(nmd_handle* h, int32_t side, int64_t block, int32_t kind, float* d_R, int64_t* rows) {
+  if (!h || !d_R) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_support_term");
+  DeviceScope dg(h);
+  Roles ro;
+  nmd_status st = roles(h, side, block, kind, &ro);
+  if (st != NMD_OK) return st;
+  if ((st = wait_all_pending(h)) != NMD_OK) return st;
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
+              h->opt.skip_zero_chunks != 0};
+  const PanelSet& P = *ro.P;
+  const int64_t r0 = P.row_ptr[block], r1 = P.row_ptr[block + 1];
+  const int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1], gd = g0 + P.segd[block];
+  const int64_t u0 = P.multi_ptr[block], u1 = P.multi_ptr[block + 1];
+  cudaStream_t s = h->stream;
+  CK(h, cudaMemsetAsync(d_R, 0, (size_t)ro.M * h->rp * sizeof(float), s));
+  {
+    TimedScope ts(h, NMD_K_SPARSE, s);
+    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, gd - g0, P.d_seg + gd, g1 - gd, P.d_multi + u0, u1 - u0,
+                  ro.qidx, ro.vals, d_R, h->ws.seg_partials, s);
+    h->launches += (r1 > r0) + (gd > g0) + 2 * (g1 > gd);
+  }
+  if ((st = after_launch(h, "support term")) != NMD_OK) return st;
+  if (rows) *rows = ro.M;
+  return NMD_OK;
+}
+
 nmd_status nmd_panel_traversal(const nmd_handle* h, int32_t side, int64_t block, int32_t kind,
                                int64_t* rows_out, int64_t* q_out, int64_t cap, int64_t* count) {
   if (!h || !count) return NMD_ERR_INVALID;

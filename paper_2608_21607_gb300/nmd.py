@@ -31,7 +31,7 @@ EXPORTS = [
     "nmd_get_factors", "nmd_block_update", "nmd_sweep", "nmd_block_order", "nmd_loss", "nmd_sync",
     "nmd_block_terms", "nmd_dense_products", "nmd_panel_traversal", "nmd_get_state", "nmd_set_state",
     "nmd_launch_count", "nmd_skip_count", "nmd_selftest_wait_timeout", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
-    "nmd_destroy", "nmd_gram_noalloc",
+    "nmd_destroy", "nmd_gram_noalloc", "nmd_support_term",
 ]
 
 
@@ -95,6 +95,7 @@ def lib() -> C.CDLL:
             "nmd_last_error": (C.c_char_p, [_P]),
             "nmd_destroy": (None, [_P]),
             "nmd_gram_noalloc": (C.c_int, [_P, C.c_int64, C.c_int32, C.c_int64, _P, _P]),
+            "nmd_support_term": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int32, _P, _i64p]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -218,6 +219,12 @@ def nmd_panel_traversal(h, side, block, kind):
     _check(h, L.nmd_panel_traversal(h, side, block, kind, rows.ctypes.data, q.ctypes.data, cnt.value,
                                     C.byref(cnt)), "traversal")
     return rows, q
+
+
+def nmd_support_term(h, side, block, kind, d_R) -> int:
+    rows = C.c_int64(0)
+    _check(h, lib().nmd_support_term(h, side, block, kind, _ptr(d_R), C.byref(rows)), "nmd_support_term")
+    return rows.value
 
 
 def nmd_get_state(h, m, n, r):
@@ -354,6 +361,19 @@ class Solver:
 
     def panel_traversal(self, side, block, kind):
         return nmd_panel_traversal(self.h, side, block, kind)
+
+    @property
+    def r_pad(self) -> int:
+        return next(p for p in (16, 32, 64, 128, 256) if self.r <= p)
+
+    def support_term(self, side, block, kind, d_R=None):
+        """The support term Rs of one block update (rows x r_pad, device
+        tensor); asynchronous on the solver's stream."""
+        import torch
+        if d_R is None:
+            d_R = torch.empty(max(self.m, self.n) * self.r_pad, dtype=torch.float32, device=self.device)
+        rows = nmd_support_term(self.h, side, block, kind, d_R)
+        return d_R[:rows * self.r_pad].view(rows, self.r_pad)
 
     def get_state(self):
         return nmd_get_state(self.h, self.m, self.n, self.r)
