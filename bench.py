@@ -86,8 +86,9 @@ def support_bytes_per_sweep(wl, elem_bytes):
 
 def measure_support(sol, wl, N):
     """The support-term kernels alone (nmd_support_term, no other work on the
-    GPU) over every step of one sweep, timed with CUDA events on the solver's
-    stream: ms for the sweep's steps."""
+    GPU) over every step of one sweep: device ms of the kernels (CUDA events
+    the library records around each step's support-term launches, on the
+    stream they run on; the hook's clearing of its output buffer is outside)."""
     import torch
     pr, pc = sol.block_order(0, N.NMD_ROW), sol.block_order(0, N.NMD_COL)
     if wl.schedule == "exact":
@@ -100,17 +101,15 @@ def measure_support(sol, wl, N):
             if t < len(pr):
                 order.append((N.NMD_ROW, int(pr[t]), N.NMD_STOCH))
     buf = torch.empty(max(wl.m, wl.n) * sol.r_pad, dtype=torch.float32, device=sol.device)
-    st = sol.stream
     for side, block, kind in order[:4]:
         sol.support_term(side, block, kind, buf)
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sol.sync()
-    e0.record(st)
+    sol.profile(True)
     for side, block, kind in order:
         sol.support_term(side, block, kind, buf)
-    e1.record(st)
-    sol.sync()
-    return e0.elapsed_time(e1), len(order)
+    ms, _ = sol.profile_read(N.NMD_K_SPARSE)
+    sol.profile(False)
+    return ms, len(order)
 
 
 def peaks():

@@ -143,7 +143,9 @@ nmd_status build_sparse(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
 }
 
 // Split every block's rows (ascending) into short rows (len <= kShort), whole
-// long rows (len <= kSeg) and kSeg slices of the longer rows.
+// long rows (len <= seg) and slices of seg entries of the longer rows, with
+// seg = the largest of kSegMax, kSegMax / 2, ... kSegMin whose segments of the
+// block's long rows number at least kSegTarget (else kSegMin).
 void finalize_panels(const std::vector<std::vector<PanelRow>>& per, PanelSet* P) {
   int64_t K = (int64_t)per.size();
   P->host.clear(); P->seg.clear(); P->multi.clear();
@@ -156,18 +158,23 @@ void finalize_panels(const std::vector<std::vector<PanelRow>>& per, PanelSet* P)
     P->row_ptr[k] = (int64_t)P->host.size();
     P->seg_ptr[k] = (int64_t)P->seg.size();
     P->multi_ptr[k] = (int64_t)P->multi.size();
+    int64_t long_entries = 0;
+    for (const PanelRow& pr : per[k])
+      if (pr.len > kShort) long_entries += pr.len;
+    int seg = kSegMax;
+    while (seg > kSegMin && long_entries / seg < kSegTarget) seg /= 2;
     for (const PanelRow& pr : per[k]) {
       if (pr.len <= kShort) P->host.push_back(pr);
-      else if (pr.len <= kSeg) P->seg.push_back(pr);
+      else if (pr.len <= seg) P->seg.push_back(pr);
     }
     P->segd[k] = (int64_t)P->seg.size() - P->seg_ptr[k];
     const int64_t s0 = (int64_t)P->seg.size();
     for (const PanelRow& pr : per[k]) {
-      if (pr.len <= kSeg) continue;
+      if (pr.len <= seg) continue;
       int64_t first = (int64_t)P->seg.size() - s0;   // slot within the block's slices
       int32_t nseg = 0;
-      for (int64_t off = 0; off < pr.len; off += kSeg, ++nseg)
-        P->seg.push_back(PanelRow{pr.row, (int32_t)std::min<int64_t>(kSeg, pr.len - off), pr.beg + off});
+      for (int64_t off = 0; off < pr.len; off += seg, ++nseg)
+        P->seg.push_back(PanelRow{pr.row, (int32_t)std::min<int64_t>(seg, pr.len - off), pr.beg + off});
       P->multi.push_back(PanelRow{pr.row, nseg, first});
     }
     P->max_segments = std::max<int64_t>(P->max_segments, (int64_t)P->seg.size() - s0);

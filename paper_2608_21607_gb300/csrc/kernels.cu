@@ -532,83 +532,123 @@ inline size_t ldlt_reg_smem_bytes(int rp) {
 
 // ---------------------------------------------------------------------------
 // Sparse correction: for every panel row i and entry (i, k) in the block,
-// L_ik = m_i . q_k, c = S_ik - min(0, L_ik), R_i += c q_k (fp32 masters).
-// This kernel takes the rows with at most kShort entries in the panel: one
-// warp per row; the lanes first fetch the entries' indices and values (one
-// per lane), then NE entries at a time are processed with their q rows in
-// flight together, lanes over the r columns; the accumulation order over
-// the entries stays ascending.  The result goes to Rs, the support term of
-// R, one writer per row (or to a partial slot when `partials` is given).
-// Rs is written only on the rows with support in the block's panel; a flag
-// byte per row tells the update which rows of Rs to add, so the other rows
-// are neither read nor cleared.  Longer rows: sparse_long_kernel below.
+// L_ik = m_i . q_k, c = S_ik - min(0, L_ik), R_i += c q_k, on the step's
+// operands (the bf16 pieces in the bf16 mode, else the fp32 masters).
+// This kernel takes the rows with at most kShort entries in the panel (the
+// connectome's panels average 1.3 entries per row): each row gets LPR lanes,
+// one 16-byte load of its row segment each (8 bf16 or 4 fp32 values; two at
+// r_pad = 256 in fp32), so a warp works on 32 / LPR rows at once and their
+// loads are in flight together.  The lanes of a row first fetch the entries'
+// indices and values (one entry per lane), then NE entries at a time are
+// processed with their q rows in flight together; each dot product is summed
+// over the row's lanes by a butterfly, and the accumulation over the entries
+// stays in ascending order.  The result goes to Rs, the support term of R,
+// one writer per row.  Rs is written only on the rows with support in the
+// block's panel; a flag byte per row tells the update which rows of Rs to
+// add, so the other rows are neither read nor cleared.  Longer rows:
+// sparse_long_kernel below.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float ldv(const float* p) { return __ldg(p); }
 __device__ __forceinline__ float ldv(const bf16* p) { return __bfloat162float(__ldg(p)); }
 
-template <int VPL, int NE, typename T>
-__global__ void __launch_bounds__(256) sparse_rows_kernel(const PanelRow* __restrict__ rows, int64_t nrows,
-                                                          const T* __restrict__ Mop, int64_t m0,
-                                                          const T* __restrict__ Qop,
-                                                          const int32_t* __restrict__ qidx,
-                                                          const float* __restrict__ vals,
-                                                          float* __restrict__ R, float* __restrict__ partials,
-                                                          int rp) {
-  const int lane = threadIdx.x & 31;
-  const int64_t w = (blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5;
-  if (w >= nrows) return;
-  const PanelRow pr = rows[w];
-  const int64_t i = pr.row;
-  int kl = 0;
-  float sl = 0.f;
-  if (lane < pr.len) {
-    kl = qidx[pr.beg + lane];
-    sl = vals[pr.beg + lane];
+// 16 bytes of a factor row as floats: 8 bf16 or 4 fp32 values
+__device__ __forceinline__ void load16(float* f, const bf16* p) {
+  const uint4 u = __ldg((const uint4*)p);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    f[2 * q] = __uint_as_float(w[q] << 16);
+    f[2 * q + 1] = __uint_as_float(w[q] & 0xffff0000u);
   }
-  float mv[VPL], acc[VPL];
+}
+__device__ __forceinline__ void load16(float* f, const float* p) {
+  const float4 v = __ldg((const float4*)p);
+  f[0] = v.x; f[1] = v.y; f[2] = v.z; f[3] = v.w;
+}
+
+template <int RP, typename T>
+__global__ void __launch_bounds__(256, 4) sparse_group_kernel(const PanelRow* __restrict__ rows, int64_t nrows,
+                                                           const T* __restrict__ Mop, int64_t m0,
+                                                           const T* __restrict__ Qop,
+                                                           const int32_t* __restrict__ qidx,
+                                                           const float* __restrict__ vals, float* __restrict__ R) {
+  constexpr int E16 = 16 / (int)sizeof(T);               // elements per 16-byte load
+  constexpr int LPR = RP / E16 < 32 ? RP / E16 : 32;     // lanes per row
+  constexpr int CH = RP / (E16 * LPR);                   // 16-byte loads per lane and row
+  constexpr int EPL = E16 * CH;                          // elements per lane
+  constexpr int RPW = 32 / LPR;                          // rows per warp
+  constexpr int NE = 2;                                  // entries whose q rows load together
+  const int lane = threadIdx.x & 31, sub = lane % LPR, grp = lane / LPR;
+  const int64_t wbase = ((blockIdx.x * (int64_t)blockDim.x + threadIdx.x) >> 5) * RPW;
+  if (wbase >= nrows) return;                            // warp-uniform
+  const int64_t w = wbase + grp;
+  const bool live_row = w < nrows;
+  const PanelRow pr = live_row ? rows[w] : PanelRow{0, 0, 0};
+  float mv[EPL], acc[EPL];
 #pragma unroll
-  for (int v = 0; v < VPL; ++v) {
-    const int c = lane + 32 * v;
-    mv[v] = c < rp ? ldv(Mop + i * rp + c) : 0.f;
-    acc[v] = 0.f;
+  for (int c = 0; c < CH; ++c) {
+    if (live_row) load16(mv + c * E16, Mop + (int64_t)pr.row * RP + (c * LPR + sub) * E16);
+    else
+#pragma unroll
+      for (int q = 0; q < E16; ++q) mv[c * E16 + q] = 0.f;
   }
-  for (int e = 0; e < pr.len; e += NE) {
-    float qv[NE][VPL], part[NE];
-    float sv[NE];
 #pragma unroll
-    for (int j = 0; j < NE; ++j) {
-      const int k = __shfl_sync(0xffffffffu, kl, (e + j) & 31);
-      sv[j] = __shfl_sync(0xffffffffu, sl, (e + j) & 31);
-      const bool live = e + j < pr.len;
-      part[j] = 0.f;
+  for (int q = 0; q < EPL; ++q) acc[q] = 0.f;
+  int maxlen = pr.len;                                   // longest row of the warp
 #pragma unroll
-      for (int v = 0; v < VPL; ++v) {
-        const int c = lane + 32 * v;
-        qv[j][v] = (live && c < rp) ? ldv(Qop + (int64_t)k * rp + c) : 0.f;
-        part[j] = fmaf(mv[v], qv[j][v], part[j]);
+  for (int o = 16; o > 0; o >>= 1) maxlen = max(maxlen, __shfl_xor_sync(0xffffffffu, maxlen, o));
+  for (int e0 = 0; e0 < maxlen; e0 += LPR) {
+    int kl = -1;
+    float sl = 0.f;
+    if (e0 + sub < pr.len) {                             // lane sub holds entry e0 + sub of its row
+      kl = __ldg(qidx + pr.beg + e0 + sub);
+      sl = __ldg(vals + pr.beg + e0 + sub);
+    }
+    const int nb = min(LPR, maxlen - e0);                // warp-uniform
+    for (int j0 = 0; j0 < nb; j0 += NE) {
+      float qv[NE][EPL], part[NE], sv[NE];
+#pragma unroll
+      for (int j = 0; j < NE; ++j) {
+        const int src = grp * LPR + ((j0 + j) & (LPR - 1));
+        const int k = __shfl_sync(0xffffffffu, kl, src);
+        sv[j] = __shfl_sync(0xffffffffu, sl, src);
+        const bool live = j0 + j < nb && k >= 0;
+#pragma unroll
+        for (int c = 0; c < CH; ++c) {
+          if (live) load16(qv[j] + c * E16, Qop + (int64_t)k * RP + (c * LPR + sub) * E16);
+          else
+#pragma unroll
+            for (int q = 0; q < E16; ++q) qv[j][c * E16 + q] = 0.f;
+        }
+        part[j] = 0.f;
+#pragma unroll
+        for (int q = 0; q < EPL; ++q) part[j] = fmaf(mv[q], qv[j][q], part[j]);
+      }
+#pragma unroll
+      for (int o = 1; o < LPR; o <<= 1)
+#pragma unroll
+        for (int j = 0; j < NE; ++j) part[j] += __shfl_xor_sync(0xffffffffu, part[j], o);
+#pragma unroll
+      for (int j = 0; j < NE; ++j) {
+        const float cval = sv[j] - fminf(0.f, part[j]);   // zero for padding entries (s = 0, q = 0)
+#pragma unroll
+        for (int q = 0; q < EPL; ++q) acc[q] = fmaf(cval, qv[j][q], acc[q]);
       }
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
-#pragma unroll
-      for (int j = 0; j < NE; ++j) part[j] += __shfl_xor_sync(0xffffffffu, part[j], o);
-#pragma unroll
-    for (int j = 0; j < NE; ++j) {
-      const float cval = sv[j] - fminf(0.f, part[j]);        // zero for the padding entries (q = 0)
-#pragma unroll
-      for (int v = 0; v < VPL; ++v) acc[v] = fmaf(cval, qv[j][v], acc[v]);
-    }
   }
-  float* dst = partials ? partials + w * rp : R + (i - m0) * rp;
+  if (live_row) {
+    float* dst = R + (pr.row - m0) * RP;
 #pragma unroll
-  for (int v = 0; v < VPL; ++v) {
-    const int c = lane + 32 * v;
-    if (c < rp) dst[c] = acc[v];
+    for (int c = 0; c < CH; ++c)
+#pragma unroll
+      for (int q = 0; q < E16; q += 4)
+        *(float4*)(dst + (c * LPR + sub) * E16 + q) =
+            make_float4(acc[c * E16 + q], acc[c * E16 + q + 1], acc[c * E16 + q + 2], acc[c * E16 + q + 3]);
   }
 }
 
-// Long rows (more than kShort entries in the panel): one warp per row or kSeg
-// slice with the lanes over the entries.  LPE = rp / 32 lanes share an entry
+// Long rows (more than kShort entries in the panel): one warp per segment (a
+// whole row, or a slice of a longer one), with the lanes over the entries.  LPE = rp / 32 lanes share an entry
 // (lane sub = lane % LPE owns columns 32 sub ... 32 sub + 31; CPL = min(32, rp)
 // of them are real), so a warp takes EPW = 32 / LPE entries at a time.  The
 // q rows of those entries are first copied into a per-warp shared buffer with
@@ -1218,11 +1258,13 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
   // The support term reads the same factor values as the rest of the step's
   // least-squares problem: the bf16 pieces in the bf16 mode (whose dense term
   // and Gram matrix are formed from them), the fp32 masters otherwise.
-#define NMD_SP(V, LPE, CPL, TT, MOP, QOP)                                                                    \
+#define NMD_SP(RPV, LPE, CPL, TT, MOP, QOP)                                                                  \
   do {                                                                                                       \
-    if (nrows > 0)                                                                                           \
-      sparse_rows_kernel<V, 4, TT><<<(unsigned)((nrows + 7) / 8), 256, 0, s>>>(rows, nrows, MOP, a.m0, QOP, qidx, \
-                                                                               vals, R, nullptr, a.rp);     \
+    if (nrows > 0) {                                                                                         \
+      constexpr int rpw = 32 / ((RPV) / (16 / (int)sizeof(TT)) < 32 ? (RPV) / (16 / (int)sizeof(TT)) : 32);  \
+      const int64_t nb = (nrows + 8 * rpw - 1) / (8 * rpw);                                                  \
+      sparse_group_kernel<RPV, TT><<<(unsigned)nb, 256, 0, s>>>(rows, nrows, MOP, a.m0, QOP, qidx, vals, R); \
+    }                                                                                                        \
     if (nwhole > 0)                                                                                          \
       sparse_long_kernel<LPE, CPL, TT><<<(unsigned)((nwhole + 7) / 8), 256, 0, s>>>(                          \
           whole, nwhole, MOP, a.m0, QOP, qidx, vals, R, nullptr, a.rp);                                      \
@@ -1232,17 +1274,17 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
       launch_reduce(multi, nmulti, partials, R, a.m0, a.rp, s);                                              \
     }                                                                                                        \
   } while (0)
-#define NMD_SP2(V, LPE, CPL)                                                                \
+#define NMD_SP2(RPV, LPE, CPL)                                                              \
   do {                                                                                      \
-    if (a.precision == NMD_BF16) NMD_SP(V, LPE, CPL, bf16, a.fm->hi, a.fq->hi);             \
-    else NMD_SP(V, LPE, CPL, float, a.fm->master, a.fq->master);                            \
+    if (a.precision == NMD_BF16) NMD_SP(RPV, LPE, CPL, bf16, a.fm->hi, a.fq->hi);           \
+    else NMD_SP(RPV, LPE, CPL, float, a.fm->master, a.fq->master);                          \
   } while (0)
   switch (a.rp) {
-    case 16: NMD_SP2(1, 1, 16); break;
-    case 32: NMD_SP2(1, 1, 32); break;
-    case 64: NMD_SP2(2, 2, 32); break;
-    case 128: NMD_SP2(4, 4, 32); break;
-    default: NMD_SP2(8, 8, 32); break;
+    case 16: NMD_SP2(16, 1, 16); break;
+    case 32: NMD_SP2(32, 1, 32); break;
+    case 64: NMD_SP2(64, 2, 32); break;
+    case 128: NMD_SP2(128, 4, 32); break;
+    default: NMD_SP2(256, 8, 32); break;
   }
 #undef NMD_SP2
 #undef NMD_SP

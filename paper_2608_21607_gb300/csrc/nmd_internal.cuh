@@ -41,20 +41,26 @@ struct PanelRow {
   int64_t beg;
 };
 
-// Panel rows of at most kShort entries are handled one warp per row with the
-// lanes over the r columns.  Longer rows go to a kernel that puts the lanes
-// over the entries, in segments of at most kSeg entries: a row of at most
-// kSeg entries is one segment that writes its result directly; a longer row
-// is split, each segment's partial sum goes to a scratch slot and the slots
-// of a row are added in a fixed order by a second pass.
+// Panel rows of at most kShort entries go to the grouped short-row kernel (a
+// few lanes per row).  Longer rows go to a kernel that puts the lanes over
+// the entries, in segments of at most `seg` entries (chosen per block): a row
+// of at most `seg` entries is one segment that writes its result directly; a
+// longer row is cut into slices of `seg` entries, each slice's partial sum
+// goes to a scratch slot and the slots of a row are added in a fixed order by
+// a second pass.  `seg` is kSegMax when the block's long rows give enough
+// segments to fill the GPU (rows of ~100 entries in a dense-ish panel), and
+// shrinks to kSegMin otherwise (the few hubs of a power-law graph, each up to
+// a whole block long, are then spread over many warps).
 constexpr int kShort = 32;
-constexpr int kSeg = 128;
+constexpr int kSegMax = 128;
+constexpr int kSegMin = 32;
+constexpr int64_t kSegTarget = 4096;   // segments a block's long rows should give
 
 // Per (side, kind): the panel lists of every block, concatenated.  For block k:
 //   short rows    [row_ptr[k], row_ptr[k+1])   of `host`/`d`   (len <= kShort)
 //   segments      [seg_ptr[k], seg_ptr[k+1])   of `seg`: first the segd[k]
-//                 whole rows of kShort < len <= kSeg, then the kSeg slices
-//                 of the longer rows
+//                 whole rows of kShort < len <= seg, then the slices of `seg`
+//                 entries of the longer rows
 //   split rows    [multi_ptr[k], multi_ptr[k+1]) of `multi`    (row, #segments,
 //                 first slice relative to the block's slices)
 // Rows are listed in ascending order.
