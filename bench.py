@@ -48,7 +48,7 @@ WORKLOADS = {
 # while the kernel's sources hash to the digest recorded with it (else null)
 DENSE_TRAFFIC = {
     # (workload, precision, epilogue): (bytes per launch, dense_source_digest() of the code measured)
-    ("connectome-139255-r64", "bf16", "z"): (18920362, "2343bf0ed2467707"),
+    ("connectome-139255-r64", "bf16", "z"): (18401792, "8dbd5df1c6cc41f5"),
 }
 
 
@@ -261,6 +261,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true", help="skip the oracle timing on the host")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg (profiling runs)")
     ap.add_argument("--no-modes", action="store_true", help="skip the fp32-accurate mode's sweep timing")
+    ap.add_argument("--support-only", action="store_true",
+                    help="only the support term alone over one sweep's steps (profiling; rank 0 only)")
     ap.add_argument("--kernel-table", action="store_true",
                     help="dense kernel alone at the paper's kernel-table shape (m = 250000 rows against a "
                          "block of 2500), one JSON line per factor rank r and precision (rank 0 only)")
@@ -324,6 +326,18 @@ def main():
         W0, H0 = WLm.init_factors(wl.m, wl.n, wl.r, 0, signs="paper")
     sol.set_factors(W0, H0)
     stream = sol.stream
+    if args.support_only:
+        if rank == 0:
+            pk, pk_kind = peaks()
+            hbm = pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
+            ms, nst = measure_support(sol, wl, N)
+            by = support_bytes_per_sweep(wl, 2 if prec == N.NMD_BF16 else 4)
+            print(json.dumps({"metric": "support term alone, algorithmic GB/s", "value": by / (ms / 1e3) / 1e9,
+                              "unit": "GB/s", "frac": by / (ms / 1e3) / 1e9 / hbm, "ms_per_sweep": ms,
+                              "steps": nst, "bytes_per_sweep": by, "workload": wl.name,
+                              "precision": args.precision}))
+        rep.close()
+        return 0
 
     def barrier():
         torch.cuda.synchronize()
