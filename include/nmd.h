@@ -168,6 +168,19 @@ nmd_status nmd_get_factors(nmd_handle* h, float* W, float* H, int on_device);
  * synchronising call and the update is skipped.  Asynchronous. */
 nmd_status nmd_block_update(nmd_handle* h, int32_t side, int64_t block, int32_t kind);
 
+/* One block update with combined row and column sub-sampling (Sec. 4.1, the
+ * remark after eq. lsqA_sto: one update that subsamples both the rows and the
+ * columns of Delta), for problems where even a block row of Z is too large:
+ *   (NMD_ROW, I, J): W_I <- W_I + E, E = eta (X - W_I) + gamma E, with
+ *                    X = argmin ||Z[I, J] - X H_:J|| (the least-squares
+ *                    solution against the column block J on S[I, J]);
+ *   (NMD_COL, I, J): H_:J likewise against W_I on S[I, J]^T.
+ * Blocks as for nmd_block_update (row blocks of block_rows rows, column blocks
+ * of block_cols columns); the momentum rows are those of the updated block.
+ * The block's Gram matrix must be nonsingular (see nmd_block_update).  Not
+ * used by nmd_sweep.  Asynchronous. */
+nmd_status nmd_block_update_combined(nmd_handle* h, int32_t side, int64_t row_block, int64_t col_block);
+
 /* One sweep: block orders are SplitMix64 + Fisher-Yates permutations of the
  * row blocks and column blocks for (seed, sweep index, side).  NMD_EXACT:
  * all row blocks, then all column blocks.  NMD_STOCH + NMD_ALTERNATE: for

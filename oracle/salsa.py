@@ -11,9 +11,10 @@ What it computes (paper notation: L = A B^T, A = W is m x r, B = H^T is n x r):
   L_ij - max(0, L_ij) = min(0, L_ij).
 * Least-squares factor updates, eqs. (lsqA)/(lsqB): A <- Z B (B^T B)^{-1},
   B <- Z^T A (A^T A)^{-1}; restricted to a contiguous row block I (parallel
-  least squares, eqs. Shat_par/Delta_par/lsqA_par, Sec. 4.1) or to a random
+  least squares, eqs. Shat_par/Delta_par/lsqA_par, Sec. 4.1), to a random
   column mini-batch J with step size eta (stochastic least squares,
-  eqs. Shat_sto/Delta_sto/lsqA_sto, Sec. 4.1).
+  eqs. Shat_sto/Delta_sto/lsqA_sto, Sec. 4.1), or to both at once (the
+  combined row and column sub-sampling remarked on after eq. lsqA_sto).
 * Momentum: "a multiple of the previously executed update" (Sec. 4.1, after
   eq. lsqA_sto), read as heavy ball E_t = U_t + gamma E_{t-1}, M += E_t.
 * Losses: objective ||Z - L||_F / ||S||_F (eq. auxCost, evaluated through
@@ -271,6 +272,20 @@ class State:
             return self.B, self.EB, (j0, j1), self.A, self.St, (0, self.m)
         return self.A, self.EA, (0, self.m), self.B[j0:j1], self.S, (j0, j1)
 
+    def _roles_combined(self, side: int, row_block: int, col_block: int):
+        """Combined row and column sub-sampling (Sec. 4.1, the remark after eq.
+        lsqA_sto: one update that subsamples rows and columns of Delta):
+
+        ROW: A_I from B_J on S[I, J]      (eq. lsqA_sto restricted to the rows I)
+        COL: B_J from A_I on S[I, J]^T    (the same for B)
+        """
+        o = self.opts
+        i0, i1 = block_range(row_block, o.block_rows, self.m)
+        j0, j1 = block_range(col_block, o.block_cols, self.n)
+        if side == ROW:
+            return self.A, self.EA, (i0, i1), self.B[j0:j1], self.S, (j0, j1)
+        return self.B, self.EB, (j0, j1), self.A[i0:i1], self.St, (i0, i1)
+
     def block_terms(self, side: int, block: int, kind: int, chunk_elems: int = 1 << 24,
                     rows=None):
         """R = Z Q for the M-side rows and G = Q^T Q.
@@ -278,7 +293,14 @@ class State:
         With ``rows`` (indices relative to the first M-side row) only those
         rows of R are formed -- each row of R depends on its own row of Z only.
         """
-        M, _, (m0, m1), Q, src, (c0, c1) = self._roles(side, block, kind)
+        return self._terms(self._roles(side, block, kind), chunk_elems, rows)
+
+    def block_terms_combined(self, side: int, row_block: int, col_block: int):
+        """R = Z Q and G = Q^T Q of a combined row and column step."""
+        return self._terms(self._roles_combined(side, row_block, col_block))
+
+    def _terms(self, roles, chunk_elems: int = 1 << 24, rows=None):
+        M, _, (m0, m1), Q, src, (c0, c1) = roles
         K = c1 - c0
         G = Q.T @ Q
         if rows is not None:
@@ -310,15 +332,23 @@ class State:
         return rows[keep] - m0, cols[keep] - c0
 
     def block_update(self, side: int, block: int, kind: int):
+        self._update(self._roles(side, block, kind), momentum=kind == STOCH)
+
+    def block_update_combined(self, side: int, row_block: int, col_block: int):
+        """A stochastic step (step size eta, momentum) on the rows of one block
+        of the updated factor against one block of the other, on S[I, J]."""
+        self._update(self._roles_combined(side, row_block, col_block), momentum=True)
+
+    def _update(self, roles, momentum: bool):
         o = self.opts
-        M, E, (m0, m1), Q, _, _ = self._roles(side, block, kind)
-        R, G = self.block_terms(side, block, kind)
+        M, E, (m0, m1), Q, _, _ = roles
+        R, G = self._terms(roles)
         if o.ridge:
             G = G + o.ridge * np.eye(self.r)
         C = cholesky(G)
         M_ls = solve_normal(C, R)
         U = o.eta * (M_ls - M[m0:m1])
-        if kind == STOCH:
+        if momentum:
             E[m0:m1] = U + o.gamma * E[m0:m1]
             M[m0:m1] += E[m0:m1]
         else:

@@ -462,7 +462,67 @@ struct Roles {
   const PanelSet* P;
   const int32_t* qidx;   // absolute Q-side index of each sparse entry
   const float* vals;
+  int64_t pblock = 0;    // the block of P whose panel the step uses
+  bool sub = false;      // the step takes only the panel's M-side rows [m0, m0 + M)
 };
+
+// The sparse work of one step: the sub-lists of a block's panel lists whose
+// M-side rows lie in the step's range (all of them, unless Roles::sub).
+struct Span {
+  const PanelRow *rows, *whole, *seg, *multi;   // device pointers
+  int64_t nrows, nwhole, nseg, nmulti;
+  int64_t seg_first;                            // first slice, relative to the block's slices
+  const uint8_t* flags;                         // one byte per M-side row of the step
+  // host-side index ranges (for nmd_panel_traversal)
+  int64_t hr0, hr1, hw0, hw1, hu0, hu1;
+};
+
+Span panel_span(const Roles& ro) {
+  const PanelSet& P = *ro.P;
+  const int64_t b = ro.pblock;
+  const int64_t r0 = P.row_ptr[b], r1 = P.row_ptr[b + 1];
+  const int64_t g0 = P.seg_ptr[b], gd = g0 + P.segd[b], g1 = P.seg_ptr[b + 1];
+  const int64_t u0 = P.multi_ptr[b], u1 = P.multi_ptr[b + 1];
+  Span sp;
+  sp.hr0 = r0; sp.hr1 = r1; sp.hw0 = g0; sp.hw1 = gd; sp.hu0 = u0; sp.hu1 = u1;
+  sp.seg_first = 0;
+  int64_t s0 = 0, s1 = g1 - gd;
+  if (ro.sub) {   // lists are ascending by row: cut them to [m0, m0 + M)
+    auto lo = [](const std::vector<PanelRow>& v, int64_t a, int64_t z, int64_t row) {
+      return (int64_t)(std::lower_bound(v.begin() + a, v.begin() + z, row,
+                                        [](const PanelRow& p, int64_t x) { return p.row < x; }) - v.begin());
+    };
+    const int64_t m1 = ro.m0 + ro.M;
+    sp.hr0 = lo(P.host, r0, r1, ro.m0); sp.hr1 = lo(P.host, r0, r1, m1);
+    sp.hw0 = lo(P.seg, g0, gd, ro.m0); sp.hw1 = lo(P.seg, g0, gd, m1);
+    sp.hu0 = lo(P.multi, u0, u1, ro.m0); sp.hu1 = lo(P.multi, u0, u1, m1);
+    if (sp.hu1 > sp.hu0) {
+      s0 = P.multi[sp.hu0].beg;
+      s1 = P.multi[sp.hu1 - 1].beg + P.multi[sp.hu1 - 1].len;
+    } else {
+      s0 = s1 = 0;
+    }
+  }
+  sp.rows = P.d + sp.hr0;
+  sp.nrows = sp.hr1 - sp.hr0;
+  sp.whole = P.d_seg + sp.hw0;
+  sp.nwhole = sp.hw1 - sp.hw0;
+  sp.seg = P.d_seg + gd + s0;
+  sp.nseg = s1 - s0;
+  sp.seg_first = s0;
+  sp.multi = P.d_multi + sp.hu0;
+  sp.nmulti = sp.hu1 - sp.hu0;
+  // stochastic panels flag every row of the M side, exact ones the block's rows
+  sp.flags = P.d_flags + P.flag_off[b] + (ro.sub ? ro.m0 : 0);
+  return sp;
+}
+
+nmd_status launch_span(nmd_handle* h, const StepArgs& a, const Roles& ro, const Span& sp, float* Rs, cudaStream_t s) {
+  launch_sparse(a, sp.rows, sp.nrows, sp.whole, sp.nwhole, sp.seg, sp.nseg, sp.multi, sp.nmulti, ro.qidx, ro.vals,
+                Rs, h->ws.seg_partials, sp.seg_first, s);
+  h->launches += (sp.nrows > 0) + (sp.nwhole > 0) + 2 * (sp.nseg > 0);
+  return NMD_OK;
+}
 
 nmd_status roles(nmd_handle* h, int side, int64_t block, int kind, Roles* R) {
   if (side != NMD_ROW && side != NMD_COL) return fail(h, NMD_ERR_INVALID, "side must be NMD_ROW or NMD_COL");
@@ -477,14 +537,38 @@ nmd_status roles(nmd_handle* h, int side, int64_t block, int kind, Roles* R) {
   int64_t i0 = block * b, i1 = std::min(N, (block + 1) * b);
   const PanelSet* P = &h->panels[side][kind];
   if (side == NMD_ROW && kind == NMD_EXACT) {        // W_I from all of B on S[I, :]
-    *R = Roles{&h->W, &h->B, i0, i1 - i0, 0, h->n, P, h->ws.col, h->ws.val};
+    *R = Roles{&h->W, &h->B, i0, i1 - i0, 0, h->n, P, h->ws.col, h->ws.val, block};
   } else if (side == NMD_COL && kind == NMD_EXACT) { // B_J from all of W on S[:, J]^T
-    *R = Roles{&h->B, &h->W, i0, i1 - i0, 0, h->m, P, h->ws.row, h->ws.valT};
+    *R = Roles{&h->B, &h->W, i0, i1 - i0, 0, h->m, P, h->ws.row, h->ws.valT, block};
   } else if (side == NMD_COL) {                      // all of W from B_J on S[:, J]
-    *R = Roles{&h->W, &h->B, 0, h->m, i0, i1 - i0, P, h->ws.col, h->ws.val};
+    *R = Roles{&h->W, &h->B, 0, h->m, i0, i1 - i0, P, h->ws.col, h->ws.val, block};
   } else {                                           // all of B from W_I on S[I, :]^T
-    *R = Roles{&h->B, &h->W, 0, h->n, i0, i1 - i0, P, h->ws.row, h->ws.valT};
+    *R = Roles{&h->B, &h->W, 0, h->n, i0, i1 - i0, P, h->ws.row, h->ws.valT, block};
   }
+  return NMD_OK;
+}
+
+// Combined row and column sub-sampling (Sec. 4.1, the remark after eq.
+// lsqA_sto): NMD_ROW updates W_I from B_J on S[I, J] (the column panel of J
+// cut to the rows I), NMD_COL updates B_J from W_I on S[I, J]^T (the row panel
+// of I cut to the columns J).
+nmd_status roles_combined(nmd_handle* h, int side, int64_t row_block, int64_t col_block, Roles* R) {
+  if (side != NMD_ROW && side != NMD_COL) return fail(h, NMD_ERR_INVALID, "side must be NMD_ROW or NMD_COL");
+  const int64_t Kr = nblocks(h->m, h->opt.block_rows), Kc = nblocks(h->n, h->opt.block_cols);
+  if (row_block < 0 || row_block >= Kr || col_block < 0 || col_block >= Kc) {
+    char b[160];
+    snprintf(b, sizeof b, "blocks (%lld, %lld) out of range [0, %lld) x [0, %lld)", (long long)row_block,
+             (long long)col_block, (long long)Kr, (long long)Kc);
+    return fail(h, NMD_ERR_INVALID, b);
+  }
+  const int64_t i0 = row_block * h->opt.block_rows, i1 = std::min(h->m, (row_block + 1) * h->opt.block_rows);
+  const int64_t j0 = col_block * h->opt.block_cols, j1 = std::min(h->n, (col_block + 1) * h->opt.block_cols);
+  if (side == NMD_ROW)
+    *R = Roles{&h->W, &h->B, i0, i1 - i0, j0, j1 - j0, &h->panels[NMD_COL][NMD_STOCH], h->ws.col, h->ws.val,
+               col_block, true};
+  else
+    *R = Roles{&h->B, &h->W, j0, j1 - j0, i0, i1 - i0, &h->panels[NMD_ROW][NMD_STOCH], h->ws.row, h->ws.valT,
+               row_block, true};
   return NMD_OK;
 }
 
@@ -530,11 +614,22 @@ nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro,
   return NMD_OK;
 }
 
+// step kinds beyond nmd_kind: a stochastic step on a (row block, column
+// block) pair (combined sub-sampling)
+constexpr int kCombined = 2;
+
+nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_update, const NextUse* next);
+
 nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_update,
                     const NextUse* next = nullptr) {
   Roles ro;
   nmd_status st = roles(h, side, block, kind, &ro);
   if (st != NMD_OK) return st;
+  return run_step_roles(h, ro, kind, do_update, next);
+}
+
+nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_update, const NextUse* next) {
+  nmd_status st = NMD_OK;
   StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
               h->opt.skip_zero_chunks != 0};
   cudaStream_t s = h->cur;
@@ -599,17 +694,12 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   }
   if ((st = after_launch(h, "gram/cholesky")) != NMD_OK) return st;
   // sparse correction over the block's support
-  const PanelSet& P = *ro.P;
-  int64_t r0 = P.row_ptr[block], r1 = P.row_ptr[block + 1];
-  int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1], gd = g0 + P.segd[block];
-  int64_t u0 = P.multi_ptr[block], u1 = P.multi_ptr[block + 1];
-  const uint8_t* flags = P.d_flags + P.flag_off[block];
+  const Span sp = panel_span(ro);
+  const uint8_t* flags = sp.flags;
   h->cur_flags = flags;
   {
     TimedScope ts(h, NMD_K_SPARSE, h->side2);
-    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, gd - g0, P.d_seg + gd, g1 - gd, P.d_multi + u0, u1 - u0,
-                  ro.qidx, ro.vals, Rs, h->ws.seg_partials, h->side2);
-    h->launches += (r1 > r0) + (gd > g0) + 2 * (g1 > gd);
+    launch_span(h, a, ro, sp, Rs, h->side2);
   }
   if ((st = after_launch(h, "sparse correction")) != NMD_OK) return st;
   CK(h, cudaEventRecord(h->ev_join, h->side));
@@ -630,7 +720,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
   CK(h, cudaStreamWaitEvent(s, h->ev_join, 0));
   CK(h, cudaStreamWaitEvent(s, h->ev_join2, 0));
   if (do_update) {
-    const bool momentum = kind == NMD_STOCH;
+    const bool momentum = kind != NMD_EXACT;
     // rows [lo, hi) (relative to m0) are updated on the main stream; when the
     // next step reads only these rows of this factor and writes the other
     // factor, the rest are updated on the aux stream, overlapping it
@@ -938,6 +1028,15 @@ nmd_status nmd_block_update(nmd_handle* h, int32_t side, int64_t block, int32_t 
   return run_step(h, side, block, kind, true);
 }
 
+nmd_status nmd_block_update_combined(nmd_handle* h, int32_t side, int64_t row_block, int64_t col_block) {
+  if (!h) return NMD_ERR_INVALID;
+  DeviceScope dg(h);
+  Roles ro;
+  nmd_status st = roles_combined(h, side, row_block, col_block, &ro);
+  if (st != NMD_OK) return st;
+  return run_step_roles(h, ro, kCombined, true, nullptr);
+}
+
 nmd_status nmd_block_order(const nmd_handle* h, int64_t sweep, int32_t side, int64_t* perm, int64_t K) {
   if (!h || !perm || (side != NMD_ROW && side != NMD_COL) || sweep < 0) return NMD_ERR_INVALID;
   int64_t Kexp = side == NMD_ROW ? nblocks(h->m, h->opt.block_rows) : nblocks(h->n, h->opt.block_cols);
@@ -1099,17 +1198,11 @@ nmd_status nmd_support_term(nmd_handle* h, int32_t side, int64_t block, int32_t 
   if ((st = wait_all_pending(h)) != NMD_OK) return st;
   StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
               h->opt.skip_zero_chunks != 0};
-  const PanelSet& P = *ro.P;
-  const int64_t r0 = P.row_ptr[block], r1 = P.row_ptr[block + 1];
-  const int64_t g0 = P.seg_ptr[block], g1 = P.seg_ptr[block + 1], gd = g0 + P.segd[block];
-  const int64_t u0 = P.multi_ptr[block], u1 = P.multi_ptr[block + 1];
   cudaStream_t s = h->stream;
   CK(h, cudaMemsetAsync(d_R, 0, (size_t)ro.M * h->rp * sizeof(float), s));
   {
     TimedScope ts(h, NMD_K_SPARSE, s);
-    launch_sparse(a, P.d + r0, r1 - r0, P.d_seg + g0, gd - g0, P.d_seg + gd, g1 - gd, P.d_multi + u0, u1 - u0,
-                  ro.qidx, ro.vals, d_R, h->ws.seg_partials, s);
-    h->launches += (r1 > r0) + (gd > g0) + 2 * (g1 > gd);
+    launch_span(h, a, ro, panel_span(ro), d_R, s);
   }
   if ((st = after_launch(h, "support term")) != NMD_OK) return st;
   if (rows) *rows = ro.M;

@@ -1254,7 +1254,10 @@ static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* pa
 
 void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole, int64_t nwhole,
                    const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
-                   const float* vals, float* R, float* partials, cudaStream_t s) {
+                   const float* vals, float* R, float* partials, int64_t seg_first, cudaStream_t s) {
+  // slice w of `seg` is slice seg_first + w of its block, whose partial slot
+  // the reduction (multi[].beg, relative to the block) reads
+  float* seg_partials = partials + seg_first * a.rp;
   // The support term reads the same factor values as the rest of the step's
   // least-squares problem: the bf16 pieces in the bf16 mode (whose dense term
   // and Gram matrix are formed from them), the fp32 masters otherwise.
@@ -1270,7 +1273,7 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
           whole, nwhole, MOP, a.m0, QOP, qidx, vals, R, nullptr, a.rp);                                      \
     if (nseg > 0) {                                                                                          \
       sparse_long_kernel<LPE, CPL, TT><<<(unsigned)((nseg + 7) / 8), 256, 0, s>>>(                            \
-          seg, nseg, MOP, a.m0, QOP, qidx, vals, R, partials, a.rp);                                         \
+          seg, nseg, MOP, a.m0, QOP, qidx, vals, R, seg_partials, a.rp);                                     \
       launch_reduce(multi, nmulti, partials, R, a.m0, a.rp, s);                                              \
     }                                                                                                        \
   } while (0)

@@ -238,7 +238,8 @@ void launch_small_gemm(const float* A, int64_t lda, const float* B, int64_t ldb,
 // (bf16 mode: the factors' hi pieces, else the fp32 masters)
 void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole,
                    int64_t nwhole, const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti,
-                   const int32_t* qidx, const float* vals, float* R, float* partials, cudaStream_t s);
+                   const int32_t* qidx, const float* vals, float* R, float* partials, int64_t seg_first,
+                   cudaStream_t s);
 // flags: one byte per row of the step (Rs is read only where it is nonzero)
 // gpart, when not nullptr and r_pad <= 64: also write the Gram partials of the
 // new rows, one per 64-row tile (gram_round: of their bf16 rounding), exactly

@@ -31,7 +31,7 @@ EXPORTS = [
     "nmd_get_factors", "nmd_block_update", "nmd_sweep", "nmd_block_order", "nmd_loss", "nmd_sync",
     "nmd_block_terms", "nmd_dense_products", "nmd_panel_traversal", "nmd_get_state", "nmd_set_state",
     "nmd_launch_count", "nmd_skip_count", "nmd_selftest_wait_timeout", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
-    "nmd_destroy", "nmd_gram_noalloc", "nmd_support_term",
+    "nmd_destroy", "nmd_gram_noalloc", "nmd_support_term", "nmd_block_update_combined",
 ]
 
 
@@ -96,6 +96,7 @@ def lib() -> C.CDLL:
             "nmd_destroy": (None, [_P]),
             "nmd_gram_noalloc": (C.c_int, [_P, C.c_int64, C.c_int32, C.c_int64, _P, _P]),
             "nmd_support_term": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int32, _P, _i64p]),
+            "nmd_block_update_combined": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int64]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -221,6 +222,10 @@ def nmd_panel_traversal(h, side, block, kind):
     return rows, q
 
 
+def nmd_block_update_combined(h, side, row_block, col_block):
+    _check(h, lib().nmd_block_update_combined(h, side, row_block, col_block), "nmd_block_update_combined")
+
+
 def nmd_support_term(h, side, block, kind, d_R) -> int:
     rows = C.c_int64(0)
     _check(h, lib().nmd_support_term(h, side, block, kind, _ptr(d_R), C.byref(rows)), "nmd_support_term")
@@ -335,6 +340,11 @@ class Solver:
 
     def block_update(self, side, block, kind):
         nmd_block_update(self.h, side, block, kind)
+
+    def block_update_combined(self, side, row_block, col_block):
+        """Combined row and column sub-sampling: W_I from H_:J (NMD_ROW) or
+        H_:J from W_I (NMD_COL), on S[I, J]."""
+        nmd_block_update_combined(self.h, side, row_block, col_block)
 
     def sweep(self):
         nmd_sweep(self.h)

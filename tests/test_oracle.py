@@ -237,6 +237,62 @@ def test_block_update_matches_dense_bruteforce(side, kind):
         np.testing.assert_allclose(st.EB, EB, rtol=1e-10, atol=1e-11)
 
 
+@pytest.mark.parametrize("side", [O.ROW, O.COL])
+def test_combined_update_matches_dense_bruteforce(side):
+    """Combined row and column sub-sampling (Sec. 4.1, after eq. lsqA_sto):
+    side ROW takes A_I to argmin_X ||Z[I, J] - X B_J^T|| with step eta and
+    momentum; side COL the same for B_J against A_I on S[I, J]^T."""
+    S, D = _rand_sparse(13, 11, 0.35, 6)
+    rng = np.random.default_rng(7)
+    r = 3
+    W = rng.standard_normal((13, r))
+    H = rng.standard_normal((r, 11))
+    opts = O.Options(block_rows=5, block_cols=4, eta=0.7, gamma=0.5)
+    st = O.State(S, W, H, opts)
+    st.EA[:] = 0.01 * rng.standard_normal(st.EA.shape)
+    st.EB[:] = 0.01 * rng.standard_normal(st.EB.shape)
+    for I in range(O.num_blocks(13, 5)):                   # ragged last blocks included
+        for J in range(O.num_blocks(11, 4)):
+            i0, i1 = O.block_range(I, 5, 13)
+            j0, j1 = O.block_range(J, 4, 11)
+            A, B, EA, EB = st.A.copy(), st.B.copy(), st.EA.copy(), st.EB.copy()
+            if side == O.ROW:
+                Z = O.update_z(D[i0:i1, j0:j1], A[i0:i1] @ B[j0:j1].T)
+                X = np.linalg.lstsq(B[j0:j1], Z.T, rcond=None)[0].T
+                EA[i0:i1] = opts.eta * (X - A[i0:i1]) + opts.gamma * EA[i0:i1]
+                A[i0:i1] += EA[i0:i1]
+            else:
+                Z = O.update_z(D[i0:i1, j0:j1].T, B[j0:j1] @ A[i0:i1].T)
+                X = np.linalg.lstsq(A[i0:i1], Z.T, rcond=None)[0].T
+                EB[j0:j1] = opts.eta * (X - B[j0:j1]) + opts.gamma * EB[j0:j1]
+                B[j0:j1] += EB[j0:j1]
+            st.block_update_combined(side, I, J)
+            np.testing.assert_allclose(st.A, A, rtol=1e-10, atol=1e-11)
+            np.testing.assert_allclose(st.B, B, rtol=1e-10, atol=1e-11)
+            np.testing.assert_allclose(st.EA, EA, rtol=1e-10, atol=1e-11)
+            np.testing.assert_allclose(st.EB, EB, rtol=1e-10, atol=1e-11)
+
+
+def test_combined_update_reduces_to_the_other_steps():
+    """A combined step whose row block is every row is the stochastic column
+    step (eq. lsqA_sto); one whose column block is every column, with eta = 1
+    and no momentum, is the parallel row step (eq. lsqA_par)."""
+    S, _ = _rand_sparse(20, 15, 0.25, 8)
+    W, H = WL.init_factors(20, 15, 3, 1)
+    for eta, gamma in ((0.8, 0.6), (1.0, 0.0)):
+        a = O.State(S, W, H, O.Options(block_rows=20, block_cols=6, eta=eta, gamma=gamma))
+        b = O.State(S, W, H, O.Options(block_rows=20, block_cols=6, eta=eta, gamma=gamma))
+        a.block_update_combined(O.ROW, 0, 1)
+        b.block_update(O.COL, 1, O.STOCH)
+        np.testing.assert_allclose(a.A, b.A, rtol=1e-12, atol=1e-13)
+        np.testing.assert_allclose(a.EA, b.EA, rtol=1e-12, atol=1e-13)
+    a = O.State(S, W, H, O.Options(block_rows=7, block_cols=15, eta=1.0, gamma=0.0))
+    b = O.State(S, W, H, O.Options(block_rows=7, block_cols=15, eta=1.0, gamma=0.0))
+    a.block_update_combined(O.ROW, 2, 0)
+    b.block_update(O.ROW, 2, O.EXACT)
+    np.testing.assert_allclose(a.A, b.A, rtol=1e-12, atol=1e-13)
+
+
 def test_stochastic_full_batch_equals_parallel():
     """A mini-batch covering every column with eta=1, gamma=0 is plain ALS (eq. lsqA)."""
     S, _ = _rand_sparse(20, 15, 0.25, 5)

@@ -146,3 +146,29 @@ def test_connectome_loss_full_width_sample(wl64, prec):
     assert abs(got["rmse"] - np.sqrt(want["err2"]) / s_sub) <= tol * np.sqrt(want["err2"]) / s_sub
     wjd = 1.0 - want["sum_min"] / want["sum_max"]
     assert abs(got["wjd"] - wjd) <= tol * wjd
+
+
+@pytest.mark.parametrize("prec", [N.NMD_BF16, N.NMD_FP32], ids=["bf16", "fp32"])
+def test_connectome_combined_full_size(wl64, prec):
+    """Combined row and column sub-sampling on the full connectome: W_I from
+    H_:J and H_:J from W_I for the ragged last blocks and a middle pair
+    (4,096 x 4,096 panels holding the hub rows)."""
+    sol, orc = make_pair(wl64.S, wl64.r, wl64.W0, wl64.H0, block_rows=wl64.block_rows,
+                         block_cols=wl64.block_cols, precision=prec, eta=wl64.eta, gamma=wl64.gamma)
+    K = -(-wl64.n // wl64.block_cols)
+    try:
+        for side, I, J in [(N.NMD_ROW, K - 1, 17), (N.NMD_COL, 5, K - 1), (N.NMD_ROW, 11, 11)]:
+            sync_oracle_to(sol, orc)
+            sol.block_update_combined(side, I, J)
+            orc.block_update_combined(side, I, J)
+            W, H, EW, EH, _ = sol.get_state()
+            if side == N.NMD_ROW:
+                a, b = I * wl64.block_rows, min(wl64.m, (I + 1) * wl64.block_rows)
+                got, want = W[a:b], orc.A[a:b]
+            else:
+                a, b = J * wl64.block_cols, min(wl64.n, (J + 1) * wl64.block_cols)
+                got, want = H.T[a:b], orc.B[a:b]
+            assert rel(got, want) <= TOL[prec], (side, I, J, rel(got, want))
+    finally:
+        del sol
+        gc.collect()
