@@ -423,7 +423,7 @@ def main():
     sp_ms, sp_steps = measure_support(sol, wl, N)
     sp_bytes = support_bytes_per_sweep(wl, 2 if prec == N.NMD_BF16 else 4)
     sp_gbs = sp_bytes / (sp_ms / 1e3) / 1e9
-    roofline_sparse = {"bound": "hbm", "kernel": "support term (sparse_rows_kernel, sparse_long_kernel, "
+    roofline_sparse = {"bound": "hbm", "kernel": "support term (sparse_group_kernel, sparse_long_kernel, "
                                                  "sparse_reduce_kernel), alone",
                        "achieved": sp_gbs, "peak": hbm, "unit": "GB/s", "frac": sp_gbs / hbm,
                        "traffic": None, "peak_kind": "%s copy bandwidth" % pk_kind,

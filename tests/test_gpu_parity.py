@@ -250,11 +250,14 @@ def test_ring_point_is_fixed(prec):
     assert rel(W @ H, W0.astype(np.float64) @ H0) < 1e-3
 
 
-def test_not_spd_is_reported_and_update_skipped():
-    # 400 columns in blocks of 133: the last block has 1 column < r = 4
-    S, _, _, _ = WL.planted(300, 400, 4, tau=0.5, seed=0)
-    W, H = WL.init_factors(300, 400, 4, 0)
-    sol = N.Solver(S, 4, block_rows=100, block_cols=133, precision=N.NMD_SIMT)
+@pytest.mark.parametrize("r, prec", [(4, N.NMD_SIMT), (200, N.NMD_BF16), (200, N.NMD_FP32)])
+def test_not_spd_is_reported_and_update_skipped(r, prec):
+    # 700 columns in blocks of 233: the last block has 1 column < r, so its
+    # Gram matrix has rank 1 (r = 4: the register-resident factorisation;
+    # r = 200, r_pad = 256: the shared-memory one)
+    S, _, _, _ = WL.planted(300, 700, 4, tau=0.5, seed=0)
+    W, H = WL.init_factors(300, 700, r, 0)
+    sol = N.Solver(S, r, block_rows=100, block_cols=233, precision=prec)
     sol.set_factors(W, H)
     sol.block_update(N.NMD_COL, 3, N.NMD_STOCH)
     with pytest.raises(N.NmdError) as e:
