@@ -207,134 +207,14 @@ __global__ void __launch_bounds__(256) small_gemm_kernel(const float* __restrict
 // G^{-1} through the Cholesky factorisation of G (the normal equations of
 // eqs. lsqA/lsqB, Sec. 3.2), in its square-root-free form G = L D L^T (L unit
 // lower triangular, D diagonal; the Cholesky factor is L D^{1/2}), then
-// Y = L^{-1} and G^{-1} = Y^T D^{-1} Y.  One thread block of T x T threads.
-// The lower triangle lives in
-// shared memory in packed row-major form (row i starts at i (i + 1) / 2);
-// thread (ty, tx) takes rows ty, ty + T, ... and within a row the columns
-// tx, tx + T, ..., so the lanes of a warp touch consecutive entries of a row.
-//  1. Right-looking factorisation, one column per step and one barrier per
-//     step: the pivot d_k = a_kk is the Schur complement (the square of the
-//     Cholesky pivot); d_k <= 4 r eps g_kk or a non-finite d_k marks G as not
-//     positive definite (NMD_ERR_NOT_SPD, detail k) and leaves G^{-1} = 0.
-//     Otherwise a_ij -= a_ik a_jk / d_k for k < j <= i; column k keeps
-//     a_ik = l_ik d_k.  Column k is read from a copy that the previous step
-//     wrote (two copies alternate), so no step reads what it writes.
-//  2. Y = L^{-1} (unit lower; its diagonal is implicit), column step k: row k
-//     of Y is final, and every row i > k subtracts l_ik Y[k, 0..k].  With
-//     room for a second triangle (r_pad <= 128, SEPY) Y has its own;
-//     otherwise (r_pad = 256) Y takes the place of L, and each warp reads
-//     l_ik before any of its lanes writes Y[i, k] over it (a warp is one row
-//     group there).  One barrier per step.
-//  3. G^{-1}[a][b] = sum over k >= max(a, b) of Y[k][a] Y[k][b] / d_k, each
-//     thread a 4 x 4 block of the lower triangle, written to both triangles
-//     so that the result is exactly symmetric.
+// Y = L^{-1} and G^{-1} = Y^T D^{-1} Y, written to both triangles so that
+// the result is exactly symmetric.  A pivot d_k <= 4 r eps g_kk (d_k is the
+// Schur complement, the square of the Cholesky pivot) or a non-finite d_k
+// marks G as not positive definite: NMD_ERR_NOT_SPD with detail k, and
+// G^{-1} = 0.  One thread block; two forms below, by r_pad.
 // ---------------------------------------------------------------------------
-__host__ __device__ __forceinline__ int tri(int i) { return (i * (i + 1)) >> 1; }
 
-inline size_t chol_smem_bytes(int r, int rp, bool sepy) {
-  return ((size_t)(sepy ? 2 : 1) * (size_t)((tri(r) + 3) & ~3) + 4 * (size_t)rp) * sizeof(float);
-}
-
-template <int T, bool SEPY>
-__global__ void __launch_bounds__(T * T) chol_inv_kernel(const float* __restrict__ G, int r, int rp,
-                                                         float* __restrict__ Ginv, int* __restrict__ status) {
-  static_assert(SEPY || T == 32, "in-place inverse needs one warp per row group");
-  extern __shared__ __align__(16) float sm[];
-  const int ntri = (tri(r) + 3) & ~3;
-  float* A = sm;                                   // the factor
-  float* Y = SEPY ? sm + ntri : sm;                // L^{-1}
-  float* colk = sm + (SEPY ? 2 : 1) * ntri;        // 2 x rp: column k of the factor, alternating
-  float* invd = colk + 2 * rp;                     // rp: 1 / d_k
-  float* diag0 = invd + rp;                        // rp: the diagonal of G
-  constexpr int NT = T * T;
-  const int tx = threadIdx.x % T, ty = threadIdx.x / T;
-  for (int i = ty; i < r; i += T)
-    for (int j = tx; j <= i; j += T) {
-      const float g = G[(size_t)i * rp + j];
-      A[tri(i) + j] = g;
-      if (j == 0) colk[i] = g;
-      if (i == j) diag0[i] = g;
-    }
-  for (int e = threadIdx.x; e < rp * rp; e += NT)
-    if (e / rp >= r || e % rp >= r) Ginv[e] = 0.f;
-  __syncthreads();
-  // 1. G = L D L^T
-  const float tol = 4.0f * (float)r * FLT_EPSILON;
-  for (int k = 0; k < r; ++k) {
-    const float* ck = colk + (k & 1) * rp;
-    float* cn = colk + ((k + 1) & 1) * rp;
-    const float d = ck[k];
-    if (!(d > tol * diag0[k]) || !isfinite(d)) {   // uniform: every thread read the same d
-      if (threadIdx.x == 0) set_status(status, NMD_ERR_NOT_SPD, k, 0);
-      for (int e = threadIdx.x; e < rp * rp; e += NT) Ginv[e] = 0.f;
-      return;
-    }
-    const float inv = 1.0f / d;
-    if (threadIdx.x == 0) invd[k] = inv;
-    for (int i = k + 1 + ty; i < r; i += T) {
-      const float ci = ck[i];
-      float* row = A + tri(i);
-      for (int j = k + 1 + tx; j <= i; j += T) {
-        const float v = fmaf(-(ci * ck[j]), inv, row[j]);
-        row[j] = v;
-        if (j == k + 1) cn[i] = v;                  // column k + 1 for the next step
-      }
-    }
-    __syncthreads();
-  }
-  // 2. Y = L^{-1}, l_ik = a_ik / d_k
-  for (int k = 0; k + 1 < r; ++k) {
-    const float* yk = Y + tri(k);
-    const float ik = invd[k];
-    for (int i = k + 1 + ty; i < r; i += T) {
-      const float lik = A[tri(i) + k] * ik;
-      if (!SEPY) __syncwarp();                     // every lane has l_ik before Y[i, k] replaces it
-      float* row = Y + tri(i);
-      for (int j = tx; j <= k; j += T) row[j] = j == k ? -lik : fmaf(-lik, yk[j], row[j]);
-    }
-    __syncthreads();
-  }
-  // 3. G^{-1} = Y^T D^{-1} Y
-  const int n4 = (r + 3) / 4;
-  for (int t = threadIdx.x; t < tri(n4); t += NT) {
-    int ta = (int)((sqrtf(8.f * (float)t + 1.f) - 1.f) * 0.5f);
-    while (tri(ta + 1) <= t) ++ta;
-    while (tri(ta) > t) --ta;
-    const int tb = t - tri(ta);
-    const int a0 = 4 * ta, b0 = 4 * tb;
-    float acc[4][4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-#pragma unroll
-      for (int v = 0; v < 4; ++v) acc[u][v] = 0.f;
-    for (int k = a0; k < r; ++k) {
-      const float* yk = Y + tri(k);
-      const float w = invd[k];
-      float ya[4], yb[4];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        ya[u] = w * (a0 + u < k ? yk[a0 + u] : (a0 + u == k ? 1.f : 0.f));
-        yb[u] = b0 + u < k ? yk[b0 + u] : (b0 + u == k ? 1.f : 0.f);
-      }
-#pragma unroll
-      for (int u = 0; u < 4; ++u)
-#pragma unroll
-        for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(ya[u], yb[v], acc[u][v]);
-    }
-#pragma unroll
-    for (int u = 0; u < 4; ++u)
-#pragma unroll
-      for (int v = 0; v < 4; ++v) {
-        const int a = a0 + u, b = b0 + v;
-        if (a < r && b <= a) {
-          Ginv[(size_t)a * rp + b] = acc[u][v];
-          Ginv[(size_t)b * rp + a] = acc[u][v];
-        }
-      }
-  }
-}
-
-// Register-resident, blocked form of the same factorisation for r_pad <= 128
+// Register-resident, blocked form for r_pad <= 32
 // (the pad rows and columns >= r get a unit diagonal, so the padded matrix
 // diag(G, I) is factored and inverted; its pad part is dropped at the end).
 // Thread t owns row i = t / 4 and the CPT = r_pad / 4 contiguous columns
@@ -528,6 +408,263 @@ __global__ void __launch_bounds__(RP * 4) ldlt_inv_reg_kernel(const float* __res
 inline size_t ldlt_reg_smem_bytes(int rp) {
   const size_t pb = rp / 4 < 8 ? rp / 4 : 8;
   return ((size_t)2 * rp + 64 + 2 * pb * rp + (size_t)rp * (rp + 1)) * sizeof(float);
+}
+
+// Tile-blocked form of the same factorisation for r_pad in {64, 128, 256}:
+// the matrix is cut into 32 x 32 tiles and only the lower triangle of tiles
+// is kept in shared memory (row stride 33, so a tile's rows and columns are
+// both read without bank conflicts); pad rows and columns >= r get a unit
+// diagonal, as in the register form.  For each tile column J:
+//  1a. one warp factors the diagonal tile in registers (lane i holds row i;
+//      every entry read by a shuffle), checks the pivots, and replaces the
+//      tile by the inverse Yt of its unit lower factor (forward substitution
+//      with shuffles), stored with its unit diagonal and zeros above;
+//  1b. the tiles below: L_IJ = A_IJ Yt^T D_J^{-1}, one warp per row, lanes
+//      over the 32 columns; the panel is also stored transposed in P;
+//  1c. the trailing tiles: A_IK -= L_IJ D_J L_KJ^T, 4 x 4 outputs per thread
+//      with float4 reads of the transposed panel.
+// Three barriers per tile column (24 at r_pad = 256).  Then
+//  2.  Y = L^{-1} by tile rows I: T_IJ = sum over K in [J, I) of L_IK Y_KJ
+//      (Y_JJ is the diagonal tile's inverse), then Y_IJ = -Yt_I T_IJ over
+//      L_IJ; two barriers per tile row;
+//  3.  G^{-1} = Y^T D^{-1} Y from the tiles, 4 x 4 outputs per thread,
+//      written to both triangles (exactly symmetric).
+// The trailing update and the products in 2 and 3 are the r^3 part, spread
+// over every thread; the serial part is the 32-step diagonal factorisation
+// of each tile in one warp.
+// ---------------------------------------------------------------------------
+template <int RP>
+struct TileChol {
+  static constexpr int TB = 32, NT = RP / TB, LDT = TB + 1, TSZ = TB * LDT;
+  static constexpr int NTILE = NT * (NT + 1) / 2;
+  static constexpr int NTHR = RP * 4 > 1024 ? 1024 : RP * 4;
+  static constexpr int PBUF = TB * RP;   // the transposed panel (32 x RP), or the T_IJ of one tile row
+  static constexpr size_t SMEM = ((size_t)NTILE * TSZ + PBUF + 3 * RP) * sizeof(float);
+  static_assert(RP % TB == 0 && NT >= 2, "tile form for r_pad >= 64");
+};
+
+__device__ __forceinline__ int tile_index(int I, int J) { return ((I * (I + 1)) >> 1) + J; }
+
+// tile (I, J) of the lower triangle of tiles from its index q
+__device__ __forceinline__ void tile_of(int q, int& I, int& J) {
+  I = 0;
+  while ((((I + 1) * (I + 2)) >> 1) <= q) ++I;
+  J = q - ((I * (I + 1)) >> 1);
+}
+
+template <int RP>
+__global__ void __launch_bounds__(TileChol<RP>::NTHR, 1) ldlt_inv_tile_kernel(const float* __restrict__ G, int r,
+                                                                          float* __restrict__ Ginv,
+                                                                          int* __restrict__ status) {
+  using C = TileChol<RP>;
+  constexpr int TB = C::TB, NT = C::NT, LDT = C::LDT, TSZ = C::TSZ, NTHR = C::NTHR;
+  extern __shared__ __align__(16) float smt[];
+  float* A = smt;                        // NTILE tiles: the matrix, then L and Y
+  float* P = A + C::NTILE * TSZ;         // PBUF
+  float* dv = P + C::PBUF;               // RP: d_k
+  float* invd = dv + RP;                 // RP: 1 / d_k
+  float* diag0 = invd + RP;              // RP: the diagonal of G
+  __shared__ int bad;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) bad = 0;
+  for (int t = tid; t < C::NTILE * TB * TB; t += NTHR) {
+    int I, J;
+    tile_of(t / (TB * TB), I, J);
+    const int e = t % (TB * TB), ii = e / TB, jj = e % TB, i = I * TB + ii, j = J * TB + jj;
+    const float g = (i < r && j < r) ? G[(size_t)i * RP + j] : (i == j ? 1.f : 0.f);
+    A[(t / (TB * TB)) * TSZ + ii * LDT + jj] = g;
+    if (i == j) diag0[i] = g;
+  }
+  for (int e = tid; e < RP * RP; e += NTHR)
+    if (e / RP >= r || e % RP >= r) Ginv[e] = 0.f;
+  __syncthreads();
+  const float tol = 4.0f * (float)r * FLT_EPSILON;
+
+  // 1. G = L D L^T, tile column by tile column
+  for (int J = 0; J < NT; ++J) {
+    if (warp == 0) {
+      float* T = A + tile_index(J, J) * TSZ;
+      float a[TB];
+#pragma unroll
+      for (int j = 0; j < TB; ++j) a[j] = T[lane * LDT + j];
+      int badk = -1;
+#pragma unroll
+      for (int k = 0; k < TB; ++k) {
+        const float d = __shfl_sync(0xffffffffu, a[k], k);
+        const float inv = 1.0f / d;
+        const int kk = J * TB + k;
+        if (badk < 0 && kk < r && (!(d > tol * diag0[kk]) || !isfinite(d))) badk = kk;   // warp-uniform
+        if (lane == k) {
+          dv[kk] = d;
+          invd[kk] = inv;
+        }
+        const float aik = a[k];
+        const float l = aik * inv;
+        if (lane > k) a[k] = l;
+#pragma unroll
+        for (int j = k + 1; j < TB; ++j) a[j] = fmaf(-aik, __shfl_sync(0xffffffffu, l, j), a[j]);
+      }
+      // the unit lower factor of the tile, then its inverse Yt in registers
+#pragma unroll
+      for (int j = 0; j < TB; ++j)
+        if (j < lane) T[lane * LDT + j] = a[j];
+      __syncwarp();
+#pragma unroll
+      for (int j = 0; j < TB; ++j) a[j] = j == lane ? 1.f : 0.f;
+#pragma unroll
+      for (int m = 0; m + 1 < TB; ++m) {
+        const float lim = lane > m ? T[lane * LDT + m] : 0.f;
+#pragma unroll
+        for (int j = 0; j <= m; ++j) a[j] = fmaf(-lim, __shfl_sync(0xffffffffu, a[j], m), a[j]);
+      }
+      __syncwarp();
+#pragma unroll
+      for (int j = 0; j < TB; ++j) T[lane * LDT + j] = a[j];   // unit diagonal, zeros above
+      if (lane == 0 && badk >= 0) {
+        bad = 1;
+        set_status(status, NMD_ERR_NOT_SPD, badk, 0);
+      }
+    }
+    __syncthreads();
+    if (bad) {   // uniform: every thread reads the flag after the barrier
+      for (int e = tid; e < RP * RP; e += NTHR) Ginv[e] = 0.f;
+      return;
+    }
+    // 1b. L_IJ = A_IJ Yt^T D_J^{-1} for the rows below the diagonal tile
+    const float* Yt = A + tile_index(J, J) * TSZ;
+    const int row0 = (J + 1) * TB;
+    for (int i = row0 + warp; i < RP; i += NTHR / 32) {
+      float* Ai = A + tile_index(i / TB, J) * TSZ + (i % TB) * LDT;
+      float acc = 0.f;
+#pragma unroll 8
+      for (int m = 0; m < TB; ++m) acc = fmaf(Ai[m], Yt[lane * LDT + m], acc);
+      acc *= invd[J * TB + lane];
+      __syncwarp();
+      Ai[lane] = acc;
+      P[lane * RP + i] = acc;
+    }
+    __syncthreads();
+    // 1c. A_IK -= L_IJ D_J L_KJ^T for J < K <= I (lower half of diagonal tiles)
+    const int nt = NT - J - 1;
+    for (int b = tid; b < (nt * (nt + 1) / 2) * 64; b += NTHR) {
+      int I, K;
+      tile_of(b / 64, I, K);
+      I += J + 1;
+      K += J + 1;
+      const int u4 = (b % 64) / 8, v4 = b % 8;
+      if (I == K && v4 > u4) continue;
+      const int i0 = I * TB + 4 * u4, j0 = K * TB + 4 * v4;
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int k = 0; k < TB; ++k) {
+        const float dk = dv[J * TB + k];
+        const float4 pa = *(const float4*)(P + k * RP + i0);
+        const float4 pb = *(const float4*)(P + k * RP + j0);
+        const float ya[4] = {pa.x * dk, pa.y * dk, pa.z * dk, pa.w * dk};
+        const float yb[4] = {pb.x, pb.y, pb.z, pb.w};
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(ya[u], yb[v], acc[u][v]);
+      }
+      float* T = A + tile_index(I, K) * TSZ + 4 * u4 * LDT + 4 * v4;
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) T[u * LDT + v] -= acc[u][v];
+    }
+    __syncthreads();
+  }
+
+  // 2. Y = L^{-1} by tile rows; the diagonal tiles already hold their inverses
+  for (int I = 1; I < NT; ++I) {
+    for (int b = tid; b < I * 64; b += NTHR) {
+      const int J = b / 64, u4 = (b % 64) / 8, v4 = b % 8;
+      float acc[4][4] = {};
+      for (int K = J; K < I; ++K) {
+        const float* L = A + tile_index(I, K) * TSZ + 4 * u4 * LDT;
+        const float* Y = A + tile_index(K, J) * TSZ + 4 * v4;
+#pragma unroll 4
+        for (int m = 0; m < TB; ++m) {
+          float la[4], yb[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) la[u] = L[u * LDT + m];
+#pragma unroll
+          for (int v = 0; v < 4; ++v) yb[v] = Y[m * LDT + v];
+#pragma unroll
+          for (int u = 0; u < 4; ++u)
+#pragma unroll
+            for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(la[u], yb[v], acc[u][v]);
+        }
+      }
+      float* T = P + J * TB * TB + 4 * u4 * TB + 4 * v4;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) *(float4*)(T + u * TB) = make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
+    }
+    __syncthreads();
+    const float* Yd = A + tile_index(I, I) * TSZ;
+    for (int b = tid; b < I * 64; b += NTHR) {
+      const int J = b / 64, u4 = (b % 64) / 8, v4 = b % 8;
+      const float* T = P + J * TB * TB + 4 * v4;
+      float acc[4][4] = {};
+#pragma unroll 4
+      for (int m = 0; m < TB; ++m) {
+        float ya[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) ya[u] = Yd[(4 * u4 + u) * LDT + m];
+        const float4 t = *(const float4*)(T + m * TB);
+        const float tb[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(ya[u], tb[v], acc[u][v]);
+      }
+      float* Y = A + tile_index(I, J) * TSZ + 4 * u4 * LDT + 4 * v4;
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int v = 0; v < 4; ++v) Y[u * LDT + v] = -acc[u][v];
+    }
+    __syncthreads();
+  }
+
+  // 3. G^{-1}[a][b] = sum over k of Y[k][a] Y[k][b] / d_k, tile rows K >= the tiles of a and b
+  for (int b = tid; b < C::NTILE * 64; b += NTHR) {
+    int I, J;
+    tile_of(b / 64, I, J);
+    const int u4 = (b % 64) / 8, v4 = b % 8;
+    if (I == J && v4 > u4) continue;
+    const int a0 = I * TB + 4 * u4, b0 = J * TB + 4 * v4;
+    if (a0 >= r || b0 >= r) continue;
+    float acc[4][4] = {};
+    for (int K = I; K < NT; ++K) {
+      const float* Ya = A + tile_index(K, I) * TSZ + 4 * u4;
+      const float* Yb = A + tile_index(K, J) * TSZ + 4 * v4;
+#pragma unroll 4
+      for (int m = 0; m < TB; ++m) {
+        const float w = invd[K * TB + m];
+        float ya[4], yb[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) ya[u] = Ya[m * LDT + u] * w;
+#pragma unroll
+        for (int v = 0; v < 4; ++v) yb[v] = Yb[m * LDT + v];
+#pragma unroll
+        for (int u = 0; u < 4; ++u)
+#pragma unroll
+          for (int v = 0; v < 4; ++v) acc[u][v] = fmaf(ya[u], yb[v], acc[u][v]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+#pragma unroll
+      for (int v = 0; v < 4; ++v) {
+        const int ga = a0 + u, gb = b0 + v;
+        if (ga < r && gb < r && (a0 != b0 || v <= u)) {
+          Ginv[(size_t)ga * RP + gb] = acc[u][v];
+          Ginv[(size_t)gb * RP + ga] = acc[u][v];
+        }
+      }
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -1215,29 +1352,30 @@ void launch_small_gemm(const float* A, int64_t lda, const float* B, int64_t ldb,
 }
 
 void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cudaStream_t s) {
-  if (rp <= 128) {
-    const size_t smem = ldlt_reg_smem_bytes(rp);
-    switch (rp) {
-      case 16: ldlt_inv_reg_kernel<16><<<1, 64, smem, s>>>(G, r, Ginv, status); break;
-      case 32: ldlt_inv_reg_kernel<32><<<1, 128, smem, s>>>(G, r, Ginv, status); break;
-      case 64: ldlt_inv_reg_kernel<64><<<1, 256, smem, s>>>(G, r, Ginv, status); break;
-      default: {
-        static std::atomic<int> attr[kMaxDevices];
-        per_device(attr, [] {
-          return cudaFuncSetAttribute(ldlt_inv_reg_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                      (int)ldlt_reg_smem_bytes(128)) == cudaSuccess ? 1 : 0;
-        });
-        ldlt_inv_reg_kernel<128><<<1, 512, smem, s>>>(G, r, Ginv, status);
-      }
+  switch (rp) {
+    case 16: ldlt_inv_reg_kernel<16><<<1, 64, ldlt_reg_smem_bytes(16), s>>>(G, r, Ginv, status); break;
+    case 32: ldlt_inv_reg_kernel<32><<<1, 128, ldlt_reg_smem_bytes(32), s>>>(G, r, Ginv, status); break;
+    case 64:
+      ldlt_inv_tile_kernel<64><<<1, TileChol<64>::NTHR, TileChol<64>::SMEM, s>>>(G, r, Ginv, status);
+      break;
+    case 128: {
+      static std::atomic<int> attr[kMaxDevices];
+      per_device(attr, [] {
+        return cudaFuncSetAttribute(ldlt_inv_tile_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)TileChol<128>::SMEM) == cudaSuccess ? 1 : 0;
+      });
+      ldlt_inv_tile_kernel<128><<<1, TileChol<128>::NTHR, TileChol<128>::SMEM, s>>>(G, r, Ginv, status);
+      break;
     }
-    return;
+    default: {
+      static std::atomic<int> attr[kMaxDevices];
+      per_device(attr, [] {
+        return cudaFuncSetAttribute(ldlt_inv_tile_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)TileChol<256>::SMEM) == cudaSuccess ? 1 : 0;
+      });
+      ldlt_inv_tile_kernel<256><<<1, TileChol<256>::NTHR, TileChol<256>::SMEM, s>>>(G, r, Ginv, status);
+    }
   }
-  static std::atomic<int> attr[kMaxDevices];
-  per_device(attr, [] {
-    return cudaFuncSetAttribute(chol_inv_kernel<32, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)chol_smem_bytes(256, 256, false)) == cudaSuccess ? 1 : 0;
-  });
-  chol_inv_kernel<32, false><<<1, 1024, chol_smem_bytes(r, rp, false), s>>>(G, r, rp, Ginv, status);
 }
 
 static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* partials, float* R, int64_t m0, int rp,
