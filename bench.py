@@ -40,6 +40,8 @@ WORKLOADS = {
     "identity": ("identity", 3, 512),
     "planted_tiny": ("planted_tiny", 4, 128),
     "connectome_dense_r64": ("connectome_dense_r64", 64, 4096),
+    "communities_r64": ("communities_r64", 64, 8192),
+    "communities_planted_r64": ("communities_planted_r64", 64, 8192),
 }
 
 
@@ -50,6 +52,27 @@ DENSE_TRAFFIC = {
     # (workload, precision, epilogue): (bytes per launch, dense_source_digest() of the code measured)
     ("connectome-139255-r64", "bf16", "z"): (18401792, "8dbd5df1c6cc41f5"),
 }
+
+
+def chunks_per_sweep(sol, wl, exact, N):
+    """(128-row M tile, Q chunk) pairs of the dense kernel in one sweep."""
+    _, bn = sol.range_mask(N.NMD_COL, 0, N.NMD_STOCH)   # the chunk size (the mask itself is not used)
+
+    def cdiv(a, b):
+        return -(-a // b)
+
+    m, n, br, bc = wl.m, wl.n, wl.block_rows, wl.block_cols
+    if exact:   # b rows against a whole factor, per block
+        return (sum(cdiv(min(br, m - i), 128) * cdiv(n, bn) for i in range(0, m, br)) +
+                sum(cdiv(min(bc, n - j), 128) * cdiv(m, bn) for j in range(0, n, bc)))
+    return (sum(cdiv(m, 128) * cdiv(min(bc, n - j), bn) for j in range(0, n, bc)) +
+            sum(cdiv(n, 128) * cdiv(min(br, m - i), bn) for i in range(0, m, br)))
+
+
+def skip_mode(args, N):
+    if args.range_search:
+        return N.NMD_SKIP_RANGE
+    return N.NMD_SKIP_VOTE if args.skip_zero_chunks else N.NMD_SKIP_NONE
 
 
 def dense_source_digest():
@@ -254,6 +277,9 @@ def main():
     ap.add_argument("--epilogue", choices=["z", "delta"], default="z")
     ap.add_argument("--skip-zero-chunks", action="store_true",
                     help="Delta form: skip the second product of chunks whose rectified tile is zero")
+    ap.add_argument("--range-search", action="store_true",
+                    help="Delta form: skip both dense products of the chunks a range search over the "
+                         "normalised factor rows clears (Sec. 4.3)")
     ap.add_argument("--schedule", choices=["workload", "exact", "stoch"], default="workload",
                     help="sweep kind: the workload's own, or exact / stochastic")
     ap.add_argument("--init", choices=["normal", "paper"], default="normal",
@@ -320,7 +346,7 @@ def main():
     sol = N.Solver(wl.S, wl.r, block_rows=wl.block_rows, block_cols=wl.block_cols,
                    schedule=N.NMD_EXACT if exact else N.NMD_STOCH,
                    eta=wl.eta, gamma=wl.gamma, precision=prec, epilogue=epi, seed=0,
-                   skip_zero_chunks=args.skip_zero_chunks)
+                   skip_zero_chunks=skip_mode(args, N))
     W0, H0 = wl.W0, wl.H0
     if args.init == "paper":
         W0, H0 = WLm.init_factors(wl.m, wl.n, wl.r, 0, signs="paper")
@@ -513,8 +539,9 @@ def main():
                            "eta": wl.eta,
                            "gamma": wl.gamma, "precision": args.precision,
                            "epilogue": args.epilogue, "init": args.init,
-                           "skip_zero_chunks": args.skip_zero_chunks,
+                           "skip_zero_chunks": ["none", "vote", "range"][skip_mode(args, N)],
                            "skipped_chunks_per_sweep": skipped / args.steps,
+                           "chunks_per_sweep": chunks_per_sweep(sol, wl, exact, N),
                            "parallelism": "replicas" if ws > 1 else "single GPU",
                            "workspace_mb": round(ws_bytes / 2**20, 1),
                            "l2": ("workspace smaller than L2: L2 flushed (512 MB write) before each timed sweep"

@@ -97,10 +97,29 @@ typedef struct {
   int32_t precision;    /* nmd_precision */
   int32_t epilogue;     /* nmd_epilogue */
   uint64_t seed;        /* block-order seed */
-  int32_t skip_zero_chunks;  /* Delta form: skip the second product of Q chunks whose rectified
-                              * tile is zero (Sec. 4.3; see nmd_skip_count).  Default 0: the check
-                              * costs the dense kernel time when no chunk vanishes */
+  int32_t skip_zero_chunks;  /* nmd_skip_mode; Delta form only (ignored otherwise).  Default
+                              * NMD_SKIP_NONE: the checks cost the dense kernel time when no
+                              * chunk vanishes */
 } nmd_options;
+
+/* Chunk skipping in the Delta-form dense term -max(0, L) Q (Sec. 4.3: the
+ * rectified matrix max(0, A B^T) is sparse when the model is mostly
+ * negative).  A chunk is the product of a 128-row M tile with 64 or 128
+ * Q-side rows (nmd_range_mask reports the count):
+ *   NMD_SKIP_VOTE  -- the first product is computed, and the second is
+ *                     skipped where max(0, L) is zero on the whole chunk;
+ *   NMD_SKIP_RANGE -- before the dense kernel, a range search over the
+ *                     normalised factor rows (eq. range-search: L_ij > 0
+ *                     exactly when ||a_i/|a_i| - b_j/|b_j|||^2 < 2) clears the
+ *                     chunks on which every L_ij <= 0, and both products are
+ *                     skipped there.  The test bounds the distance of every
+ *                     pair from below by that of the balls around the tile's
+ *                     and the chunk's normalised rows, with a margin for the
+ *                     rounding of the operands, so a cleared chunk adds
+ *                     exactly zero and the results equal those without
+ *                     skipping.
+ * Both count the skipped chunks (nmd_skip_count). */
+typedef enum { NMD_SKIP_NONE = 0, NMD_SKIP_VOTE = 1, NMD_SKIP_RANGE = 2 } nmd_skip_mode;
 
 typedef struct {
   double obj;        /* ||Z - L||_F / ||S||_F  (eq. auxCost) */
@@ -295,14 +314,28 @@ nmd_status nmd_selftest_wait_timeout(nmd_handle* h, int64_t limit_ns);
 /* Number of kernel launches this handle has issued (for launch accounting). */
 int64_t nmd_launch_count(const nmd_handle* h);
 
-/* Delta form (epilogue NMD_EPI_DELTA): number of Q chunks (64 or 128 Q-side
- * rows against a 128-row M tile) whose second product the tensor-core panel
- * kernel skipped because max(0, L) was zero on the whole chunk -- the tile
- * skipping of Sec. 4.3 (the rectified tile is sparse where the model is
- * mostly negative).  The first chunk of every tile is always computed.
- * Counts since creation or the last reset; synchronises; reset != 0 sets
- * the count back to zero. */
+/* Delta form (epilogue NMD_EPI_DELTA) with chunk skipping on: the number of
+ * Q chunks (64 or 128 Q-side rows against a 128-row M tile) that the
+ * tensor-core panel kernel skipped -- NMD_SKIP_VOTE: chunks whose second
+ * product was skipped because max(0, L) was zero on the whole chunk;
+ * NMD_SKIP_RANGE: chunks the range search cleared, both products skipped
+ * (Sec. 4.3).  The first chunk of a tile is always computed under
+ * NMD_SKIP_VOTE, and a tile with every chunk cleared computes its first
+ * under NMD_SKIP_RANGE.  Counts since creation or the last reset;
+ * synchronises; reset != 0 sets the count back to zero. */
 nmd_status nmd_skip_count(nmd_handle* h, int64_t* skipped, int32_t reset);
+
+/* Verification hook: the range-search mask of one block update (Sec. 4.3,
+ * eq. range-search), computed from the current factors exactly as the step
+ * would compute it under NMD_SKIP_RANGE, whatever the options say.  Writes
+ * *ntiles (128-row M tiles), *words (32-bit words per tile), *chunk_rows
+ * (Q-side rows per chunk) and, if mask != NULL and capacity >= ntiles x
+ * words, the mask to host memory: word w of tile t at mask[t words + w],
+ * bit c set = chunk 32 w + c is cleared (every L_ij of the tile's rows and
+ * the chunk's rows is <= 0).  NMD_ERR_UNSUPPORTED for NMD_SIMT.
+ * Synchronises. */
+nmd_status nmd_range_mask(nmd_handle* h, int32_t side, int64_t block, int32_t kind, uint32_t* mask,
+                          int64_t capacity, int64_t* ntiles, int64_t* words, int64_t* chunk_rows);
 
 const char* nmd_status_string(nmd_status s);
 const char* nmd_last_error(const nmd_handle* h);

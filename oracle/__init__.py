@@ -6,4 +6,5 @@ of ``bench.py``; the CUDA library and its Python binding never import it.
 from .salsa import *  # noqa: F401,F403
 from .salsa import (ROW, COL, EXACT, STOCH, ALTERNATE, PHASED, NotSPD, Options, State,  # noqa: F401
                     Sparse, block_permutation, block_range, num_blocks, cholesky,
-                    solve_normal, update_z, loss, splitmix64_mix, SplitMix64)
+                    solve_normal, update_z, loss, splitmix64_mix, SplitMix64,
+                    positive_set, range_search_set)

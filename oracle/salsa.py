@@ -19,6 +19,9 @@ What it computes (paper notation: L = A B^T, A = W is m x r, B = H^T is n x r):
   eq. lsqA_sto), read as heavy ball E_t = U_t + gamma E_{t-1}, M += E_t.
 * Losses: objective ||Z - L||_F / ||S||_F (eq. auxCost, evaluated through
   eq. SLloss), RMSE (eq. RMSE) and weighted Jaccard distance (eq. WJD).
+* The index set Omega of the positive entries of L (Sec. 4.3), both by its
+  definition (eq. nonzeros) and as a range search over the normalised rows
+  (eq. range-search).
 
 Every Z panel is materialised explicitly in fp64, the right-hand side R = Z Q
 and Gram matrix G = Q^T Q are formed with plain matrix products, G is factored
@@ -214,6 +217,38 @@ def loss(Sp: Sparse, A: np.ndarray, B: np.ndarray, rows: Optional[np.ndarray] = 
 # ---------------------------------------------------------------------------
 # The solver state and one block update
 # ---------------------------------------------------------------------------
+
+# ---------------------------------------------------------------------------
+# The positive entries of L (Sec. 4.3, "Fast similarity search")
+# ---------------------------------------------------------------------------
+
+def positive_set(A: np.ndarray, B: np.ndarray) -> np.ndarray:
+    """Omega of eq. nonzeros: the pairs (i, j) with (A B^T)_ij > 0, as an
+    m x n boolean array (fp64 product)."""
+    return (np.asarray(A, np.float64) @ np.asarray(B, np.float64).T) > 0
+
+
+def range_search_set(A: np.ndarray, B: np.ndarray) -> np.ndarray:
+    """Omega of eq. range-search: the pairs whose normalised rows a_i/|a_i|
+    and b_j/|b_j| are less than two units of squared distance apart, found
+    by comparing every pair (brute force).  A zero row has no direction and
+    takes part in no pair (its entries of L are zero)."""
+    A = np.asarray(A, np.float64)
+    B = np.asarray(B, np.float64)
+    na = np.sqrt((A * A).sum(axis=1))
+    nb = np.sqrt((B * B).sum(axis=1))
+    out = np.zeros((A.shape[0], B.shape[0]), dtype=bool)
+    for i in range(A.shape[0]):
+        if na[i] == 0:
+            continue
+        ahat = A[i] / na[i]
+        for j in range(B.shape[0]):
+            if nb[j] == 0:
+                continue
+            d = ahat - B[j] / nb[j]
+            out[i, j] = float(d @ d) < 2.0
+    return out
+
 
 @dataclasses.dataclass
 class Options:

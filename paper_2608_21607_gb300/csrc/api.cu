@@ -74,6 +74,9 @@ nmd_status check_options(const nmd_options* o, std::string* why) {
     *why = "unknown precision"; return NMD_ERR_INVALID;
   }
   if (o->epilogue != NMD_EPI_Z && o->epilogue != NMD_EPI_DELTA) { *why = "unknown epilogue"; return NMD_ERR_INVALID; }
+  if (o->skip_zero_chunks < NMD_SKIP_NONE || o->skip_zero_chunks > NMD_SKIP_RANGE) {
+    *why = "unknown chunk-skipping mode"; return NMD_ERR_INVALID;
+  }
   return NMD_OK;
 }
 
@@ -257,6 +260,15 @@ struct Carver {
   }
 };
 
+// Words of the range-search mask of any step: per 128-row M tile one bit
+// per Q chunk (chunks of at least 64 rows), words rounded up per tile.  A
+// stochastic step has tiles over a whole factor and chunks over a block, an
+// exact step the other way round; both are bounded by tiles(N) x words(N).
+int64_t range_mask_words(int64_t m, int64_t n) {
+  const int64_t N = std::max(m, n);
+  return ((N + 127) / 128) * ((((N + 63) / 64) + 31) / 32);
+}
+
 void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanels, int64_t maxseg,
             int64_t nflags, Workspace* w, Factor* W, Factor* B) {
   w->rowptr = c.take<int64_t>(m + 1);
@@ -291,6 +303,12 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->seg_partials = c.take<float>((size_t)std::max<int64_t>(maxseg, 1) * rp);
   w->flags = c.take<uint8_t>((size_t)std::max<int64_t>(nflags, 1));
   w->rpart = c.take<float>((size_t)kRpartRows * rp);
+  const int64_t N = std::max(m, n);
+  w->ball_m = c.take<float>((size_t)((N + 127) / 128) * rp);
+  w->rad_m = c.take<float>((size_t)((N + 127) / 128));
+  w->ball_q = c.take<float>((size_t)((N + 63) / 64) * rp);
+  w->rad_q = c.take<float>((size_t)((N + 63) / 64));
+  w->rmask = c.take<uint32_t>((size_t)range_mask_words(m, n));
   w->loss_part = c.take<double>((size_t)kLossParts * 8);
   w->loss_out = c.take<double>(8);
   w->status = c.take<int>(kStatusWords);
@@ -618,6 +636,27 @@ nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro,
 // block) pair (combined sub-sampling)
 constexpr int kCombined = 2;
 
+// The range-search mask of a step (Sec. 4.3, eq. range-search): balls around
+// the normalised rows of its 128-row M tiles and of its Q chunks, then one
+// bit per (tile, chunk) pair whose balls are far enough apart that L <= 0
+// on all of it.  Sets a->rmask and a->rwords.
+void range_pass(nmd_handle* h, const Roles& ro, StepArgs* a, cudaStream_t s) {
+  const int bn = panel_chunk_rows(h->rp, h->opt.precision);
+  const int64_t ntiles = (ro.M + 127) / 128, nchunks = (ro.K + bn - 1) / bn, words = (nchunks + 31) / 32;
+  launch_range_balls(ro.fm->master, ro.m0, ro.M, ro.fq->master, ro.q0, ro.K, bn, h->rp, h->ws.ball_m,
+                     h->ws.rad_m, h->ws.ball_q, h->ws.rad_q, s);
+  launch_range_mask(h->ws.ball_m, h->ws.rad_m, ntiles, h->ws.ball_q, h->ws.rad_q, nchunks, words, h->rp,
+                    h->ws.rmask, s);
+  h->launches += 2;
+  a->rmask = h->ws.rmask;
+  a->rwords = words;
+}
+
+bool range_on(const nmd_handle* h) {
+  return h->opt.skip_zero_chunks == NMD_SKIP_RANGE && h->opt.epilogue == NMD_EPI_DELTA &&
+         h->opt.precision != NMD_SIMT;
+}
+
 nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_update, const NextUse* next);
 
 nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_update,
@@ -631,7 +670,7 @@ nmd_status run_step(nmd_handle* h, int side, int64_t block, int kind, bool do_up
 nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_update, const NextUse* next) {
   nmd_status st = NMD_OK;
   StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
-              h->opt.skip_zero_chunks != 0};
+              h->opt.skip_zero_chunks == NMD_SKIP_VOTE};
   cudaStream_t s = h->cur;
   // wait for deferred updates of rows this step reads or writes, and for
   // those of two steps back (they read the copies of R and G^{-1} reused now)
@@ -705,6 +744,7 @@ nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_upda
   CK(h, cudaEventRecord(h->ev_join, h->side));
   CK(h, cudaEventRecord(h->ev_join2, h->side2));
   // dense Z-panel contraction R = P(L) Q over every (M-side, Q-side) pair
+  if (range_on(h)) range_pass(h, ro, &a, s);
   {
     TimedScope ts(h, NMD_K_DENSE);
     if (h->opt.precision == NMD_SIMT) {
@@ -1179,13 +1219,34 @@ nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_
   if (st != NMD_OK) return st;
   if (h->opt.precision == NMD_SIMT) return fail(h, NMD_ERR_UNSUPPORTED, "dense products hook needs a tensor-core precision");
   StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
-              h->opt.skip_zero_chunks != 0};
+              h->opt.skip_zero_chunks == NMD_SKIP_VOTE};
   st = launch_panel_tc(a, h->ws.R, h->ws.status, h->ws.counters, h->num_sms, h->stream, &h->launches, d_L);
   if (st != NMD_OK) return fail(h, st, "no tensor-core kernel for this rank/precision on this device");
   if ((st = after_launch(h, "dense products")) != NMD_OK) return st;
   if ((st = sync_and_check(h)) != NMD_OK) return st;
   if (rows) *rows = ro.M;
   if (cols) *cols = ro.K;
+  return NMD_OK;
+}
+
+nmd_status nmd_range_mask(nmd_handle* h, int32_t side, int64_t block, int32_t kind, uint32_t* mask,
+                          int64_t capacity, int64_t* ntiles, int64_t* words, int64_t* chunk_rows) {
+  if (!h || !ntiles || !words || !chunk_rows) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_range_mask");
+  DeviceScope dg(h);
+  Roles ro;
+  nmd_status st = roles(h, side, block, kind, &ro);
+  if (st != NMD_OK) return st;
+  if (h->opt.precision == NMD_SIMT) return fail(h, NMD_ERR_UNSUPPORTED, "range mask hook needs a tensor-core precision");
+  if ((st = wait_all_pending(h)) != NMD_OK) return st;
+  StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms};
+  range_pass(h, ro, &a, h->stream);
+  if ((st = after_launch(h, "range mask")) != NMD_OK) return st;
+  if ((st = sync_and_check(h)) != NMD_OK) return st;
+  *ntiles = (ro.M + 127) / 128;
+  *words = a.rwords;
+  *chunk_rows = panel_chunk_rows(h->rp, h->opt.precision);
+  if (mask && capacity >= *ntiles * *words)
+    CK(h, cudaMemcpy(mask, h->ws.rmask, (size_t)(*ntiles * *words) * sizeof(uint32_t), cudaMemcpyDeviceToHost));
   return NMD_OK;
 }
 
@@ -1197,7 +1258,7 @@ nmd_status nmd_support_term(nmd_handle* h, int32_t side, int64_t block, int32_t 
   if (st != NMD_OK) return st;
   if ((st = wait_all_pending(h)) != NMD_OK) return st;
   StepArgs a{ro.fm, ro.fq, ro.m0, ro.M, ro.q0, ro.K, h->r, h->rp, h->opt.precision, h->opt.epilogue, h->num_sms,
-              h->opt.skip_zero_chunks != 0};
+              h->opt.skip_zero_chunks == NMD_SKIP_VOTE};
   cudaStream_t s = h->stream;
   CK(h, cudaMemsetAsync(d_R, 0, (size_t)ro.M * h->rp * sizeof(float), s));
   {

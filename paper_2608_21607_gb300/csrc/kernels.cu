@@ -1378,6 +1378,212 @@ void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cu
   }
 }
 
+// ---------------------------------------------------------------------------
+// Range search over the normalised factor rows (Sec. 4.3, eqs. nonzeros and
+// range-search): L_ij > 0 exactly when ||a^_i - b^_j||^2 < 2, with a^ and b^
+// the rows scaled to unit length.  A one-level spatial index: a ball (centre
+// c, radius rho) around the normalised nonzero rows of every 128-row M tile
+// and of every Q chunk of a step.  By the triangle inequality every pair of
+// a tile and a chunk has
+//     ||a^ - b^|| >= ||c_A - c_B|| - rho_A - rho_B;
+// where that bound is at least sqrt(2 + 2 gamma), every pair has
+// a^ . b^ <= -gamma, so L < 0 (or L = 0 for zero rows) on the whole (tile,
+// chunk), and the Delta-form dense term -max(0, L) Q adds nothing there: the
+// dense kernel skips both of its products for that chunk.
+// gamma = 2^-7 covers the bf16 rounding of the operands that the dense
+// kernel multiplies (its L differs from the masters' a . b by at most about
+// 2^-8 |a| |b|) and its fp32 accumulation; the ball arithmetic is rounded
+// outwards by 2^-12 relative plus 2^-14 (the fp32 normalisation of the rows
+// is good to about 1e-6).  The balls come from the fp32 masters.
+// ---------------------------------------------------------------------------
+// Balls of groups of T consecutive rows: groups [0, g1) over the rows of the
+// first set (the M tiles), groups [g1, gridDim.x) over the second (the Q
+// chunks), in one launch.  Each row is read by RP / 8 lanes (8 columns each,
+// two 16-byte loads), so a warp holds 256 / RP rows at once; two passes:
+// the mean of the unit vectors of the nonzero rows, then the largest
+// distance from it.
+struct BallSet {
+  const float* X;
+  int64_t x0, N;
+  int T;
+  float* centre;
+  float* radius;
+};
+
+template <int RP>
+__global__ void __launch_bounds__(256) range_ball_kernel(BallSet a, int64_t g1, BallSet b) {
+  constexpr int LPR = RP / 8;           // lanes per row
+  constexpr int RPW = 32 / LPR;         // rows per warp at once
+  __shared__ float part[8][RP];
+  __shared__ float cs[RP];
+  __shared__ float rmax[8];
+  __shared__ int cnt[8];
+  const bool first = blockIdx.x < g1;
+  const BallSet& S = first ? a : b;
+  const int64_t g = first ? blockIdx.x : blockIdx.x - g1;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int sub = lane % LPR, c0 = 8 * sub;   // this lane's 8 columns
+  const int64_t r0 = g * S.T, r1 = r0 + S.T < S.N ? r0 + S.T : S.N;
+  // the unit vector of row i (zero for a zero row or a row past the group)
+  auto unit = [&](int64_t i, float (&v)[8]) {
+    if (i < r1) {
+      const float4* row = (const float4*)(S.X + (S.x0 + i) * RP + c0);
+      const float4 p = __ldg(row), q = __ldg(row + 1);
+      v[0] = p.x; v[1] = p.y; v[2] = p.z; v[3] = p.w; v[4] = q.x; v[5] = q.y; v[6] = q.z; v[7] = q.w;
+    } else {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) v[k] = 0.f;
+    }
+    float ss = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) ss = fmaf(v[k], v[k], ss);
+#pragma unroll
+    for (int o = 1; o < LPR; o <<= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+    const float inv = ss > 0.f ? rsqrtf(ss) : 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] *= inv;
+    return ss > 0.f;
+  };
+  float acc[8];
+#pragma unroll
+  for (int k = 0; k < 8; ++k) acc[k] = 0.f;
+  int n = 0;
+  for (int64_t i0 = r0 + warp * RPW; i0 < r1; i0 += 8 * RPW) {
+    float v[8];
+    if (unit(i0 + lane / LPR, v)) {
+      n += sub == 0;
+#pragma unroll
+      for (int k = 0; k < 8; ++k) acc[k] += v[k];
+    }
+  }
+  // column sums over the warp's row slots, then over the warps
+#pragma unroll
+  for (int o = LPR; o < 32; o <<= 1) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) acc[k] += __shfl_xor_sync(0xffffffffu, acc[k], o);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) n += __shfl_xor_sync(0xffffffffu, n, o);
+  if (lane < LPR)
+#pragma unroll
+    for (int k = 0; k < 8; ++k) part[warp][c0 + k] = acc[k];
+  if (lane == 0) cnt[warp] = n;
+  __syncthreads();
+  int ntot = 0;
+#pragma unroll
+  for (int w = 0; w < 8; ++w) ntot += cnt[w];
+  for (int c = threadIdx.x; c < RP; c += 256) {
+    float sum = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) sum += part[w][c];
+    cs[c] = ntot > 0 ? sum / (float)ntot : 0.f;
+  }
+  __syncthreads();
+  float rm = 0.f;
+  for (int64_t i0 = r0 + warp * RPW; i0 < r1; i0 += 8 * RPW) {
+    float v[8];
+    const bool nz = unit(i0 + lane / LPR, v);
+    float d2 = 0.f;
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const float e = v[k] - cs[c0 + k];
+      d2 = fmaf(e, e, d2);
+    }
+#pragma unroll
+    for (int o = 1; o < LPR; o <<= 1) d2 += __shfl_xor_sync(0xffffffffu, d2, o);
+    if (nz) rm = fmaxf(rm, d2);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) rm = fmaxf(rm, __shfl_xor_sync(0xffffffffu, rm, o));
+  if (lane == 0) rmax[warp] = rm;
+  __syncthreads();
+  for (int c = threadIdx.x; c < RP; c += 256) S.centre[g * RP + c] = cs[c];
+  if (threadIdx.x == 0) {
+    float m = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) m = fmaxf(m, rmax[w]);
+    S.radius[g] = ntot > 0 ? sqrtf(m) : -1.f;   // -1: the group has no nonzero row
+  }
+}
+
+// One block per M tile: bit c of word w of the tile's mask is set when the
+// ball test clears Q chunk 32 w + c (every pair of the tile and the chunk has
+// L <= 0).  A group without a nonzero row has L = 0 against everything.
+// Warp w takes chunks w, w + 8, ...; its lanes read a chunk's centre
+// together.
+template <int RP>
+__global__ void __launch_bounds__(256) range_mask_kernel(const float* __restrict__ cm, const float* __restrict__ rm,
+                                                         const float* __restrict__ cq, const float* __restrict__ rq,
+                                                         int64_t nchunks, int64_t words, uint32_t* __restrict__ mask) {
+  constexpr float kOut = 1.0f + 1.0f / 4096.0f;
+  constexpr float kIn = 1.0f - 1.0f / 4096.0f;
+  constexpr float kThresh = 1.4201f;   // sqrt(2 + 2^-6) (1 + 2^-12) = 1.42007...
+  constexpr int CPL = RP >= 32 ? RP / 32 : 1;
+  __shared__ float ca[RP];
+  __shared__ uint32_t bits[64];
+  const int64_t t = blockIdx.x;
+  for (int c = threadIdx.x; c < RP; c += 256) ca[c] = cm[t * RP + c];
+  const float ra = rm[t];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int64_t w0 = 0; w0 < words; w0 += 64) {
+    const int nw = (int)(words - w0 < 64 ? words - w0 : 64);
+    __syncthreads();
+    if (threadIdx.x < 64) bits[threadIdx.x] = 0u;
+    __syncthreads();
+    const int64_t cend = (w0 + nw) * 32 < nchunks ? (w0 + nw) * 32 : nchunks;
+    for (int64_t c = w0 * 32 + warp; c < cend; c += 8) {
+      const float rb = rq[c];
+      bool skip;
+      if (ra < 0.f || rb < 0.f) {
+        skip = true;
+      } else {
+        float d2 = 0.f;
+#pragma unroll
+        for (int j = 0; j < CPL; ++j) {
+          const int k = lane + 32 * j;
+          const float e = k < RP ? ca[k] - cq[c * RP + k] : 0.f;
+          d2 = fmaf(e, e, d2);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) d2 += __shfl_xor_sync(0xffffffffu, d2, o);
+        const float lb = sqrtf(d2) * kIn - (ra + rb) * kOut - 1.0f / 16384.0f;
+        skip = lb >= kThresh;
+      }
+      if (skip && lane == 0) atomicOr(&bits[(c >> 5) - w0], 1u << (c & 31));
+    }
+    __syncthreads();
+    for (int w = threadIdx.x; w < nw; w += 256) mask[t * words + w0 + w] = bits[w];
+  }
+}
+
+void launch_range_balls(const float* Xm, int64_t m0, int64_t M, const float* Xq, int64_t q0, int64_t K, int bn,
+                        int rp, float* cm, float* rm, float* cq, float* rq, cudaStream_t s) {
+  const int64_t g1 = (M + 127) / 128, g2 = (K + bn - 1) / bn;
+  if (g1 + g2 == 0) return;
+  const BallSet a{Xm, m0, M, 128, cm, rm}, b{Xq, q0, K, bn, cq, rq};
+  const unsigned grid = (unsigned)(g1 + g2);
+  switch (rp) {
+    case 16: range_ball_kernel<16><<<grid, 256, 0, s>>>(a, g1, b); break;
+    case 32: range_ball_kernel<32><<<grid, 256, 0, s>>>(a, g1, b); break;
+    case 64: range_ball_kernel<64><<<grid, 256, 0, s>>>(a, g1, b); break;
+    case 128: range_ball_kernel<128><<<grid, 256, 0, s>>>(a, g1, b); break;
+    default: range_ball_kernel<256><<<grid, 256, 0, s>>>(a, g1, b); break;
+  }
+}
+
+void launch_range_mask(const float* cm, const float* rm, int64_t ntiles, const float* cq, const float* rq,
+                       int64_t nchunks, int64_t words, int rp, uint32_t* mask, cudaStream_t s) {
+  if (ntiles == 0) return;
+  const unsigned g = (unsigned)ntiles;
+  switch (rp) {
+    case 16: range_mask_kernel<16><<<g, 256, 0, s>>>(cm, rm, cq, rq, nchunks, words, mask); break;
+    case 32: range_mask_kernel<32><<<g, 256, 0, s>>>(cm, rm, cq, rq, nchunks, words, mask); break;
+    case 64: range_mask_kernel<64><<<g, 256, 0, s>>>(cm, rm, cq, rq, nchunks, words, mask); break;
+    case 128: range_mask_kernel<128><<<g, 256, 0, s>>>(cm, rm, cq, rq, nchunks, words, mask); break;
+    default: range_mask_kernel<256><<<g, 256, 0, s>>>(cm, rm, cq, rq, nchunks, words, mask); break;
+  }
+}
+
 static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* partials, float* R, int64_t m0, int rp,
                           cudaStream_t s) {
   const unsigned grid = (unsigned)nmulti;

@@ -102,6 +102,10 @@ struct StepArgs {
   int precision, epilogue;
   int num_sms = 152;         // streaming multiprocessors of the device (grid sizing)
   bool skip_zero = false;    // Delta form: skip chunks whose rectified tile is zero
+  // Delta form, range search: per 128-row M tile, `rwords` words whose bit c
+  // marks Q chunk c as all L <= 0 (both dense products skipped); or nullptr
+  const uint32_t* rmask = nullptr;
+  int64_t rwords = 0;
 };
 
 struct Workspace {
@@ -140,6 +144,13 @@ struct Workspace {
   float* seg_partials = nullptr;  // max segments x rp (sparse correction of long rows)
   uint8_t* flags = nullptr;       // the panels' support-row flags, concatenated
   float* rpart = nullptr;         // kRpartRows x rp: partial R's of split-K steps
+  // range search (Delta form): balls of the M tiles and Q chunks of a step
+  // (centres rp floats each, radii) and the skip mask of its (tile, chunk) pairs
+  float* ball_m = nullptr;        // ceil(max(m, n) / 128) x rp
+  float* rad_m = nullptr;
+  float* ball_q = nullptr;        // ceil(max(m, n) / 64) x rp
+  float* rad_q = nullptr;
+  uint32_t* rmask = nullptr;      // range_mask_words(m, n)
 };
 
 constexpr int kGramParts = 64;
@@ -269,5 +280,13 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
 nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts,
                                 int* status, cudaStream_t s, int64_t* launches);
 bool tc_supported(int rp, int precision);
+// Q-side rows per chunk of the tensor-core dense kernel (64 or 128)
+int panel_chunk_rows(int rp, int precision);
+// balls of the 128-row M tiles of rows [m0, m0 + M) of Xm and of the bn-row
+// Q chunks of rows [q0, q0 + K) of Xq (one launch)
+void launch_range_balls(const float* Xm, int64_t m0, int64_t M, const float* Xq, int64_t q0, int64_t K, int bn,
+                        int rp, float* cm, float* rm, float* cq, float* rq, cudaStream_t s);
+void launch_range_mask(const float* cm, const float* rm, int64_t ntiles, const float* cq, const float* rq,
+                       int64_t nchunks, int64_t words, int rp, uint32_t* mask, cudaStream_t s);
 
 }  // namespace nmd

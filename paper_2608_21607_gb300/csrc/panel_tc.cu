@@ -138,6 +138,11 @@ struct TcParams {
   // [q0 + z ksplit, ...) and writes its partial R at R + z rstride
   int64_t ksplit;              // 0: no split
   int64_t rstride;
+  // range-search skipping (Delta form): bit c of tile t's words
+  // rmask[t rwords ...] set = Q chunk c of the step is all L <= 0 for the
+  // tile's rows (see range_mask_kernel); nullptr: no chunk is skipped
+  const uint32_t* rmask;
+  int64_t rwords;
 };
 
 __device__ __forceinline__ void record(int* status, int code, int detail) {
@@ -187,16 +192,71 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   return ok != 0;
 }
 
-// SKIP (Delta form only): skip the second product of chunks whose rectified
-// tile is zero; a separate instantiation, so that the kernel without it
-// carries none of the checks.
-template <int RP, int EPI, bool SPLIT, bool LOSS, bool SKIP>
+// The live Q chunks [0, n) of one tile (this CTA's split of it starts at
+// chunk c0 of the tile's mask): those whose mask bit is clear.  A tile whose
+// chunks are all masked still computes its chunk 0, which gives R = 0 (its L
+// is <= 0 throughout), so that every tile has a first and a last chunk and
+// the R hand-off is the same as without skipping.  The first 64 chunks'
+// bits are kept in a register (a stochastic step has at most 64 chunks).
+struct ChunkMask {
+  const uint32_t* m;   // the tile's words, or nullptr (every chunk live)
+  int64_t c0;
+  bool none;           // every chunk masked
+  uint64_t live64;     // bit c: chunk c (< 64) is live
+  __device__ __forceinline__ bool masked_far(int64_t c) const {
+    const int64_t b = c0 + c;
+    return (m[b >> 5] >> (b & 31)) & 1u;
+  }
+  __device__ __forceinline__ bool live(int64_t c) const {
+    if (m == nullptr) return true;
+    if (none) return c == 0;
+    return c < 64 ? ((live64 >> c) & 1ull) != 0 : !masked_far(c);
+  }
+};
+
+template <bool RANGE>
+__device__ __forceinline__ ChunkMask chunk_mask(const TcParams& p, int64_t t, int64_t c0, int64_t n,
+                                                int64_t* last, int64_t* nlive) {
+  ChunkMask cm{nullptr, c0, false, ~0ull};
+  *last = n - 1;
+  *nlive = n;
+  if (!RANGE || p.rmask == nullptr) return cm;
+  cm.m = p.rmask + t * p.rwords;
+  // bits c0 .. c0 + 63 of the tile's words (words past the end read as masked)
+  const int64_t w = c0 >> 5;
+  const int sh = (int)(c0 & 31);
+  const uint32_t w0 = w < p.rwords ? cm.m[w] : ~0u;
+  const uint32_t w1 = w + 1 < p.rwords ? cm.m[w + 1] : ~0u;
+  const uint32_t w2 = w + 2 < p.rwords ? cm.m[w + 2] : ~0u;
+  const uint64_t lo = ((uint64_t)w1 << 32) | w0;
+  const uint64_t bits = sh ? (lo >> sh) | ((uint64_t)w2 << (64 - sh)) : lo;
+  const uint64_t inrange = n >= 64 ? ~0ull : ((1ull << n) - 1ull);
+  cm.live64 = ~bits & inrange;
+  int64_t cnt = __popcll(cm.live64), lst = cm.live64 ? 63 - __clzll(cm.live64) : -1;
+  for (int64_t c = 64; c < n; ++c)
+    if (!cm.masked_far(c)) {
+      ++cnt;
+      lst = c;
+    }
+  cm.none = cnt == 0;
+  *last = cm.none ? 0 : lst;
+  *nlive = cm.none ? 1 : cnt;
+  return cm;
+}
+
+// SKIPM (Delta form only): 1 skips the second product of chunks whose
+// rectified tile is zero (a vote of the epilogue warps); 2 skips both
+// products of the chunks that the range-search mask clears.  Separate
+// instantiations, so that the kernel without them carries none of the checks.
+template <int RP, int EPI, bool SPLIT, bool LOSS, int SKIPM>
 __global__ void __launch_bounds__(kThreads, 1)
     panel_tc_kernel(const __grid_constant__ CUtensorMap tq_hi, const __grid_constant__ CUtensorMap tq_lo,
                     const __grid_constant__ CUtensorMap tq_lo2, const __grid_constant__ CUtensorMap tw,
                     const TcParams p) {
   using C = Cfg<RP, SPLIT, LOSS>;
   constexpr int BN = C::BN, NB = C::NB, NSTAGE = C::NSTAGE, NWB = C::NWB;
+  constexpr bool VOTE = SKIPM == 1, RANGE = SKIPM == 2;
+  static_assert(SKIPM == 0 || (EPI == 1 && !LOSS), "skipping is a Delta-form option");
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
   uint8_t* stages = smem;
@@ -262,6 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int64_t kK = p.ksplit ? (p.K - kz * p.ksplit < p.ksplit ? p.K - kz * p.ksplit : p.ksplit) : p.K;
   float* const Rout = p.ksplit ? p.R + kz * p.rstride : p.R;
   const int64_t nchunks = (kK + BN - 1) / BN;
+  const int64_t kc0 = (kq0 - p.q0) / BN;   // this CTA's first chunk within the tile's mask
 
   if (warp == kProducerWarp) {
     // ------------------------------------------------------------ producer
@@ -279,7 +340,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_2d(wsm0 + wb * C::W_BYTES + pn * C::W_PANEL_BYTES, &tw, b_wfull + 8 * wb, pn * C::PANEL_W,
                         (int)(p.m0 + t * BM));
         }
-        for (int64_t c = 0; c < nchunks; ++c, ++G) {
+        int64_t clast, nlive;
+        const ChunkMask cm = chunk_mask<RANGE>(p, t, kc0, nchunks, &clast, &nlive);
+        for (int64_t c = 0; c < nchunks; ++c) {
+          if (RANGE && !cm.live(c)) continue;
           const int s = (int)(G % NSTAGE);
           if (!(ok = wait_bar(b_empty + 8 * s, (uint32_t)((G / NSTAGE) & 1) ^ 1u, abort_flag, p.status, 1)))
             break;
@@ -295,6 +359,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               tma_load_2d(dst + 2 * C::OPER_BYTES + pn * C::PANEL_BYTES, &tq_lo2, b_full + 8 * s, pn * C::PANEL_W,
                           y);
           }
+          ++G;
         }
       }
       if (!ok) {  // drain the copies still in flight before shared memory goes away
@@ -318,48 +383,51 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ------------------------------------------------------------ MMA1 issuer
     // L[lb] = W tile x chunk^T for every chunk G of this CTA's tiles, in order.
     constexpr uint32_t idesc1 = idesc_bf16(BM, BN, false);   // Q K-major
-    const int64_t my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
-    const int64_t total = my_tiles * nchunks;
     const uint32_t stage0 = smem_u32(stages);
     int s1 = 0, l1 = 0, wb1 = 0;
     uint32_t ph_full = 0, ph_lfree = 1, ph_wfull = 0;
-    int64_t c1 = 0;
     bool ok = true;
-    for (int64_t G = 0; G < total && ok; ++G) {
-      if (c1 == 0 && !(ok = conv_wait(b_wfull + 8 * wb1, ph_wfull, abort_flag, p.status, 2))) break;
-      if (!(ok = conv_wait(b_full + 8 * s1, ph_full, abort_flag, p.status, 3))) break;
-      if (!(ok = conv_wait(b_lfree + 8 * l1, ph_lfree, abort_flag, p.status, 4))) break;
-      fence_after();
-      const uint32_t wh = tmem + C::COL_W + wb1 * C::WCOLS;
-      const uint32_t wl = wh + RP / 2;
-      const uint64_t d1 = sdesc(stage0 + s1 * C::STAGE_BYTES, 16, 8 * C::ROWB, C::SWZ);
-      // WSMEM: the W tile in the same K-major swizzled panels as a chunk
-      const uint64_t a1 = sdesc(wsm0 + wb1 * C::W_BYTES, 16, 8 * C::ROWB, C::SWZ);
-      const uint32_t d = tmem + C::COL_L + l1 * BN;
+    for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+      int64_t clast, nlive;
+      const ChunkMask cm = chunk_mask<RANGE>(p, t, kc0, nchunks, &clast, &nlive);
+      if (RANGE && p.skips != nullptr && lane == 0 && nlive < nchunks)
+        atomicAdd(p.skips, (unsigned long long)(nchunks - nlive));
+      bool first = true;
+      for (int64_t c = 0; c < nchunks; ++c) {
+        if (RANGE && !cm.live(c)) continue;
+        if (first && !(ok = conv_wait(b_wfull + 8 * wb1, ph_wfull, abort_flag, p.status, 2))) break;
+        first = false;
+        if (!(ok = conv_wait(b_full + 8 * s1, ph_full, abort_flag, p.status, 3))) break;
+        if (!(ok = conv_wait(b_lfree + 8 * l1, ph_lfree, abort_flag, p.status, 4))) break;
+        fence_after();
+        const uint32_t wh = tmem + C::COL_W + wb1 * C::WCOLS;
+        const uint32_t wl = wh + RP / 2;
+        const uint64_t d1 = sdesc(stage0 + s1 * C::STAGE_BYTES, 16, 8 * C::ROWB, C::SWZ);
+        // WSMEM: the W tile in the same K-major swizzled panels as a chunk
+        const uint64_t a1 = sdesc(wsm0 + wb1 * C::W_BYTES, 16, 8 * C::ROWB, C::SWZ);
+        const uint32_t d = tmem + C::COL_L + l1 * BN;
 #pragma unroll
-      for (int k = 0; k < RP / 16; ++k) {
-        const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
-        const uint64_t bh = d1 + (off >> 4);
-        if (C::WSMEM)
-          mma_ss_elect(d, a1 + (((k * 16 / C::PANEL_W) * C::W_PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2) >> 4), bh,
-                       idesc1, k > 0);
-        else
-          mma_ts_elect(d, wh + k * 8, bh, idesc1, k > 0);
-        if (SPLIT) {
-          const uint64_t bl = d1 + ((C::OPER_BYTES + off) >> 4);
-          mma_ts_elect(d, wh + k * 8, bl, idesc1, 1);
-          mma_ts_elect(d, wl + k * 8, bh, idesc1, 1);
+        for (int k = 0; k < RP / 16; ++k) {
+          const uint32_t off = (k * 16 / C::PANEL_W) * C::PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2;
+          const uint64_t bh = d1 + (off >> 4);
+          if (C::WSMEM)
+            mma_ss_elect(d, a1 + (((k * 16 / C::PANEL_W) * C::W_PANEL_BYTES + ((k * 16) % C::PANEL_W) * 2) >> 4), bh,
+                         idesc1, k > 0);
+          else
+            mma_ts_elect(d, wh + k * 8, bh, idesc1, k > 0);
+          if (SPLIT) {
+            const uint64_t bl = d1 + ((C::OPER_BYTES + off) >> 4);
+            mma_ts_elect(d, wh + k * 8, bl, idesc1, 1);
+            mma_ts_elect(d, wl + k * 8, bh, idesc1, 1);
+          }
         }
+        commit_elect(b_lfull + 8 * l1);
+        if (LOSS) commit_elect(b_empty + 8 * s1);
+        if (c == clast) commit_elect(b_wempty + 8 * wb1);
+        if (++s1 == NSTAGE) { s1 = 0; ph_full ^= 1u; }
+        if (++l1 == NB) { l1 = 0; ph_lfree ^= 1u; }
       }
-      commit_elect(b_lfull + 8 * l1);
-      if (LOSS) commit_elect(b_empty + 8 * s1);
-      if (c1 == nchunks - 1) commit_elect(b_wempty + 8 * wb1);
-      if (++s1 == NSTAGE) { s1 = 0; ph_full ^= 1u; }
-      if (++l1 == NB) { l1 = 0; ph_lfree ^= 1u; }
-      if (++c1 == nchunks) {
-        c1 = 0;
-        if (++wb1 == NWB) { wb1 = 0; ph_wfull ^= 1u; }
-      }
+      if (++wb1 == NWB) { wb1 = 0; ph_wfull ^= 1u; }
     }
     // wait until every MMA issued by this warp has completed
     commit_elect(b_drain);
@@ -377,50 +445,52 @@ __global__ void __launch_bounds__(kThreads, 1)
       constexpr uint32_t idesc2 = idesc_bf16(BM, C::NR, true, EPI == 1 && !SPLIT);   // Q MN-major
       // R columns [hcol, hcol + NR) of Q: their panels start hcol / PANEL_W panels in
       const uint32_t hpan = C::RHALF ? (uint32_t)blockIdx.y * (C::NR / C::PANEL_W) * C::PANEL_BYTES : 0u;
-      const int64_t my_tiles = blockIdx.x < ntiles ? (ntiles - 1 - blockIdx.x) / gridDim.x + 1 : 0;
-      const int64_t total = my_tiles * nchunks;
       const uint32_t stage0 = smem_u32(stages);
       int s2 = 0, l2 = 0;
       uint32_t ph_pfull = 0, ph_rempty = 1;
-      int64_t c2 = 0;
       bool ok = true;
-      for (int64_t D = 0; D < total && ok; ++D) {
-        if (!(ok = conv_wait(b_pfull + 8 * l2, ph_pfull, abort_flag, p.status, 5))) break;
-        if (c2 == 0 && !(ok = conv_wait(b_rempty, ph_rempty, abort_flag, p.status, 6))) break;
-        fence_after();
-        // Delta form: a chunk whose P is zero in every row adds nothing to R
-        // (Sec. 4.3); its MMAs are skipped, except for the first chunk of a
-        // tile, which initialises the accumulator
-        bool skip = false;
-        static_assert(!SKIP || (EPI == 1 && !LOSS), "skipping is a Delta-form option");
-        if (SKIP && c2 > 0)
-          skip = (pflag[4 * l2] | pflag[4 * l2 + 1] | pflag[4 * l2 + 2] | pflag[4 * l2 + 3]) == 0u;
-        if (skip && p.skips != nullptr && lane == 0) atomicAdd(p.skips, 1ull);
-        const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES + hpan, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
-        const uint32_t pl = tmem + C::COL_L + l2 * BN;
+      for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+        int64_t clast, nlive;
+        const ChunkMask cm = chunk_mask<RANGE>(p, t, kc0, nchunks, &clast, &nlive);
+        bool first = true;
+        for (int64_t c = 0; c < nchunks; ++c) {
+          if (RANGE && !cm.live(c)) continue;
+          if (!(ok = conv_wait(b_pfull + 8 * l2, ph_pfull, abort_flag, p.status, 5))) break;
+          if (first && !(ok = conv_wait(b_rempty, ph_rempty, abort_flag, p.status, 6))) break;
+          fence_after();
+          // Delta form: a chunk whose P is zero in every row adds nothing to R
+          // (Sec. 4.3); its MMAs are skipped, except for the first chunk of a
+          // tile, which initialises the accumulator
+          bool skip = false;
+          if (VOTE && !first)
+            skip = (pflag[4 * l2] | pflag[4 * l2 + 1] | pflag[4 * l2 + 2] | pflag[4 * l2 + 3]) == 0u;
+          if (VOTE && skip && p.skips != nullptr && lane == 0) atomicAdd(p.skips, 1ull);
+          const uint64_t d2 = sdesc(stage0 + s2 * C::STAGE_BYTES + hpan, C::PANEL_BYTES, 8 * C::ROWB, C::SWZ);
+          const uint32_t pl = tmem + C::COL_L + l2 * BN;
 #pragma unroll
-        for (int k = 0; k < BN / 16 && !(SKIP && skip); ++k) {
-          const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
-          const uint32_t acc = (c2 > 0 || k > 0) ? 1u : 0u;
-          if (!SPLIT) {             // P q_hi
-            mma_ts_elect(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
-          } else {                  // P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
-            const uint64_t bl = bh + (C::OPER_BYTES >> 4);
-            const uint64_t bl2 = bh + ((2 * C::OPER_BYTES) >> 4);
-            const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
-            mma_ts_elect(tmem + C::COL_R, ph, bh, idesc2, acc);
-            mma_ts_elect(tmem + C::COL_R, ph, bl, idesc2, 1);
-            mma_ts_elect(tmem + C::COL_R, ph, bl2, idesc2, 1);
-            mma_ts_elect(tmem + C::COL_R, plo, bh, idesc2, 1);
+          for (int k = 0; k < BN / 16 && !(VOTE && skip); ++k) {
+            const uint64_t bh = d2 + ((k * 16 * C::ROWB) >> 4);
+            const uint32_t acc = (!first || k > 0) ? 1u : 0u;
+            if (!SPLIT) {             // P q_hi
+              mma_ts_elect(tmem + C::COL_R, pl + k * 8, bh, idesc2, acc);
+            } else {                  // P_hi (q_hi + q_lo + q_lo2) + P_lo q_hi
+              const uint64_t bl = bh + (C::OPER_BYTES >> 4);
+              const uint64_t bl2 = bh + ((2 * C::OPER_BYTES) >> 4);
+              const uint32_t ph = pl + (k / 2) * 32 + (k % 2) * 8, plo = ph + 16;
+              mma_ts_elect(tmem + C::COL_R, ph, bh, idesc2, acc);
+              mma_ts_elect(tmem + C::COL_R, ph, bl, idesc2, 1);
+              mma_ts_elect(tmem + C::COL_R, ph, bl2, idesc2, 1);
+              mma_ts_elect(tmem + C::COL_R, plo, bh, idesc2, 1);
+            }
           }
+          commit_elect(b_empty + 8 * s2);
+          commit_elect(b_lfree + 8 * l2);
+          if (c == clast) commit_elect(b_rfull);
+          if (++s2 == NSTAGE) s2 = 0;
+          if (++l2 == NB) { l2 = 0; ph_pfull ^= 1u; }
+          if (first) ph_rempty ^= 1u;
+          first = false;
         }
-        commit_elect(b_empty + 8 * s2);
-        commit_elect(b_lfree + 8 * l2);
-        if (c2 == nchunks - 1) commit_elect(b_rfull);
-        if (++s2 == NSTAGE) s2 = 0;
-        if (++l2 == NB) { l2 = 0; ph_pfull ^= 1u; }
-        if (c2 == 0) ph_rempty ^= 1u;
-        if (++c2 == nchunks) c2 = 0;
       }
       commit_elect(b_drain2);
       if (lane == 0) {
@@ -478,7 +548,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int64_t t = blockIdx.x; t < ntiles && tt < NWB; t += gridDim.x, ++tt) load_w(t, (int)tt);
     }
     int64_t tt = 0;
+    int64_t Gc = 0;   // chunks this CTA has processed
     for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++tt) {
+      int64_t clast, nlive;
+      const ChunkMask cm = chunk_mask<RANGE>(p, t, kc0, nchunks, &clast, &nlive);
       if (LOSS) {
         const int64_t li = t * BM + row;
         se = li < p.M ? p.rowptr[li] : 0;
@@ -486,7 +559,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         snext = se < send ? p.cidx[se] : INT64_MAX;
       }
       for (int64_t c = 0; c < nchunks; ++c) {
-        const int64_t G = tt * nchunks + c;
+        if (RANGE && !cm.live(c)) continue;
+        const int64_t G = Gc++;
         if ((int)(G & 1) != wg) continue;
         if (LOSS) {   // skip the support columns of the other warpgroup's chunks
           while (snext < c * BN) {
@@ -546,7 +620,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 pk[i] = min0_bf16x2(pack_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1])));
               } else {          // max(0, L); the MMA negates it
                 pk[i] = pack_relu_bf16x2(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-                if (SKIP) nzacc |= pk[i] & 0x7fff7fffu;   // -0 counts as zero
+                if (VOTE) nzacc |= pk[i] & 0x7fff7fffu;   // -0 counts as zero
               }
             }
             tmem_st16(lcol + g * 16, pk);
@@ -562,7 +636,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               const float h0 = __uint_as_float(hp << 16), h1 = __uint_as_float(hp & 0xffff0000u);
               ph[i] = hp;
               pl[i] = pack_bf16x2(e0 - h0, e1 - h1);
-              if (SKIP) nzacc |= (ph[i] | pl[i]) & 0x7fff7fffu;   // -0 counts as zero
+              if (VOTE) nzacc |= (ph[i] | pl[i]) & 0x7fff7fffu;   // -0 counts as zero
             }
             tmem_st16(lcol + g * 32, ph);
             tmem_st16(lcol + g * 32 + 16, pl);
@@ -591,7 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(b_lfree + 8 * lb);
         } else {
-          if (SKIP) {   // published before the arrive (release) that MMA2 acquires
+          if (VOTE) {   // published before the arrive (release) that MMA2 acquires
             const bool nz = __any_sync(0xffffffffu, nzacc != 0u);
             if (lane == 0) pflag[4 * lb + (warp & 3)] = nz ? 1u : 0u;
           }
@@ -729,7 +803,7 @@ bool tensor_map(const bf16* base, int64_t rows, int rp, int panel_w, int bn, CUt
   return true;
 }
 
-template <int RP, int EPI, bool SPLIT, bool LOSS, bool SKIP = false>
+template <int RP, int EPI, bool SPLIT, bool LOSS, int SKIPM = 0>
 nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, cudaStream_t s) {
   using C = Cfg<RP, SPLIT, LOSS>;
   CUtensorMap th, tl, tl2;
@@ -743,12 +817,12 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
   // the shared-memory attribute belongs to the current device
   static std::atomic<int> attr_set[kMaxDevices];
   if (!per_device(attr_set, [] {
-        return cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP>,
+        return cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIPM>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) == cudaSuccess ? 1 : 0;
       }))
     return NMD_ERR_CUDA;
   const unsigned gz = p.ksplit ? (unsigned)((p.K + p.ksplit - 1) / p.ksplit) : 1u;
-  panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIP><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u, gz), kThreads, C::SMEM, s>>>(
+  panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIPM><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u, gz), kThreads, C::SMEM, s>>>(
       th, tl, tl2, tw, p);
   return NMD_OK;
 }
@@ -757,9 +831,13 @@ template <int RP, bool LOSS>
 nmd_status dispatch_rp(int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p, int grid,
                        cudaStream_t s) {
   if (LOSS) return split ? run<RP, 0, true, LOSS>(fm, fq, p, grid, s) : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
+  if (epilogue == NMD_EPI_DELTA && p.rmask != nullptr) {
+    if (split) return run<RP, 1, true, false, 2>(fm, fq, p, grid, s);
+    return run<RP, 1, false, false, 2>(fm, fq, p, grid, s);
+  }
   if (epilogue == NMD_EPI_DELTA && p.skip_on) {
-    if (split) return run<RP, 1, true, false, true>(fm, fq, p, grid, s);
-    return run<RP, 1, false, false, true>(fm, fq, p, grid, s);
+    if (split) return run<RP, 1, true, false, 1>(fm, fq, p, grid, s);
+    return run<RP, 1, false, false, 1>(fm, fq, p, grid, s);
   }
   if (split)
     return epilogue == NMD_EPI_DELTA ? run<RP, 1, true, LOSS>(fm, fq, p, grid, s)
@@ -783,6 +861,17 @@ nmd_status dispatch(int rp, int epilogue, bool split, const Factor& fm, const Fa
 
 }  // namespace
 
+int panel_chunk_rows(int rp, int precision) {
+  const bool split = precision == NMD_FP32;
+  switch (rp) {
+    case 16: return split ? Cfg<16, true, false>::BN : Cfg<16, false, false>::BN;
+    case 32: return split ? Cfg<32, true, false>::BN : Cfg<32, false, false>::BN;
+    case 64: return split ? Cfg<64, true, false>::BN : Cfg<64, false, false>::BN;
+    case 128: return split ? Cfg<128, true, false>::BN : Cfg<128, false, false>::BN;
+    default: return split ? Cfg<256, true, false>::BN : Cfg<256, false, false>::BN;
+  }
+}
+
 bool tc_supported(int rp, int precision) {
   if (precision == NMD_SIMT) return false;
   return rp == 16 || rp == 32 || rp == 64 || rp == 128 || rp == 256;
@@ -802,7 +891,7 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
                            int64_t* launches, float* Lout, float* rpart, int64_t rpart_rows) {
   if (!tc_supported(a.rp, a.precision)) return NMD_ERR_UNSUPPORTED;
   TcParams p{a.m0, a.M, a.q0, a.K, a.fm->hi, a.fm->lo, R, nullptr, status, Lout, nullptr, nullptr,
-             (unsigned long long*)counter, a.skip_zero ? 1 : 0, 0, 0};
+             (unsigned long long*)counter, a.skip_zero ? 1 : 0, 0, 0, a.rmask, a.rwords};
   const int64_t ntiles = (a.M + BM - 1) / BM;
   // a step with fewer tiles than SMs (the exact steps: b rows against all of
   // the other factor) splits K so that tiles x splits fill the SMs, each split

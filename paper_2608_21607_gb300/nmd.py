@@ -24,6 +24,7 @@ NMD_ALTERNATE, NMD_PHASED = 0, 1
 NMD_BF16, NMD_FP32, NMD_SIMT = 0, 1, 2
 NMD_EPI_Z, NMD_EPI_DELTA = 0, 1
 NMD_K_DENSE, NMD_K_SPARSE, NMD_K_GRAM, NMD_K_UPDATE, NMD_K_LOSS = 0, 1, 2, 3, 4
+NMD_SKIP_NONE, NMD_SKIP_VOTE, NMD_SKIP_RANGE = 0, 1, 2
 
 # every symbol include/nmd.h declares
 EXPORTS = [
@@ -31,7 +32,7 @@ EXPORTS = [
     "nmd_get_factors", "nmd_block_update", "nmd_sweep", "nmd_block_order", "nmd_loss", "nmd_sync",
     "nmd_block_terms", "nmd_dense_products", "nmd_panel_traversal", "nmd_get_state", "nmd_set_state",
     "nmd_launch_count", "nmd_skip_count", "nmd_selftest_wait_timeout", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
-    "nmd_destroy", "nmd_gram_noalloc", "nmd_support_term", "nmd_block_update_combined",
+    "nmd_destroy", "nmd_gram_noalloc", "nmd_support_term", "nmd_block_update_combined", "nmd_range_mask",
 ]
 
 
@@ -97,6 +98,8 @@ def lib() -> C.CDLL:
             "nmd_gram_noalloc": (C.c_int, [_P, C.c_int64, C.c_int32, C.c_int64, _P, _P]),
             "nmd_support_term": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int32, _P, _i64p]),
             "nmd_block_update_combined": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int64]),
+            "nmd_range_mask": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int32, _P, C.c_int64, _i64p, _i64p,
+                                         _i64p]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -232,6 +235,19 @@ def nmd_support_term(h, side, block, kind, d_R) -> int:
     return rows.value
 
 
+def nmd_range_mask(h, side, block, kind):
+    """(mask, chunk_rows): mask[t, w] = word w of 128-row M tile t, bit c set =
+    Q chunk 32 w + c cleared by the range search."""
+    nt, nw, cr = C.c_int64(0), C.c_int64(0), C.c_int64(0)
+    L = lib()
+    _check(h, L.nmd_range_mask(h, side, block, kind, None, 0, C.byref(nt), C.byref(nw), C.byref(cr)),
+           "nmd_range_mask")
+    mask = np.zeros((nt.value, nw.value), dtype=np.uint32)
+    _check(h, L.nmd_range_mask(h, side, block, kind, mask.ctypes.data, mask.size, C.byref(nt), C.byref(nw),
+                               C.byref(cr)), "nmd_range_mask")
+    return mask, cr.value
+
+
 def nmd_get_state(h, m, n, r):
     W = np.zeros((m, r), np.float32); H = np.zeros((r, n), np.float32)
     EW = np.zeros((m, r), np.float32); EH = np.zeros((r, n), np.float32)
@@ -304,7 +320,7 @@ class Solver:
         o.schedule, o.order = int(schedule), int(order)
         o.eta, o.gamma, o.ridge = float(eta), float(gamma), float(ridge)
         o.precision, o.epilogue, o.seed = int(precision), int(epilogue), int(seed)
-        o.skip_zero_chunks = 1 if skip_zero_chunks else 0
+        o.skip_zero_chunks = int(skip_zero_chunks)   # False/True or an NMD_SKIP_* mode
         self.opts = o
         self.device = torch.device(device) if device is not None else torch.device("cuda", torch.cuda.current_device())
         nbytes = nmd_workspace_bytes(S, self.r, o)
@@ -403,5 +419,10 @@ class Solver:
         return nmd_launch_count(self.h)
 
     def skip_count(self, reset: bool = False) -> int:
-        """Delta form: chunks whose second product was skipped (all-zero P)."""
+        """Delta form: chunks skipped (NMD_SKIP_VOTE: second product of an
+        all-zero P; NMD_SKIP_RANGE: both products of a cleared chunk)."""
         return nmd_skip_count(self.h, reset)
+
+    def range_mask(self, side, block, kind):
+        """The range-search mask of one block update and its chunk size."""
+        return nmd_range_mask(self.h, side, block, kind)

@@ -152,6 +152,62 @@ def planted(m: int = 600, n: int = 400, d: int = 4, tau: Optional[float] = 0.5,
     return S, U, V, tau
 
 
+def community_of(N: int, clusters: int, run: Optional[int] = None) -> np.ndarray:
+    """Community of each of N indices: contiguous ranges (run None), or runs
+    of `run` consecutive indices taking the communities in turn."""
+    if run is None:
+        return (np.arange(N) * clusters) // N
+    return (np.arange(N) // run) % clusters
+
+
+def community_factors(m: int, n: int, r: int, clusters: int, noise: float = 0.01, neg: float = 0.6,
+                      seed: int = 0, run: Optional[int] = None):
+    """W (m x r) and H (r x n), float32, whose rows fall into `clusters` tight
+    groups of directions (communities by community_of): row i of W points
+    along e_c of its community c, column j of H along 2 e_d - neg (the
+    all-ones vector on the first `clusters` coordinates) of its community d,
+    each with iid N(0, noise^2) added and a length drawn from U(0.5, 2).
+    W_i . H_j is about (2 - neg) times the lengths within a community and
+    about -neg times them across: the rectified product max(0, W H) is block
+    diagonal up to the ordering.  Needs r >= clusters.  Also returns the
+    communities of the rows of W and of the columns of H."""
+    if r < clusters:
+        raise ValueError("r must be at least the number of communities")
+    rng = np.random.default_rng([seed, 0xC0DE])
+    cw = community_of(m, clusters, run)
+    ch = community_of(n, clusters, run)
+    W = np.zeros((m, r))
+    W[np.arange(m), cw] = 1.0
+    H = np.zeros((n, r))
+    H[:, :clusters] = -neg
+    H[np.arange(n), ch] += 2.0
+    W += noise * rng.standard_normal((m, r))
+    H += noise * rng.standard_normal((n, r))
+    W *= rng.uniform(0.5, 2.0, (m, 1))
+    H *= rng.uniform(0.5, 2.0, (n, 1))
+    return W.astype(np.float32), np.ascontiguousarray(H.T).astype(np.float32), cw, ch
+
+
+def communities(m: int, n: int, clusters: int, mean_degree: float, seed: int = 0, run: Optional[int] = None,
+                dtype=np.float32) -> CSR:
+    """A stochastic block model: row i has Poisson(mean_degree) entries (at
+    most the size of its community), at columns drawn uniformly without
+    replacement from the columns of its own community (community_of), with
+    values ceil(exp(1 + N(0, 1))); no entry joins two communities."""
+    rng = np.random.default_rng([seed, 0x5B3])
+    cw = community_of(m, clusters, run)
+    ch = community_of(n, clusters, run)
+    members = [np.nonzero(ch == c)[0] for c in range(clusters)]
+    rows_cols, rows_vals = [], []
+    for i in range(m):
+        cols = members[cw[i]]
+        k = min(len(cols), rng.poisson(mean_degree))
+        c = np.sort(rng.choice(cols, size=k, replace=False)) if k else np.zeros(0, np.int64)
+        rows_cols.append(c)
+        rows_vals.append(np.ceil(np.exp(1.0 + rng.standard_normal(k))))
+    return _csr_from_rows(m, n, rows_cols, rows_vals, dtype)
+
+
 def identity(n: int = 4096, dtype=np.float32) -> CSR:
     """S = I_n in CSR (n nonzeros of value 1)."""
     return CSR(n, n, np.arange(n + 1, dtype=np.int64), np.arange(n, dtype=np.int32),
@@ -255,6 +311,40 @@ def _connectome(seed=0, n=139255, r=64, block=4096, sweeps=10, mean_degree=20.0,
                     0.5, 0.9, seed, {"mean_degree": mean_degree})
 
 
+def _communities(seed=0, n=139255, r=64, block=8192, clusters=64, run=128, **kw):
+    # runs of 128 indices per community, taken in turn: every 128-row tile and
+    # 128-row chunk lies in one community, and every block of 8192 holds all
+    # 64 communities (so that its Gram matrix has full rank)
+    S = communities(n, n, clusters, 20.0, seed=seed, run=run)
+    W, H, _, _ = community_factors(n, n, r, clusters, seed=seed, run=run)
+    return Workload("communities-%d-r%d-c%d" % (n, r, clusters), S, r, W, H, block, block, "stoch", 10,
+                    0.5, 0.9, seed, {"clusters": clusters, "run": run, "mean_degree": 20.0})
+
+
+def _communities_planted(seed=0, n=40960, r=64, block=8192, clusters=64, run=128, **kw):
+    # S = max(0, W H) of clustered factors: a zero-loss fixed point whose
+    # rectified product is block diagonal, so that the factors stay clustered.
+    # With 64 communities in 64 dimensions the cosine across communities is
+    # only about -1/8, so the groups must be tight (noise 0.002) for the
+    # range search to separate them.
+    W, H, _, _ = community_factors(n, n, r, clusters, noise=0.002, seed=seed, run=run)
+    rows_cols, rows_vals = [], []
+    Hd = H.astype(np.float64)
+    for r0 in range(0, n, 2048):
+        L = W[r0:r0 + 2048].astype(np.float64) @ Hd
+        for row in L:
+            c = np.nonzero(row > 0)[0]
+            rows_cols.append(c)
+            rows_vals.append(row[c])
+    S = _csr_from_rows(n, n, rows_cols, rows_vals, np.float32)
+    # no momentum: in the bf16 mode the rounding of the operands moves the
+    # factors off the planted point a little every sweep (objective about
+    # 2e-3), and momentum 0.9 keeps amplifying that drift until a block Gram
+    # matrix loses rank after several sweeps; with gamma = 0 it settles
+    return Workload("communities-planted-%d-r%d-c%d" % (n, r, clusters), S, r, W, H, block, block, "stoch", 10,
+                    0.5, 0.0, seed, {"clusters": clusters, "run": run})
+
+
 WORKLOADS = {
     "planted_tiny": _planted_tiny,
     "identity": _identity,
@@ -265,6 +355,10 @@ WORKLOADS = {
     # (rho+ = 0.00102 of the n^2 entries: mean out-degree 142, ~19.8M nonzeros)
     "connectome_dense_r64": lambda seed=0, **kw: _connectome(seed, r=64, block=4096, sweeps=10,
                                                              mean_degree=0.00102 * 139254, tag="-dense", **kw),
+    # a block-structured graph started from factors whose rows cluster by
+    # community (the situation of Sec. 4.3 in which max(0, W H) is sparse)
+    "communities_r64": _communities,
+    "communities_planted_r64": _communities_planted,
 }
 
 

@@ -498,3 +498,35 @@ def test_stochastic_sweep_decreases_loss_on_planted():
     for _ in range(10):
         st.sweep()
     assert st.loss()["obj"] < 0.5 * l0
+
+
+def test_range_search_set_hand_examples():
+    """Eq. range-search on pairs worked out by hand: L > 0 exactly when the
+    normalised rows are less than sqrt(2) apart; an orthogonal pair sits at
+    squared distance exactly 2 (L = 0: not in Omega); a zero row is in no
+    pair."""
+    A = np.array([[3.0, 4.0, 0.0], [1.0, 0.0, 0.0], [2.0, 0.0, 0.0], [0.0, 0.0, 0.0]])
+    B = np.array([[4.0, 3.0, 0.0], [0.0, 0.0, 5.0], [-1.0, -1.0, 0.0]])
+    # (0,0): L = 24, |a^ - b^|^2 = 0.08; (1,1): L = 0, distance^2 = 2; (2,2): L = -2,
+    # distance^2 = 2 + sqrt(2); row 3 is zero
+    want = np.array([[1, 0, 0], [1, 0, 0], [1, 0, 0], [0, 0, 0]], dtype=bool)
+    np.testing.assert_array_equal(O.range_search_set(A, B), want)
+    np.testing.assert_array_equal(O.positive_set(A, B), want)
+
+
+def test_range_search_set_equals_positive_set():
+    """Eq. nonzeros and eq. range-search define the same set (Sec. 4.3), on
+    random factors with zero rows and with rows of very different lengths."""
+    rng = np.random.default_rng(4)
+    A = rng.standard_normal((30, 5)) * rng.uniform(0.01, 100.0, (30, 1))
+    B = rng.standard_normal((40, 5)) * rng.uniform(0.01, 100.0, (40, 1))
+    A[[3, 17]] = 0.0
+    B[[0, 25, 39]] = 0.0
+    got = O.range_search_set(A, B)
+    want = np.zeros((30, 40), dtype=bool)
+    for i in range(30):
+        for j in range(40):
+            want[i, j] = sum(A[i, k] * B[j, k] for k in range(5)) > 0
+    np.testing.assert_array_equal(got, want)
+    np.testing.assert_array_equal(O.positive_set(A, B), want)
+    assert 0 < want.sum() < want.size
