@@ -8,3 +8,4 @@ from .salsa import (ROW, COL, EXACT, STOCH, ALTERNATE, PHASED, NotSPD, Options, 
                     Sparse, block_permutation, block_range, num_blocks, cholesky,
                     solve_normal, update_z, loss, splitmix64_mix, SplitMix64,
                     positive_set, range_search_set)
+from . import embed  # noqa: F401,E402  (Sec. 5.3: cell embedding and 1-NN error)
