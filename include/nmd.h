@@ -337,6 +337,38 @@ nmd_status nmd_skip_count(nmd_handle* h, int64_t* skipped, int32_t reset);
 nmd_status nmd_range_mask(nmd_handle* h, int32_t side, int64_t block, int32_t kind, uint32_t* mask,
                           int64_t capacity, int64_t* ntiles, int64_t* words, int64_t* chunk_rows);
 
+/* Cell embedding (Sec. 5.3, eqs. Lsvd and embed), for a square S (m = n:
+ * rows and columns are the same cells) and r <= 128: with the model
+ * L = W H = U Sigma V^T (its thin SVD, computed from the factors without
+ * forming L), cell i is the unit vector
+ *     xi_i = [u_i Sigma^{1/2}, v_i Sigma^{1/2}] / norm
+ * of 2r elements (u_i, v_i the i-th rows of U and V; singular triples in
+ * descending order; a triple is determined up to a common sign, which the
+ * distances between cells do not see).  d_xi: device, n x 2r fp32 row-major,
+ * caller-owned.  d_sigma: device, r fp32 (the singular values, descending) or
+ * NULL.  Asynchronous on the handle's stream.  NMD_ERR_INVALID if m != n,
+ * r > 128 or n < 6 r. */
+nmd_status nmd_embed(nmd_handle* h, float* d_xi, float* d_sigma);
+
+/* Device workspace (bytes) of nmd_nearest_neighbors for N points of d
+ * coordinates (2 <= N < 2^31, 1 <= d <= 256). */
+nmd_status nmd_nn_workspace_bytes(int64_t N, int32_t d, size_t* bytes);
+
+/* Held-out one-nearest-neighbour search (Sec. 5.3): for each of the N points
+ * (rows of d_x, N x d fp32 row-major, device), the other point j != i with the
+ * largest inner product x_i . x_j -- for the unit vectors of nmd_embed the
+ * nearest in Euclidean distance -- on the tensor cores (each coordinate as
+ * three bf16 pieces, products accumulated in fp32: inner products good to
+ * about 1e-5 of |x_i| |x_j|; ties and near-ties within that go to either
+ * point, among exactly equal values to the smaller index).  d_nn: device,
+ * N int32 (the neighbour); d_best: device, N fp32 (its inner product) or
+ * NULL.  d_labels: device, N int32, or NULL; with labels and errors != NULL,
+ * *errors = the number of points whose neighbour carries another label (the
+ * 1-NN error count).  d_workspace: at least nmd_nn_workspace_bytes, 256-byte
+ * aligned, caller-owned.  Synchronises the stream. */
+nmd_status nmd_nearest_neighbors(const float* d_x, int64_t N, int32_t d, const int32_t* d_labels, int32_t* d_nn,
+                                 float* d_best, int64_t* errors, void* d_workspace, size_t ws_bytes, void* stream);
+
 const char* nmd_status_string(nmd_status s);
 const char* nmd_last_error(const nmd_handle* h);
 void nmd_destroy(nmd_handle* h);

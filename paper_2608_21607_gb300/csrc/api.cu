@@ -1229,6 +1229,22 @@ nmd_status nmd_dense_products(nmd_handle* h, int32_t side, int64_t block, int32_
   return NMD_OK;
 }
 
+nmd_status nmd_embed(nmd_handle* h, float* d_xi, float* d_sigma) {
+  if (!h || !d_xi) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_embed");
+  if (h->m != h->n) return fail(h, NMD_ERR_INVALID, "the cell embedding needs a square matrix (m == n)");
+  if (h->r > embed_max_rank()) return fail(h, NMD_ERR_INVALID, "the cell embedding supports r <= 128");
+  DeviceScope dg(h);
+  nmd_status st = wait_all_pending(h);
+  if (st != NMD_OK) return st;
+  if ((int64_t)h->n * h->rp < 6 * (int64_t)h->r * h->r)   // the r x r work space lives in R
+    return fail(h, NMD_ERR_INVALID, "the cell embedding needs at least 6 r cells");
+  h->gpre.active = false;   // the Gram partials are overwritten
+  st = launch_embed(h->W, h->B, h->n, h->r, h->rp, h->ws.gram_part, h->ws.G, h->ws.G2, h->ws.R, h->ws.Gx,
+                    h->ws.Tm, d_sigma ? d_sigma : h->ws.Ginv2, d_xi, h->num_sms, h->stream, &h->launches);
+  if (st != NMD_OK) return fail(h, st, "cudaFuncSetAttribute(embed_rows_kernel)");
+  return after_launch(h, "embedding");
+}
+
 nmd_status nmd_range_mask(nmd_handle* h, int32_t side, int64_t block, int32_t kind, uint32_t* mask,
                           int64_t capacity, int64_t* ntiles, int64_t* words, int64_t* chunk_rows) {
   if (!h || !ntiles || !words || !chunk_rows) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_range_mask");

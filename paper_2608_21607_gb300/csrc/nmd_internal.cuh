@@ -280,6 +280,18 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
 nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts,
                                 int* status, cudaStream_t s, int64_t* launches);
 bool tc_supported(int rp, int precision);
+// The nearest-neighbour pass of the tensor-core kernel over one point set
+// (rows [0, N) of f, all three bf16 pieces packed): per row the largest
+// inner product with another row, as an orderable key (zeroed by the caller)
+nmd_status launch_nearest_tc(const Factor& f, int64_t N, int rp, unsigned long long* keys, int* status,
+                             int num_sms, cudaStream_t s);
+// The cell embedding (Sec. 5.3): G_A = W^T W and G_B = B^T B into GA, GB,
+// their eigendecompositions and the SVD of the r x r core (scratch: six
+// r x r matrices), T_A, T_B (r x r), sigma (r) and the n x 2r rows xi.
+int embed_max_rank();
+nmd_status launch_embed(const Factor& W, const Factor& B, int64_t n, int r, int rp, float* gram_part, float* GA,
+                        float* GB, float* scratch, float* TA, float* TB, float* sigma, float* xi, int num_sms,
+                        cudaStream_t s, int64_t* launches);
 // Q-side rows per chunk of the tensor-core dense kernel (64 or 128)
 int panel_chunk_rows(int rp, int precision);
 // balls of the 128-row M tiles of rows [m0, m0 + M) of Xm and of the bn-row

@@ -143,6 +143,10 @@ struct TcParams {
   // tile's rows (see range_mask_kernel); nullptr: no chunk is skipped
   const uint32_t* rmask;
   int64_t rwords;
+  // nearest-neighbour pass (M side = Q side = one point set): per row the
+  // largest L_ij over j != i, as an orderable key (value bits << 32 |
+  // ~j); the caller zeroes the keys
+  unsigned long long* nn_key;
 };
 
 __device__ __forceinline__ void record(int* status, int code, int detail) {
@@ -244,15 +248,20 @@ __device__ __forceinline__ ChunkMask chunk_mask(const TcParams& p, int64_t t, in
   return cm;
 }
 
+// MODE: 0 the panel contraction R = P(L) Q; 1 the loss pass (first product
+// only, sums of max(0, L)^2 and max(0, L) off the support); 2 the nearest-
+// neighbour pass (first product only, per row the largest L_ij, j != i).
 // SKIPM (Delta form only): 1 skips the second product of chunks whose
 // rectified tile is zero (a vote of the epilogue warps); 2 skips both
 // products of the chunks that the range-search mask clears.  Separate
 // instantiations, so that the kernel without them carries none of the checks.
-template <int RP, int EPI, bool SPLIT, bool LOSS, int SKIPM>
+template <int RP, int EPI, bool SPLIT, int MODE, int SKIPM>
 __global__ void __launch_bounds__(kThreads, 1)
     panel_tc_kernel(const __grid_constant__ CUtensorMap tq_hi, const __grid_constant__ CUtensorMap tq_lo,
                     const __grid_constant__ CUtensorMap tq_lo2, const __grid_constant__ CUtensorMap tw,
                     const TcParams p) {
+  constexpr bool LOSS = MODE != 0;     // the first product only
+  constexpr bool SUMS = MODE == 1, NEAREST = MODE == 2;
   using C = Cfg<RP, SPLIT, LOSS>;
   constexpr int BN = C::BN, NB = C::NB, NSTAGE = C::NSTAGE, NWB = C::NWB;
   constexpr bool VOTE = SKIPM == 1, RANGE = SKIPM == 2;
@@ -510,6 +519,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int et = threadIdx.x;                          // 0 .. 255
     const uint32_t lane_base = ((uint32_t)((warp & 3) * 32)) << 16;
     double s2 = 0.0, s1 = 0.0;
+    float nbest = -INFINITY;   // nearest-neighbour pass: this thread's best L of its row so far
+    int64_t nidx = -1;
     bool ok = true;
     // loss pass: this thread's row of S, walked alongside the column chunks so
     // that support entries are left to the support pass (no cancellation)
@@ -552,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     for (int64_t t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++tt) {
       int64_t clast, nlive;
       const ChunkMask cm = chunk_mask<RANGE>(p, t, kc0, nchunks, &clast, &nlive);
-      if (LOSS) {
+      if (SUMS) {
         const int64_t li = t * BM + row;
         se = li < p.M ? p.rowptr[li] : 0;
         send = li < p.M ? p.rowptr[li + 1] : 0;
@@ -562,7 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (RANGE && !cm.live(c)) continue;
         const int64_t G = Gc++;
         if ((int)(G & 1) != wg) continue;
-        if (LOSS) {   // skip the support columns of the other warpgroup's chunks
+        if (SUMS) {   // skip the support columns of the other warpgroup's chunks
           while (snext < c * BN) {
             ++se;
             snext = se < send ? p.cidx[se] : INT64_MAX;
@@ -583,7 +594,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (kv < BN) {   // last chunk: columns past the block end contribute nothing
 #pragma unroll
             for (int i = 0; i < 32; ++i)
-              if (g * 32 + i >= kv) v[i] = LOSS ? 0u : (EPI == 0 ? 0u : 0xff800000u);   // -inf -> relu 0
+              if (g * 32 + i >= kv) v[i] = SUMS ? 0u : (EPI == 0 ? 0u : 0xff800000u);   // -inf -> relu 0
           }
           if (p.Lout != nullptr) {
             const int64_t li = t * BM + row;
@@ -593,7 +604,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (g * 32 + i < kv) p.Lout[li * p.K + c * BN + g * 32 + i] = __uint_as_float(v[i]);
             }
           }
-          if (LOSS) {
+          if (NEAREST) {   // columns past the set or the row itself do not count
+            const int64_t cb = c * BN + g * 32, self = t * BM + row;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const float x = __uint_as_float(v[i]);
+              if (g * 32 + i < kv && cb + i != self && x > nbest) {
+                nbest = x;
+                nidx = cb + i;
+              }
+            }
+          } else if (SUMS) {
             const int64_t cb = c * BN + g * 32;
             if (snext < cb + 32) {   // support columns in this group: zero them
 #pragma unroll
@@ -659,8 +680,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           group(v0, BN / 32 - 1);
         }
         if (LOSS) {
-          s2 += (double)c2;
-          s1 += (double)c1;
+          if (SUMS) {
+            s2 += (double)c2;
+            s1 += (double)c1;
+          }
           fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(b_lfree + 8 * lb);
@@ -676,6 +699,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
       if (!ok) break;
+      if (NEAREST) {   // this warpgroup's best of the row; the two are merged by atomicMax
+        const int64_t li = t * BM + row;
+        if (li < p.M && nidx >= 0) {
+          const uint32_t b = __float_as_uint(nbest);
+          const uint32_t ord = (b & 0x80000000u) ? ~b : (b | 0x80000000u);   // float order as unsigned
+          atomicMax(p.nn_key + li, ((unsigned long long)ord << 32) | (unsigned long long)(~(uint32_t)nidx));
+        }
+        nbest = -INFINITY;
+        nidx = -1;
+      }
       if (!LOSS) {
         if (!(ok = warp_wait(b_rfull, (uint32_t)(tt & 1), abort_flag, p.status, 8))) break;
         fence_after();
@@ -718,7 +751,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         load_w(tn, wb);
       }
     }
-    if (LOSS) {
+    if (SUMS) {
       // fixed-order reduction over the 256 epilogue threads
       red[2 * et] = s2;
       red[2 * et + 1] = s1;
@@ -803,9 +836,9 @@ bool tensor_map(const bf16* base, int64_t rows, int rp, int panel_w, int bn, CUt
   return true;
 }
 
-template <int RP, int EPI, bool SPLIT, bool LOSS, int SKIPM = 0>
+template <int RP, int EPI, bool SPLIT, int MODE, int SKIPM = 0>
 nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, cudaStream_t s) {
-  using C = Cfg<RP, SPLIT, LOSS>;
+  using C = Cfg<RP, SPLIT, MODE != 0>;
   CUtensorMap th, tl, tl2;
   if (!tensor_map(fq.hi, fq.rows, RP, C::PANEL_W, C::BN, &th)) return NMD_ERR_CUDA;
   if (!tensor_map(fq.lo, fq.rows, RP, C::PANEL_W, C::BN, &tl)) return NMD_ERR_CUDA;
@@ -817,44 +850,48 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
   // the shared-memory attribute belongs to the current device
   static std::atomic<int> attr_set[kMaxDevices];
   if (!per_device(attr_set, [] {
-        return cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIPM>,
+        return cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, MODE, SKIPM>,
                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) == cudaSuccess ? 1 : 0;
       }))
     return NMD_ERR_CUDA;
   const unsigned gz = p.ksplit ? (unsigned)((p.K + p.ksplit - 1) / p.ksplit) : 1u;
-  panel_tc_kernel<RP, EPI, SPLIT, LOSS, SKIPM><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u, gz), kThreads, C::SMEM, s>>>(
+  panel_tc_kernel<RP, EPI, SPLIT, MODE, SKIPM><<<dim3((unsigned)grid, C::RHALF ? 2u : 1u, gz), kThreads, C::SMEM, s>>>(
       th, tl, tl2, tw, p);
   return NMD_OK;
 }
 
-template <int RP, bool LOSS>
+template <int RP, int MODE>
 nmd_status dispatch_rp(int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p, int grid,
                        cudaStream_t s) {
-  if (LOSS) return split ? run<RP, 0, true, LOSS>(fm, fq, p, grid, s) : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
+  if constexpr (MODE == 2) {
+    return run<RP, 0, true, 2>(fm, fq, p, grid, s);   // nearest neighbours: always the split pieces
+  } else if constexpr (MODE == 1) {
+    return split ? run<RP, 0, true, 1>(fm, fq, p, grid, s) : run<RP, 0, false, 1>(fm, fq, p, grid, s);
+  }
   if (epilogue == NMD_EPI_DELTA && p.rmask != nullptr) {
-    if (split) return run<RP, 1, true, false, 2>(fm, fq, p, grid, s);
-    return run<RP, 1, false, false, 2>(fm, fq, p, grid, s);
+    if (split) return run<RP, 1, true, 0, 2>(fm, fq, p, grid, s);
+    return run<RP, 1, false, 0, 2>(fm, fq, p, grid, s);
   }
   if (epilogue == NMD_EPI_DELTA && p.skip_on) {
-    if (split) return run<RP, 1, true, false, 1>(fm, fq, p, grid, s);
-    return run<RP, 1, false, false, 1>(fm, fq, p, grid, s);
+    if (split) return run<RP, 1, true, 0, 1>(fm, fq, p, grid, s);
+    return run<RP, 1, false, 0, 1>(fm, fq, p, grid, s);
   }
   if (split)
-    return epilogue == NMD_EPI_DELTA ? run<RP, 1, true, LOSS>(fm, fq, p, grid, s)
-                                     : run<RP, 0, true, LOSS>(fm, fq, p, grid, s);
-  return epilogue == NMD_EPI_DELTA ? run<RP, 1, false, LOSS>(fm, fq, p, grid, s)
-                                   : run<RP, 0, false, LOSS>(fm, fq, p, grid, s);
+    return epilogue == NMD_EPI_DELTA ? run<RP, 1, true, 0>(fm, fq, p, grid, s)
+                                     : run<RP, 0, true, 0>(fm, fq, p, grid, s);
+  return epilogue == NMD_EPI_DELTA ? run<RP, 1, false, 0>(fm, fq, p, grid, s)
+                                   : run<RP, 0, false, 0>(fm, fq, p, grid, s);
 }
 
-template <bool LOSS>
+template <int MODE>
 nmd_status dispatch(int rp, int epilogue, bool split, const Factor& fm, const Factor& fq, const TcParams& p,
                     int grid, cudaStream_t s) {
   switch (rp) {
-    case 16: return dispatch_rp<16, LOSS>(epilogue, split, fm, fq, p, grid, s);
-    case 32: return dispatch_rp<32, LOSS>(epilogue, split, fm, fq, p, grid, s);
-    case 64: return dispatch_rp<64, LOSS>(epilogue, split, fm, fq, p, grid, s);
-    case 128: return dispatch_rp<128, LOSS>(epilogue, split, fm, fq, p, grid, s);
-    case 256: return dispatch_rp<256, LOSS>(epilogue, split, fm, fq, p, grid, s);
+    case 16: return dispatch_rp<16, MODE>(epilogue, split, fm, fq, p, grid, s);
+    case 32: return dispatch_rp<32, MODE>(epilogue, split, fm, fq, p, grid, s);
+    case 64: return dispatch_rp<64, MODE>(epilogue, split, fm, fq, p, grid, s);
+    case 128: return dispatch_rp<128, MODE>(epilogue, split, fm, fq, p, grid, s);
+    case 256: return dispatch_rp<256, MODE>(epilogue, split, fm, fq, p, grid, s);
   }
   return NMD_ERR_UNSUPPORTED;
 }
@@ -915,7 +952,7 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
     const int64_t rounds = (ntiles + num_sms - 1) / num_sms;
     grid = (int)((ntiles + rounds - 1) / rounds);
   }
-  nmd_status st = dispatch<false>(a.rp, a.epilogue, a.precision == NMD_FP32, *a.fm, *a.fq, p, grid, s);
+  nmd_status st = dispatch<0>(a.rp, a.epilogue, a.precision == NMD_FP32, *a.fm, *a.fq, p, grid, s);
   if (st != NMD_OK) return st;
   ++*launches;
   if (splits > 1) {
@@ -931,6 +968,17 @@ void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s) {
   wait_selftest_kernel<<<1, 32, 0, s>>>(status, limit_ns);
 }
 
+nmd_status launch_nearest_tc(const Factor& f, int64_t N, int rp, unsigned long long* keys, int* status,
+                             int num_sms, cudaStream_t s) {
+  if (!tc_supported(rp, NMD_FP32)) return NMD_ERR_UNSUPPORTED;
+  TcParams p{0, N, 0, N, f.hi, f.lo, nullptr, nullptr, status, nullptr, nullptr, nullptr, nullptr, 0, 0, 0,
+             nullptr, 0, keys};
+  const int64_t ntiles = (N + BM - 1) / BM;
+  const int64_t rounds = (ntiles + num_sms - 1) / num_sms;
+  const int grid = (int)((ntiles + rounds - 1) / rounds);
+  return dispatch<2>(rp, 0, true, f, f, p, grid, s);
+}
+
 nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts, int* nparts, int* status,
                                 cudaStream_t s, int64_t* launches) {
   if (!tc_supported(h->rp, h->opt.precision)) return NMD_ERR_UNSUPPORTED;
@@ -939,7 +987,7 @@ nmd_status launch_loss_dense_tc(const nmd_handle* h, double* parts, int maxparts
   int64_t ntiles = (h->m + BM - 1) / BM;
   int grid = (int)(ntiles < h->num_sms ? ntiles : h->num_sms);
   if (grid > maxparts) grid = maxparts;
-  nmd_status st = dispatch<true>(h->rp, 0, h->opt.precision == NMD_FP32, h->W, h->B, p, grid, s);
+  nmd_status st = dispatch<1>(h->rp, 0, h->opt.precision == NMD_FP32, h->W, h->B, p, grid, s);
   if (st == NMD_OK) {
     ++*launches;
     *nparts = grid;

@@ -33,6 +33,7 @@ EXPORTS = [
     "nmd_block_terms", "nmd_dense_products", "nmd_panel_traversal", "nmd_get_state", "nmd_set_state",
     "nmd_launch_count", "nmd_skip_count", "nmd_selftest_wait_timeout", "nmd_profile", "nmd_profile_read", "nmd_status_string", "nmd_last_error",
     "nmd_destroy", "nmd_gram_noalloc", "nmd_support_term", "nmd_block_update_combined", "nmd_range_mask",
+    "nmd_embed", "nmd_nn_workspace_bytes", "nmd_nearest_neighbors",
 ]
 
 
@@ -100,6 +101,10 @@ def lib() -> C.CDLL:
             "nmd_block_update_combined": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int64]),
             "nmd_range_mask": (C.c_int, [_P, C.c_int32, C.c_int64, C.c_int32, _P, C.c_int64, _i64p, _i64p,
                                          _i64p]),
+            "nmd_embed": (C.c_int, [_P, _P, _P]),
+            "nmd_nn_workspace_bytes": (C.c_int, [C.c_int64, C.c_int32, C.POINTER(C.c_size_t)]),
+            "nmd_nearest_neighbors": (C.c_int, [_P, C.c_int64, C.c_int32, _P, _P, _P, _i64p, _P, C.c_size_t,
+                                                _P]),
         }
         for name, (res, args) in sig.items():
             f = getattr(L, name)
@@ -246,6 +251,42 @@ def nmd_range_mask(h, side, block, kind):
     _check(h, L.nmd_range_mask(h, side, block, kind, mask.ctypes.data, mask.size, C.byref(nt), C.byref(nw),
                                C.byref(cr)), "nmd_range_mask")
     return mask, cr.value
+
+
+def nmd_embed(h, d_xi, d_sigma=None):
+    _check(h, lib().nmd_embed(h, _ptr(d_xi), _ptr(d_sigma)), "nmd_embed")
+
+
+def nmd_nn_workspace_bytes(N: int, d: int) -> int:
+    v = C.c_size_t(0)
+    _check(None, lib().nmd_nn_workspace_bytes(N, d, C.byref(v)), "nmd_nn_workspace_bytes")
+    return v.value
+
+
+def nmd_nearest_neighbors(d_x, N: int, d: int, d_labels, d_nn, d_best, workspace, stream_ptr: int):
+    """Runs the search; returns the 1-NN error count (None without labels)."""
+    err = C.c_int64(-1)
+    _check(None, lib().nmd_nearest_neighbors(_ptr(d_x), N, d, _ptr(d_labels), _ptr(d_nn), _ptr(d_best),
+                                             C.byref(err) if d_labels is not None else None, _ptr(workspace),
+                                             workspace.numel(), stream_ptr), "nmd_nearest_neighbors")
+    return err.value if d_labels is not None else None
+
+
+def nearest_neighbors(x, labels=None):
+    """(nn, best, errors) for the rows of a CUDA tensor x (N x d): the other
+    row with the largest inner product, that inner product, and the number of
+    rows whose neighbour has another label (None without labels).  The
+    workspace is a torch tensor on x's device."""
+    import torch
+    x = x.contiguous().float()
+    N, d = x.shape
+    with torch.cuda.device(x.device):
+        ws = torch.empty(nmd_nn_workspace_bytes(N, d), dtype=torch.uint8, device=x.device)
+        nn = torch.empty(N, dtype=torch.int32, device=x.device)
+        best = torch.empty(N, dtype=torch.float32, device=x.device)
+        lab = None if labels is None else torch.as_tensor(labels, dtype=torch.int32).to(x.device).contiguous()
+        errors = nmd_nearest_neighbors(x, N, d, lab, nn, best, ws, torch.cuda.current_stream(x.device).cuda_stream)
+    return nn, best, errors
 
 
 def nmd_get_state(h, m, n, r):
@@ -422,6 +463,16 @@ class Solver:
         """Delta form: chunks skipped (NMD_SKIP_VOTE: second product of an
         all-zero P; NMD_SKIP_RANGE: both products of a cleared chunk)."""
         return nmd_skip_count(self.h, reset)
+
+    def embed(self):
+        """(xi, sigma) as CUDA tensors: the n x 2r unit rows of the cell
+        embedding (Sec. 5.3) and the r singular values of W H, descending."""
+        import torch
+        with torch.cuda.device(self.device):
+            xi = torch.empty((self.n, 2 * self.r), dtype=torch.float32, device=self.device)
+            sigma = torch.empty(self.r, dtype=torch.float32, device=self.device)
+            nmd_embed(self.h, xi, sigma)
+        return xi, sigma
 
     def range_mask(self, side, block, kind):
         """The range-search mask of one block update and its chunk size."""
