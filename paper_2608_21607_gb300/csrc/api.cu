@@ -309,6 +309,13 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->ball_q = c.take<float>((size_t)((N + 63) / 64) * rp);
   w->rad_q = c.take<float>((size_t)((N + 63) / 64));
   w->rmask = c.take<uint32_t>((size_t)range_mask_words(m, n));
+  for (Factor& g : w->gi) {
+    g.rows = rp;
+    g.master = c.take<float>((size_t)rp * rp);
+    g.hi = c.take<bf16>((size_t)rp * rp);
+    g.lo = c.take<bf16>((size_t)rp * rp);
+    g.lo2 = c.take<bf16>((size_t)rp * rp);
+  }
   w->loss_part = c.take<double>((size_t)kLossParts * 8);
   w->loss_out = c.take<double>(8);
   w->status = c.take<int>(kStatusWords);
@@ -617,6 +624,19 @@ struct NextUse {
   int kind;
 };
 
+// bf16 mode at r_pad = 256: X = R G^{-1} costs 2 r^2 flops per row, more
+// than the CUDA cores deliver at the update's memory rate, so it runs on the
+// tensor cores (the update pass of the dense kernel; R and G^{-1} as two bf16
+// pieces each, three products, fp32 accumulation)
+bool tc_update(const nmd_handle* h) {
+  return h->rp == 256 && h->opt.precision == NMD_BF16 && tc_supported(h->rp, h->opt.precision);
+}
+
+// the pieces of the G^{-1} buffer in use (by step parity, or the exact steps' cache)
+const Factor* gi_of(const nmd_handle* h, const float* Ginv) {
+  return Ginv == h->ws.Ginv ? &h->ws.gi[0] : Ginv == h->ws.Ginv2 ? &h->ws.gi[1] : &h->ws.gi[2];
+}
+
 nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro, float* R, float* Rs,
                               const uint8_t* flags, const float* Ginv, int64_t lo, int64_t hi, bool momentum,
                               cudaStream_t s, bool gram = false) {
@@ -625,9 +645,16 @@ nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro,
   sub.m0 = ro.m0 + lo;
   sub.M = hi - lo;
   TimedScope ts(h, NMD_K_UPDATE, s);
-  launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, Ginv, (float)h->opt.eta,
-                momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, gram ? h->ws.gram_part : nullptr,
-                h->opt.precision == NMD_BF16, s);
+  if (tc_update(h)) {
+    const nmd_status st = launch_update_tc(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, *gi_of(h, Ginv),
+                                           (float)h->opt.eta, momentum ? (float)h->opt.gamma : 0.f, momentum,
+                                           h->ws.status, h->num_sms, s);
+    if (st != NMD_OK) return fail(h, st, "tensor-core update");
+  } else {
+    launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, Ginv, (float)h->opt.eta,
+                  momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, gram ? h->ws.gram_part : nullptr,
+                  h->opt.precision == NMD_BF16, s);
+  }
   h->launches++;
   return NMD_OK;
 }
@@ -730,6 +757,11 @@ nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_upda
                 (float)h->opt.ridge, G, h->side);
     launch_chol_inv(G, h->r, h->rp, Ginv, h->ws.status, h->side);
     h->launches += pre ? 2 : 3;
+    if (tc_update(h)) {   // the pieces of G^{-1} for the tensor-core update
+      Factor gi = *gi_of(h, Ginv);
+      launch_pack(Ginv, false, h->rp, h->rp, h->rp, gi, h->side);
+      h->launches++;
+    }
   }
   if ((st = after_launch(h, "gram/cholesky")) != NMD_OK) return st;
   // sparse correction over the block's support

@@ -151,6 +151,9 @@ struct Workspace {
   float* ball_q = nullptr;        // ceil(max(m, n) / 64) x rp
   float* rad_q = nullptr;
   uint32_t* rmask = nullptr;      // range_mask_words(m, n)
+  // the bf16 pieces of G^{-1}, G2^{-1} and the cached G^{-1} of exact steps
+  // (rp rows each), for the tensor-core update at r_pad = 256
+  Factor gi[3];
 };
 
 constexpr int kGramParts = 64;
@@ -292,6 +295,13 @@ int embed_max_rank();
 nmd_status launch_embed(const Factor& W, const Factor& B, int64_t n, int r, int rp, float* gram_part, float* GA,
                         float* GB, float* scratch, float* TA, float* TB, float* sigma, float* xi, int num_sms,
                         cudaStream_t s, int64_t* launches);
+// The update on the tensor cores (bf16 mode, r_pad = 256): X = (R + Rs)
+// G^{-1} by the update pass of the dense kernel, R and G^{-1} in two bf16
+// pieces each (gi: the pieces of G^{-1}, rp rows), the step applied to rows
+// [a.m0, a.m0 + a.M) of a.fm in its epilogue
+nmd_status launch_update_tc(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags,
+                            const Factor& gi, float eta, float gamma, bool momentum, int* status, int num_sms,
+                            cudaStream_t s);
 // Q-side rows per chunk of the tensor-core dense kernel (64 or 128)
 int panel_chunk_rows(int rp, int precision);
 // balls of the 128-row M tiles of rows [m0, m0 + M) of Xm and of the bn-row

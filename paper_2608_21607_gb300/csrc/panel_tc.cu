@@ -147,6 +147,21 @@ struct TcParams {
   // largest L_ij over j != i, as an orderable key (value bits << 32 |
   // ~j); the caller zeroes the keys
   unsigned long long* nn_key;
+  // update pass (M side = the step's right-hand side R, Q side = G^{-1}):
+  // X = (R + Rs) G^{-1} with R and Rs fp32 rows (relative to the range, Rs
+  // only where upd_flags is set) split into two bf16 pieces as they are
+  // loaded; the epilogue applies the update of eqs. lsqA_sto / spLsqA to the
+  // factor rows upd_row0 + i of upd_M (fp32 master), upd_E (momentum) and
+  // upd_hi (bf16 piece)
+  const float* upd_R;
+  const float* upd_Rs;
+  const uint8_t* upd_flags;
+  float* upd_M;
+  float* upd_E;
+  bf16* upd_hi;
+  int64_t upd_row0;
+  float eta, gamma;
+  int momentum, delta_form;
 };
 
 __device__ __forceinline__ void record(int* status, int code, int detail) {
@@ -250,7 +265,9 @@ __device__ __forceinline__ ChunkMask chunk_mask(const TcParams& p, int64_t t, in
 
 // MODE: 0 the panel contraction R = P(L) Q; 1 the loss pass (first product
 // only, sums of max(0, L)^2 and max(0, L) off the support); 2 the nearest-
-// neighbour pass (first product only, per row the largest L_ij, j != i).
+// neighbour pass (first product only, per row the largest L_ij, j != i);
+// 3 the update pass (first product only: X = R G^{-1} and the step applied
+// to the factor rows in the epilogue).
 // SKIPM (Delta form only): 1 skips the second product of chunks whose
 // rectified tile is zero (a vote of the epilogue warps); 2 skips both
 // products of the chunks that the range-search mask clears.  Separate
@@ -261,7 +278,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const __grid_constant__ CUtensorMap tq_lo2, const __grid_constant__ CUtensorMap tw,
                     const TcParams p) {
   constexpr bool LOSS = MODE != 0;     // the first product only
-  constexpr bool SUMS = MODE == 1, NEAREST = MODE == 2;
+  constexpr bool SUMS = MODE == 1, NEAREST = MODE == 2, UPDATE = MODE == 3;
+  static_assert(!UPDATE || SPLIT, "the update pass splits R and G^{-1} into two pieces");
+  // the update is skipped under a sticky error (as the CUDA-core update is);
+  // every thread reads the same word before any barrier or TMEM exists
+  if (UPDATE && *(volatile int*)p.status != 0) return;
   using C = Cfg<RP, SPLIT, LOSS>;
   constexpr int BN = C::BN, NB = C::NB, NSTAGE = C::NSTAGE, NWB = C::NWB;
   constexpr bool VOTE = SKIPM == 1, RANGE = SKIPM == 2;
@@ -532,6 +553,40 @@ __global__ void __launch_bounds__(kThreads, 1)
       if constexpr (C::WSMEM) return;   // loaded by the producer's TMA
       const int64_t li = tile * BM + row;
       const bool valid = li < p.M;
+      if constexpr (UPDATE) {
+        // R + Rs of this row, split into hi = bf16(x) and lo = bf16(x - hi)
+        const float* src = p.upd_R + (valid ? li : 0) * RP;
+        const float* srs = p.upd_Rs + (valid ? li : 0) * RP;
+        const bool flg = valid && p.upd_flags[li] != 0;
+        const uint32_t wcol = tmem + lane_base + C::COL_W + wb * C::WCOLS;
+#pragma unroll 1
+        for (int q = wg; q < RP / 16; q += 2) {
+          float x[16];
+#pragma unroll
+          for (int k = 0; k < 16; k += 4) {
+            float4 a = valid ? __ldg((const float4*)(src + 16 * q + k)) : make_float4(0.f, 0.f, 0.f, 0.f);
+            if (flg) {
+              const float4 b = __ldg((const float4*)(srs + 16 * q + k));
+              a.x += b.x; a.y += b.y; a.z += b.z; a.w += b.w;
+            }
+            x[k] = a.x; x[k + 1] = a.y; x[k + 2] = a.z; x[k + 3] = a.w;
+          }
+          uint32_t vh[8], vl[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) {
+            const uint32_t h = pack_bf16x2(x[2 * k], x[2 * k + 1]);
+            vh[k] = h;
+            vl[k] = pack_bf16x2(x[2 * k] - __uint_as_float(h << 16), x[2 * k + 1] - __uint_as_float(h & 0xffff0000u));
+          }
+          tmem_st8(wcol + q * 8, vh);
+          tmem_st8(wcol + RP / 2 + q * 8, vl);
+        }
+        tmem_wait_st();
+        fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(b_wfull + 8 * wb);
+        return;
+      }
       const uint4* src = (const uint4*)(p.Mhi + (p.m0 + (valid ? li : 0)) * RP);
       const uint4* srcl = (const uint4*)(p.Mlo + (p.m0 + (valid ? li : 0)) * RP);
       const uint32_t wcol = tmem + lane_base + C::COL_W + wb * C::WCOLS;
@@ -604,7 +659,39 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (g * 32 + i < kv) p.Lout[li * p.K + c * BN + g * 32 + i] = __uint_as_float(v[i]);
             }
           }
-          if (NEAREST) {   // columns past the set or the row itself do not count
+          if (UPDATE) {   // X for columns [col0, col0 + 32) of this row: the step
+            const int64_t li = t * BM + row;
+            if (li < p.M) {
+              const int64_t col0 = c * BN + g * 32;
+              float* mrow = p.upd_M + (p.upd_row0 + li) * RP + col0;
+              float* erow = p.upd_E + (p.upd_row0 + li) * RP + col0;
+              uint32_t hw[16];
+              bool finite = true;
+#pragma unroll
+              for (int k = 0; k < 32; k += 4) {
+                const float4 mo = *(const float4*)(mrow + k);
+                const float4 eo = p.momentum ? *(const float4*)(erow + k) : make_float4(0.f, 0.f, 0.f, 0.f);
+                const float mv[4] = {mo.x, mo.y, mo.z, mo.w}, evo[4] = {eo.x, eo.y, eo.z, eo.w};
+                float nv[4], ev[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                  const float x = __uint_as_float(v[k + j]);
+                  const float u = p.delta_form ? p.eta * x : p.eta * (x - mv[j]);
+                  ev[j] = p.momentum ? fmaf(p.gamma, evo[j], u) : u;
+                  nv[j] = mv[j] + ev[j];
+                  finite = finite && isfinite(nv[j]);
+                }
+                *(float4*)(mrow + k) = make_float4(nv[0], nv[1], nv[2], nv[3]);
+                if (p.momentum) *(float4*)(erow + k) = make_float4(ev[0], ev[1], ev[2], ev[3]);
+                hw[k / 2] = pack_bf16x2(nv[0], nv[1]);
+                hw[k / 2 + 1] = pack_bf16x2(nv[2], nv[3]);
+              }
+              uint4* hrow = (uint4*)(p.upd_hi + (p.upd_row0 + li) * RP + col0);
+#pragma unroll
+              for (int k = 0; k < 4; ++k) hrow[k] = make_uint4(hw[4 * k], hw[4 * k + 1], hw[4 * k + 2], hw[4 * k + 3]);
+              if (!finite) record(p.status, NMD_ERR_DIVERGED, (int)(p.upd_row0 + li));
+            }
+          } else if (NEAREST) {   // columns past the set or the row itself do not count
             const int64_t cb = c * BN + g * 32, self = t * BM + row;
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
@@ -966,6 +1053,20 @@ nmd_status launch_panel_tc(const StepArgs& a, float* R, int* status, int* counte
 
 void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s) {
   wait_selftest_kernel<<<1, 32, 0, s>>>(status, limit_ns);
+}
+
+nmd_status launch_update_tc(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags,
+                            const Factor& gi, float eta, float gamma, bool momentum, int* status, int num_sms,
+                            cudaStream_t s) {
+  if (a.M <= 0) return NMD_OK;
+  TcParams p{0, a.M, 0, a.rp, nullptr, nullptr, nullptr, nullptr, status, nullptr, nullptr, nullptr, nullptr, 0,
+             0, 0, nullptr, 0, nullptr, R, Rs, flags, a.fm->master, a.fm->E, a.fm->hi, a.m0, eta, gamma,
+             momentum ? 1 : 0, a.epilogue == NMD_EPI_DELTA ? 1 : 0};
+  const int64_t ntiles = (a.M + BM - 1) / BM;
+  const int64_t rounds = (ntiles + num_sms - 1) / num_sms;
+  const int grid = (int)((ntiles + rounds - 1) / rounds);
+  if (a.rp != 256) return NMD_ERR_UNSUPPORTED;
+  return run<256, 0, true, 3>(*a.fm, gi, p, grid, s);
 }
 
 nmd_status launch_nearest_tc(const Factor& f, int64_t N, int rp, unsigned long long* keys, int* status,
