@@ -309,6 +309,7 @@ void layout(Carver& c, int64_t m, int64_t n, int64_t nnz, int rp, int64_t npanel
   w->ball_q = c.take<float>((size_t)((N + 63) / 64) * rp);
   w->rad_q = c.take<float>((size_t)((N + 63) / 64));
   w->rmask = c.take<uint32_t>((size_t)range_mask_words(m, n));
+  for (bf16*& g : w->gsplit) g = c.take<bf16>((size_t)2 * rp * split_stride(rp));
   for (Factor& g : w->gi) {
     g.rows = rp;
     g.master = c.take<float>((size_t)rp * rp);
@@ -637,6 +638,12 @@ const Factor* gi_of(const nmd_handle* h, const float* Ginv) {
   return Ginv == h->ws.Ginv ? &h->ws.gi[0] : Ginv == h->ws.Ginv2 ? &h->ws.gi[1] : &h->ws.gi[2];
 }
 
+// the transposed pieces of the same buffer (bf16 mode, r_pad <= 128)
+bf16* gsplit_of(const nmd_handle* h, const float* Ginv) {
+  if (h->opt.precision != NMD_BF16 || h->rp > 128) return nullptr;
+  return Ginv == h->ws.Ginv ? h->ws.gsplit[0] : Ginv == h->ws.Ginv2 ? h->ws.gsplit[1] : h->ws.gsplit[2];
+}
+
 nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro, float* R, float* Rs,
                               const uint8_t* flags, const float* Ginv, int64_t lo, int64_t hi, bool momentum,
                               cudaStream_t s, bool gram = false) {
@@ -651,7 +658,7 @@ nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro,
                                            h->ws.status, h->num_sms, s);
     if (st != NMD_OK) return fail(h, st, "tensor-core update");
   } else {
-    launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, Ginv, (float)h->opt.eta,
+    launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, Ginv, gsplit_of(h, Ginv), (float)h->opt.eta,
                   momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, gram ? h->ws.gram_part : nullptr,
                   h->opt.precision == NMD_BF16, s);
   }
@@ -755,7 +762,7 @@ nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_upda
     TimedScope ts(h, NMD_K_GRAM, h->side);
     launch_gram(pre ? nullptr : ro.fq, rounded, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, chunk,
                 (float)h->opt.ridge, G, h->side);
-    launch_chol_inv(G, h->r, h->rp, Ginv, h->ws.status, h->side);
+    launch_chol_inv(G, h->r, h->rp, Ginv, gsplit_of(h, Ginv), h->ws.status, h->side);
     h->launches += pre ? 2 : 3;
     if (tc_update(h)) {   // the pieces of G^{-1} for the tensor-core update
       Factor gi = *gi_of(h, Ginv);

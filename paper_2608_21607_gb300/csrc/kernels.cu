@@ -232,9 +232,20 @@ __global__ void __launch_bounds__(256) small_gemm_kernel(const float* __restrict
 //     (two buffers) and every row below subtracts sum_k l_ik Y[k, :].  One
 //     barrier per panel.
 //  3. G^{-1} = Y^T D^{-1} Y from shared memory.
+// entry (k, n) of G^{-1} as hi + lo bf16 pieces at row n, column k of the
+// transposed split (hi rows first, then lo rows)
+template <int RP>
+__device__ __forceinline__ void store_split(bf16* gsplit, int n, int k, float v) {
+  constexpr int SB = split_stride(RP);
+  const bf16 hi = __float2bfloat16_rn(v);
+  gsplit[n * SB + k] = hi;
+  gsplit[RP * SB + n * SB + k] = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
 template <int RP>
 __global__ void __launch_bounds__(RP * 4) ldlt_inv_reg_kernel(const float* __restrict__ G, int r,
-                                                              float* __restrict__ Ginv, int* __restrict__ status) {
+                                                              float* __restrict__ Ginv, bf16* __restrict__ gsplit,
+                                                              int* __restrict__ status) {
   constexpr int CPT = RP / 4, PB = CPT < 8 ? CPT : 8, LD = RP + 1;
   extern __shared__ __align__(16) float smr[];
   float* invd = smr;                 // RP: 1 / d_k
@@ -403,6 +414,9 @@ __global__ void __launch_bounds__(RP * 4) ldlt_inv_reg_kernel(const float* __res
 #pragma unroll
   for (int j = 0; j < CPT; j += 4)
     *(float4*)(Ginv + (size_t)i * RP + c0 + j) = make_float4(a[j], a[j + 1], a[j + 2], a[j + 3]);
+  if (gsplit)
+#pragma unroll
+    for (int j = 0; j < CPT; ++j) store_split<RP>(gsplit, c0 + j, i, a[j]);
 }
 
 inline size_t ldlt_reg_smem_bytes(int rp) {
@@ -455,6 +469,7 @@ __device__ __forceinline__ void tile_of(int q, int& I, int& J) {
 template <int RP>
 __global__ void __launch_bounds__(TileChol<RP>::NTHR, 1) ldlt_inv_tile_kernel(const float* __restrict__ G, int r,
                                                                           float* __restrict__ Ginv,
+                                                                          bf16* __restrict__ gsplit,
                                                                           int* __restrict__ status) {
   using C = TileChol<RP>;
   constexpr int TB = C::TB, NT = C::NT, LDT = C::LDT, TSZ = C::TSZ, NTHR = C::NTHR;
@@ -476,7 +491,10 @@ __global__ void __launch_bounds__(TileChol<RP>::NTHR, 1) ldlt_inv_tile_kernel(co
     if (i == j) diag0[i] = g;
   }
   for (int e = tid; e < RP * RP; e += NTHR)
-    if (e / RP >= r || e % RP >= r) Ginv[e] = 0.f;
+    if (e / RP >= r || e % RP >= r) {
+      Ginv[e] = 0.f;
+      if (gsplit) store_split<RP>(gsplit, e % RP, e / RP, 0.f);
+    }
   __syncthreads();
   const float tol = 4.0f * (float)r * FLT_EPSILON;
 
@@ -662,6 +680,10 @@ __global__ void __launch_bounds__(TileChol<RP>::NTHR, 1) ldlt_inv_tile_kernel(co
         if (ga < r && gb < r && (a0 != b0 || v <= u)) {
           Ginv[(size_t)ga * RP + gb] = acc[u][v];
           Ginv[(size_t)gb * RP + ga] = acc[u][v];
+          if (gsplit) {
+            store_split<RP>(gsplit, gb, ga, acc[u][v]);
+            store_split<RP>(gsplit, ga, gb, acc[u][v]);
+          }
         }
       }
   }
@@ -946,15 +968,23 @@ __global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __re
 // columns 4 tx + 4 TX g (g < CPT / 4), so that a quarter warp reads 128
 // contiguous bytes of G^{-1} and a half warp writes whole 256-byte rows.
 // ---------------------------------------------------------------------------
-template <int RP>
+template <int RP, bool TC = false>
 struct UpdCfg {
   static constexpr int CW = RP <= 128 ? RP : 128;   // output columns per block
   static constexpr int TR = RP <= 128 ? 64 : 32;    // rows per tile
   static constexpr int TY = TR / 4;                  // row groups of four
   static constexpr int TX = 256 / TY;                // column groups
   static constexpr int CPT = CW / TX;                // columns per thread (1, 2, 4 or 8)
-  static constexpr size_t SMEM = ((size_t)RP * CW + 2 * (size_t)TR * RP) * sizeof(float);
+  // tensor-core product: the staged tile's rows padded to RP + 8 floats and
+  // the two bf16 pieces of G^{-1} transposed, rows padded to RP + 8, so that
+  // the fragment loads and stores of a half warp meet 16 different bank pairs;
+  // one tile buffer (a block updates one tile)
+  static constexpr int SR = TC ? RP + 8 : RP;        // row stride of a staged tile (floats)
+  static constexpr int SB = split_stride(RP);        // row stride of a split G^{-1} (bf16)
+  static constexpr size_t SMEM = TC ? (size_t)TR * SR * sizeof(float) + 2 * (size_t)RP * SB * sizeof(bf16)
+                                    : ((size_t)RP * CW + 2 * (size_t)TR * RP) * sizeof(float);
   static_assert(CPT >= 1 && (CPT < 4 || CPT % 4 == 0), "column split");
+  static_assert(!TC || (CW == RP && TR == 64), "tensor-core product: one block column, tiles of 64 rows");
 };
 
 template <int CPT, int TX>
@@ -970,48 +1000,91 @@ __device__ __forceinline__ void cp_async16(void* smem_dst, const void* gsrc) {
 }
 __device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_0() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
 
-template <int RP>
+// D += A B on one 16 x 8 x 16 tile (bf16 operands, fp32 accumulation), the
+// fragment layouts of the PTX ISA's mma.m16n8k16: a[0..3] hold A's (row g,
+// columns 2c, 2c+1), (g+8, 2c..), (g, 2c+8..), (g+8, 2c+8..); b0, b1 hold B's
+// (rows 2c, 2c+1; column g) and (2c+8, 2c+9; g); d holds (g, 2c), (g, 2c+1),
+// (g+8, 2c), (g+8, 2c+1), with g = lane / 4 and c = lane % 4
+__device__ __forceinline__ void mma_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// two fp32 values as hi + lo pieces (bf16, round to nearest), packed in pairs
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+  const __nv_bfloat162 l = __floats2bfloat162_rn(x0 - __low2float(h), x1 - __high2float(h));
+  hi = reinterpret_cast<const uint32_t&>(h);
+  lo = reinterpret_cast<const uint32_t&>(l);
+}
+
+template <int RP, bool TC>
 __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
                                                      bf16* __restrict__ Mlo, bf16* __restrict__ Mlo2,
                                                      float* __restrict__ E, int64_t m0, int64_t rows,
                                                      const float* __restrict__ R, const float* __restrict__ Rs,
                                                      const uint8_t* __restrict__ flags,
-                                                     const float* __restrict__ Ginv, float eta,
+                                                     const float* __restrict__ Ginv,
+                                                     const bf16* __restrict__ gsplit, float eta,
                                                      float gamma, int momentum, int delta_form, int write_lo,
                                                      int* __restrict__ status, float* __restrict__ gpart,
                                                      int gram_round) {
-  using C = UpdCfg<RP>;
+  using C = UpdCfg<RP, TC>;
   constexpr int NV = C::TR * RP / 4 / 256;   // float4 of a tile per thread
-  constexpr int CW = C::CW, TR = C::TR, TX = C::TX, CPT = C::CPT;
+  constexpr int CW = C::CW, TR = C::TR, TX = C::TX, CPT = C::CPT, SR = C::SR;
   extern __shared__ __align__(16) float sm[];
-  float* Gs = sm;                               // RP x CW
-  float* Rb = sm + RP * CW;                     // 2 x TR x RP, row-major like R
+  // CUDA cores: G^{-1} (RP x CW) and two tile buffers (TR x RP, row-major
+  // like R).  Tensor cores: one tile buffer (TR x SR) and G^{-1}'s bf16
+  // pieces, transposed (RP x SB each).
+  float* Gs = sm;
+  float* Rb = TC ? sm : sm + RP * CW;
+  bf16* GhT = reinterpret_cast<bf16*>(sm + TR * SR);
+  bf16* GlT = GhT + RP * C::SB;
   if (*(volatile int*)status != 0) return;
   const int cw0 = blockIdx.y * CW;
   const int tx = threadIdx.x % TX, ty = threadIdx.x / TX;
   const int64_t ntiles = (rows + TR - 1) / TR;
   const int64_t total = rows * RP;              // floats of R in this step
+  // float4 e of a tile sits at row 4e / RP, column 4e % RP of the staged tile
+  auto soff = [](int e) { return ((4 * e) / RP) * SR + (4 * e) % RP; };
   auto issue = [&](int64_t tile, int buf) {
     const int64_t base = tile * TR * RP;
-    float* dst = Rb + buf * TR * RP;
+    float* dst = Rb + buf * TR * SR;
 #pragma unroll
     for (int u = 0; u < NV; ++u) {
       const int e = threadIdx.x + 256 * u;
-      if (base + 4 * e < total) cp_async16(dst + 4 * e, R + base + 4 * e);
+      if (base + 4 * e < total) cp_async16(dst + soff(e), R + base + 4 * e);
     }
   };
   int64_t t = blockIdx.x;
-  // G^{-1} (its CW columns) and the first tile of R in one copy group
-  for (int e = threadIdx.x; e < RP * CW / 4; e += 256) {
-    const int k = (4 * e) / CW, c = (4 * e) % CW;
-    cp_async16(Gs + 4 * e, Ginv + k * RP + cw0 + c);
+  if constexpr (TC) {
+    // G^{-1}'s pieces, transposed (GhT[n][k] = hi(G^{-1}[k][n]): a B
+    // fragment's pair of k values is one 32-bit load), and the first tile
+    for (int e = threadIdx.x; e < RP * C::SB / 4; e += 256) cp_async16(GhT + 8 * e, gsplit + 8 * e);
+    if (t < ntiles) issue(t, 0);
+    cp_async_commit();
+  } else {
+    // G^{-1} (its CW columns) and the first tile of R in one copy group
+    for (int e = threadIdx.x; e < RP * CW / 4; e += 256) {
+      const int k = (4 * e) / CW, c = (4 * e) % CW;
+      cp_async16(Gs + 4 * e, Ginv + k * RP + cw0 + c);
+    }
+    if (t < ntiles) issue(t, 0);
+    cp_async_commit();
   }
-  if (t < ntiles) issue(t, 0);
-  cp_async_commit();
   int buf = 0;
-  for (; t < ntiles; t += gridDim.x, buf ^= 1) {
-    if (t + gridDim.x < ntiles) issue(t + gridDim.x, buf ^ 1);
+  for (; t < ntiles; t += gridDim.x, buf ^= (TC ? 0 : 1)) {
+    if constexpr (TC) {
+      // (the buffer was released by the barrier that ended the last tile)
+      if (t != blockIdx.x) issue(t, 0);
+    } else if (t + gridDim.x < ntiles) {
+      issue(t + gridDim.x, buf ^ 1);
+    }
     cp_async_commit();
     const int64_t base = t * TR;
     // the support term of this tile: Rs on the rows flagged as having
@@ -1052,7 +1125,8 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
         }
       }
     }
-    cp_async_wait_1();
+    if constexpr (TC) cp_async_wait_0();
+    else cp_async_wait_1();
     // add the support term to the entries this thread copied (its own copies
     // have landed), then publish the tile
 #pragma unroll
@@ -1060,15 +1134,74 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
       const int e = threadIdx.x + 256 * u;
       const int64_t o = base * RP + 4 * e;
       if (o < total) {
-        float4* d = (float4*)(Rb + buf * TR * RP + 4 * e);
+        float4* d = (float4*)(Rb + buf * TR * SR + soff(e));
         float4 v = *d;
         v.x += sv[u].x; v.y += sv[u].y; v.z += sv[u].z; v.w += sv[u].w;
         *d = v;
       }
     }
     __syncthreads();
-    const float* Rt = Rb + buf * TR * RP + (4 * ty) * RP;
     float x[4][CPT];
+    if constexpr (TC) {
+      // X = (R + Rs) G^{-1} on the tensor cores: both factors as hi + lo
+      // bf16 pieces, three products (lo hi, hi lo, hi hi; lo lo dropped), fp32
+      // accumulation.  Warp w takes rows 16 (w % 4) .. + 15 and columns
+      // (w / 4) RP / 2 .. + RP / 2 - 1 of the tile's product.
+      constexpr int NT = RP / 16;   // 8-column tiles per warp (and 16-wide k steps)
+      float* Rt = Rb;
+      const int lane = threadIdx.x % 32, warp = threadIdx.x / 32, g = lane / 4, c2 = 2 * (lane % 4);
+      const int r0 = 16 * (warp % 4), n0 = (warp / 4) * (RP / 2);
+      float acc[NT][4];
+#pragma unroll
+      for (int n = 0; n < NT; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < RP / 16; ++ks) {
+        const int k0 = 16 * ks;
+        uint32_t ah[4], al[4];
+        const float2 v0 = *(const float2*)(Rt + (r0 + g) * SR + k0 + c2);
+        const float2 v1 = *(const float2*)(Rt + (r0 + g + 8) * SR + k0 + c2);
+        const float2 v2 = *(const float2*)(Rt + (r0 + g) * SR + k0 + 8 + c2);
+        const float2 v3 = *(const float2*)(Rt + (r0 + g + 8) * SR + k0 + 8 + c2);
+        split_pair(v0.x, v0.y, ah[0], al[0]);
+        split_pair(v1.x, v1.y, ah[1], al[1]);
+        split_pair(v2.x, v2.y, ah[2], al[2]);
+        split_pair(v3.x, v3.y, ah[3], al[3]);
+#pragma unroll
+        for (int n = 0; n < NT; ++n) {
+          const int row = (n0 + 8 * n + g) * C::SB + k0 + c2;
+          const uint32_t bh0 = *reinterpret_cast<const uint32_t*>(GhT + row);
+          const uint32_t bh1 = *reinterpret_cast<const uint32_t*>(GhT + row + 8);
+          const uint32_t bl0 = *reinterpret_cast<const uint32_t*>(GlT + row);
+          const uint32_t bl1 = *reinterpret_cast<const uint32_t*>(GlT + row + 8);
+          mma_16816(acc[n], al, bh0, bh1);
+          mma_16816(acc[n], ah, bl0, bl1);
+          mma_16816(acc[n], ah, bh0, bh1);
+        }
+      }
+      __syncthreads();   // every warp has read its rows of the tile: X replaces it
+#pragma unroll
+      for (int n = 0; n < NT; ++n) {
+        float* o = Rt + (r0 + g) * SR + n0 + 8 * n + c2;
+        *(float2*)o = make_float2(acc[n][0], acc[n][1]);
+        *(float2*)(o + 8 * SR) = make_float2(acc[n][2], acc[n][3]);
+      }
+      __syncthreads();
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const float* xr = Rt + (4 * ty + i) * SR;
+        if (CPT >= 4) {
+#pragma unroll
+          for (int j = 0; j < CPT; j += 4) {
+            const float4 v = *(const float4*)(xr + upd_col<CPT, TX>(tx, j));
+            x[i][j] = v.x; x[i][j + 1] = v.y; x[i][j + 2] = v.z; x[i][j + 3] = v.w;
+          }
+        } else {
+#pragma unroll
+          for (int j = 0; j < CPT; ++j) x[i][j] = xr[upd_col<CPT, TX>(tx, j)];
+        }
+      }
+    } else {
+    const float* Rt = Rb + buf * TR * RP + (4 * ty) * RP;
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
@@ -1100,12 +1233,13 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
         }
       }
     }
+    }
     // Gram partials of the new rows (r_pad <= 64, one block column): the
     // tile's R staging buffer receives the new rows once every thread is done
     // with it (rows past the end read as zero)
     constexpr bool GRAM_OK = RP <= 64 && CW == RP && TR == 64;
     const bool gram = GRAM_OK && gpart != nullptr;
-    float* Ms = Rb + buf * TR * RP;
+    float* Ms = Rb + buf * TR * SR;
     if (gram) __syncthreads();
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
@@ -1113,7 +1247,7 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
       if (li >= rows) {
         if (gram)
 #pragma unroll
-          for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * RP + upd_col<CPT, TX>(tx, j)] = 0.f;
+          for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * SR + upd_col<CPT, TX>(tx, j)] = 0.f;
         continue;
       }
       const int64_t g = (m0 + li) * RP + cw0;
@@ -1164,7 +1298,7 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
       if (!finite) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
       if (gram)
 #pragma unroll
-        for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * RP + upd_col<CPT, TX>(tx, j)] = nv[j];
+        for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * SR + upd_col<CPT, TX>(tx, j)] = nv[j];
     }
     if constexpr (GRAM_OK) {
       if (gram) {
@@ -1185,8 +1319,8 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
           float av[GA], bv[GA];
 #pragma unroll
           for (int u = 0; u < GA; ++u) {
-            av[u] = Ms[rr * RP + a0 + u];
-            bv[u] = Ms[rr * RP + b0 + u];
+            av[u] = Ms[rr * SR + a0 + u];
+            bv[u] = Ms[rr * SR + b0 + u];
             if (gram_round) {
               av[u] = __bfloat162float(__float2bfloat16_rn(av[u]));
               bv[u] = __bfloat162float(__float2bfloat16_rn(bv[u]));
@@ -1351,12 +1485,12 @@ void launch_small_gemm(const float* A, int64_t lda, const float* B, int64_t ldb,
   small_gemm_kernel<<<grid, 256, 0, s>>>(A, lda, B, ldb, C, ldc, M, N, K);
 }
 
-void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cudaStream_t s) {
+void launch_chol_inv(const float* G, int r, int rp, float* Ginv, bf16* gsplit, int* status, cudaStream_t s) {
   switch (rp) {
-    case 16: ldlt_inv_reg_kernel<16><<<1, 64, ldlt_reg_smem_bytes(16), s>>>(G, r, Ginv, status); break;
-    case 32: ldlt_inv_reg_kernel<32><<<1, 128, ldlt_reg_smem_bytes(32), s>>>(G, r, Ginv, status); break;
+    case 16: ldlt_inv_reg_kernel<16><<<1, 64, ldlt_reg_smem_bytes(16), s>>>(G, r, Ginv, gsplit, status); break;
+    case 32: ldlt_inv_reg_kernel<32><<<1, 128, ldlt_reg_smem_bytes(32), s>>>(G, r, Ginv, gsplit, status); break;
     case 64:
-      ldlt_inv_tile_kernel<64><<<1, TileChol<64>::NTHR, TileChol<64>::SMEM, s>>>(G, r, Ginv, status);
+      ldlt_inv_tile_kernel<64><<<1, TileChol<64>::NTHR, TileChol<64>::SMEM, s>>>(G, r, Ginv, gsplit, status);
       break;
     case 128: {
       static std::atomic<int> attr[kMaxDevices];
@@ -1364,7 +1498,7 @@ void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cu
         return cudaFuncSetAttribute(ldlt_inv_tile_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     (int)TileChol<128>::SMEM) == cudaSuccess ? 1 : 0;
       });
-      ldlt_inv_tile_kernel<128><<<1, TileChol<128>::NTHR, TileChol<128>::SMEM, s>>>(G, r, Ginv, status);
+      ldlt_inv_tile_kernel<128><<<1, TileChol<128>::NTHR, TileChol<128>::SMEM, s>>>(G, r, Ginv, gsplit, status);
       break;
     }
     default: {
@@ -1373,7 +1507,7 @@ void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cu
         return cudaFuncSetAttribute(ldlt_inv_tile_kernel<256>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     (int)TileChol<256>::SMEM) == cudaSuccess ? 1 : 0;
       });
-      ldlt_inv_tile_kernel<256><<<1, TileChol<256>::NTHR, TileChol<256>::SMEM, s>>>(G, r, Ginv, status);
+      ldlt_inv_tile_kernel<256><<<1, TileChol<256>::NTHR, TileChol<256>::SMEM, s>>>(G, r, Ginv, nullptr, status);
     }
   }
 }
@@ -1637,17 +1771,18 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
 #undef NMD_SP
 }
 
-template <int RP>
+template <int RP, bool TC>
 static void update_rp(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
-                      float eta, float gamma, bool momentum, int* status, float* gpart, bool gram_round,
+                      const bf16* gsplit, float eta, float gamma, bool momentum, int* status, float* gpart, bool gram_round,
                       cudaStream_t s) {
-  using C = UpdCfg<RP>;
+  using C = UpdCfg<RP, TC>;
   // the attribute and the occupancy belong to the current device
   static std::atomic<int> cache[kMaxDevices];
   const int per_sm = per_device(cache, [] {
     int n = 0;
-    cudaFuncSetAttribute(update_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, update_kernel<RP>, 256, C::SMEM) != cudaSuccess || n < 1)
+    cudaFuncSetAttribute(update_kernel<RP, TC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, update_kernel<RP, TC>, 256, C::SMEM) != cudaSuccess ||
+        n < 1)
       n = 1;
     return n;
   });
@@ -1659,20 +1794,29 @@ static void update_rp(const StepArgs& a, const float* R, const float* Rs, const 
   const int64_t tiles = (a.M + C::TR - 1) / C::TR;
   dim3 grid((unsigned)std::min<int64_t>(tiles, (int64_t)a.num_sms * per_sm * 65535), RP / C::CW);
   const Factor& f = *a.fm;
-  update_kernel<RP><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, flags, Ginv, eta,
-                                               gamma,
-                                               momentum, a.epilogue == NMD_EPI_DELTA,
-                                               a.precision == NMD_FP32, status, gpart, gram_round ? 1 : 0);
+  update_kernel<RP, TC><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, flags, Ginv,
+                                                   gsplit, eta, gamma, momentum, a.epilogue == NMD_EPI_DELTA,
+                                                   a.precision == NMD_FP32, status, gpart, gram_round ? 1 : 0);
 }
 
+// X = (R + Rs) G^{-1}: in the bf16 mode on the tensor cores (two bf16 pieces
+// per factor, three products, fp32 accumulation: mma.sync, since the SMs the
+// deferred update shares with the dense kernel have no tensor memory free),
+// in the other modes on the CUDA cores in fp32
 void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
-                   float eta, float gamma, bool momentum, int* status, float* gpart, bool gram_round, cudaStream_t s) {
+                   const bf16* gsplit, float eta, float gamma, bool momentum, int* status, float* gpart,
+                   bool gram_round, cudaStream_t s) {
+  const bool tc = a.precision == NMD_BF16 && gsplit != nullptr;
   switch (a.rp) {
-    case 16: update_rp<16>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, gpart, gram_round, s); break;
-    case 32: update_rp<32>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, gpart, gram_round, s); break;
-    case 64: update_rp<64>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, gpart, gram_round, s); break;
-    case 128: update_rp<128>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, nullptr, false, s); break;
-    default: update_rp<256>(a, R, Rs, flags, Ginv, eta, gamma, momentum, status, nullptr, false, s); break;
+#define NMD_UPD(RPV, GP, GR)                                                                     \
+  (tc ? update_rp<RPV, true>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, GP, GR, s)     \
+      : update_rp<RPV, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, GP, GR, s))
+    case 16: NMD_UPD(16, gpart, gram_round); break;
+    case 32: NMD_UPD(32, gpart, gram_round); break;
+    case 64: NMD_UPD(64, gpart, gram_round); break;
+    case 128: NMD_UPD(128, nullptr, false); break;
+    default: update_rp<256, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, nullptr, false, s); break;
+#undef NMD_UPD
   }
 }
 

@@ -154,7 +154,16 @@ struct Workspace {
   // the bf16 pieces of G^{-1}, G2^{-1} and the cached G^{-1} of exact steps
   // (rp rows each), for the tensor-core update at r_pad = 256
   Factor gi[3];
+  // the same three, transposed, for the update's tensor-core product at
+  // r_pad <= 128 in the bf16 mode: hi then lo, rp rows of split_stride(rp)
+  // each, written by the G^{-1} kernels
+  bf16* gsplit[3] = {nullptr, nullptr, nullptr};
 };
+
+// row stride (bf16 elements) of a transposed, split G^{-1}: 8 past r_pad, so
+// that the rows start 16-byte aligned and the fragment loads of a half warp
+// fall in 16 different bank pairs
+constexpr int split_stride(int rp) { return rp + 8; }
 
 constexpr int kGramParts = 64;
 constexpr int64_t kRpartRows = 256 * 128;   // splits x tiles x 128 rows never exceed 256 SMs' worth
@@ -243,7 +252,10 @@ void launch_gram(const Factor* fq, bool rounded, int64_t q0, int64_t K, int r, i
                  int64_t chunk, float ridge, float* G, cudaStream_t s);
 // Ginv = G^{-1} through the Cholesky (L D L^T) factorisation; NMD_ERR_NOT_SPD
 // in the status words on failure
-void launch_chol_inv(const float* G, int r, int rp, float* Ginv, int* status, cudaStream_t s);
+// G^{-1} (rp x rp, row-major); with gsplit also its hi and lo bf16 pieces,
+// transposed (gsplit[n * split_stride(rp) + k] = hi(G^{-1}[k][n]), lo at
+// gsplit + rp * split_stride(rp)), pad entries zero
+void launch_chol_inv(const float* G, int r, int rp, float* Ginv, bf16* gsplit, int* status, cudaStream_t s);
 // C = A B (row-major fp32, M x K times K x N, N and K <= 256)
 void launch_small_gemm(const float* A, int64_t lda, const float* B, int64_t ldb, float* C, int64_t ldc, int64_t M,
                        int N, int K, cudaStream_t s);
@@ -258,9 +270,11 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
 // gpart, when not nullptr and r_pad <= 64: also write the Gram partials of the
 // new rows, one per 64-row tile (gram_round: of their bf16 rounding), exactly
 // as launch_gram would with parts of 64 rows
+// gsplit: G^{-1}'s pieces as written by launch_chol_inv (read by the bf16
+// mode's tensor-core product at r_pad <= 128)
 void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags,
-                   const float* Ginv, float eta, float gamma, bool momentum, int* status, float* gpart,
-                   bool gram_round, cudaStream_t s);
+                   const float* Ginv, const bf16* gsplit, float eta, float gamma, bool momentum, int* status,
+                   float* gpart, bool gram_round, cudaStream_t s);
 void launch_combine(float* R, const float* Rs, const uint8_t* flags, int64_t rows, int rp, cudaStream_t s);
 // the bounded pipeline wait, run on a barrier that never completes
 void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);
