@@ -646,7 +646,7 @@ bf16* gsplit_of(const nmd_handle* h, const float* Ginv) {
 
 nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro, float* R, float* Rs,
                               const uint8_t* flags, const float* Ginv, int64_t lo, int64_t hi, bool momentum,
-                              cudaStream_t s, bool gram = false) {
+                              cudaStream_t s) {
   if (hi <= lo) return NMD_OK;
   StepArgs sub = a;
   sub.m0 = ro.m0 + lo;
@@ -659,8 +659,7 @@ nmd_status launch_update_rows(nmd_handle* h, const StepArgs& a, const Roles& ro,
     if (st != NMD_OK) return fail(h, st, "tensor-core update");
   } else {
     launch_update(sub, R + lo * h->rp, Rs + lo * h->rp, flags + lo, Ginv, gsplit_of(h, Ginv), (float)h->opt.eta,
-                  momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, gram ? h->ws.gram_part : nullptr,
-                  h->opt.precision == NMD_BF16, s);
+                  momentum ? (float)h->opt.gamma : 0.f, momentum, h->ws.status, s);
   }
   h->launches++;
   return NMD_OK;
@@ -746,24 +745,19 @@ nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_upda
   // term of R.  None reads what another writes, so they overlap; the update
   // joins them.
   // Gram partials over parts of 64 Q-side rows where there are at most
-  // kGramParts of them (then the previous step's update of exactly these rows
-  // may already have written them, with the same arithmetic), else over
-  // kGramParts equal parts
+  // kGramParts of them, else over kGramParts equal parts
   const bool rows64 = (ro.K + 63) / 64 <= kGramParts;
   const int nparts = rows64 ? (int)((ro.K + 63) / 64) : kGramParts;
   const int64_t chunk = rows64 ? 64 : ((ro.K + nparts - 1) / nparts + 31) / 32 * 32;
-  const bool pre = h->gpre.active && kind == NMD_STOCH && h->gpre.f == fq && h->gpre.q0 == ro.q0 &&
-                   h->gpre.K == ro.K && h->gpre.step == h->step_index;
-  h->gpre.active = false;
   CK(h, cudaEventRecord(h->ev_fork, s));
   CK(h, cudaStreamWaitEvent(h->side, h->ev_fork, 0));
   CK(h, cudaStreamWaitEvent(h->side2, h->ev_fork, 0));
   if (need_gram) {
     TimedScope ts(h, NMD_K_GRAM, h->side);
-    launch_gram(pre ? nullptr : ro.fq, rounded, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, chunk,
-                (float)h->opt.ridge, G, h->side);
+    launch_gram(ro.fq, rounded, ro.q0, ro.K, h->r, h->rp, h->ws.gram_part, nparts, chunk, (float)h->opt.ridge, G,
+                h->side);
     launch_chol_inv(G, h->r, h->rp, Ginv, gsplit_of(h, Ginv), h->ws.status, h->side);
-    h->launches += pre ? 2 : 3;
+    h->launches += 3;
     if (tc_update(h)) {   // the pieces of G^{-1} for the tensor-core update
       Factor gi = *gi_of(h, Ginv);
       launch_pack(Ginv, false, h->rp, h->rp, h->rp, gi, h->side);
@@ -804,27 +798,14 @@ nmd_status run_step_roles(nmd_handle* h, const Roles& ro, int kind, bool do_upda
     // next step reads only these rows of this factor and writes the other
     // factor, the rest are updated on the aux stream, overlapping it
     int64_t lo = 0, hi = ro.M;
-    // the next step's Q-side block is exactly these rows (an alternating
-    // stochastic sweep): their update also writes that step's Gram partials
-    bool gram_next = false;
     if (next) {
       Roles rn;
       if (roles(h, next->side, next->block, next->kind, &rn) == NMD_OK && rn.fq == ro.fm && rn.fm != ro.fm) {
         lo = std::min(std::max(rn.q0 - ro.m0, (int64_t)0), ro.M);
         hi = std::max(std::min(rn.q0 + rn.K - ro.m0, ro.M), lo);
-        gram_next = next->kind == NMD_STOCH && h->rp <= 64 && lo == rn.q0 - ro.m0 && hi - lo == rn.K &&
-                    (rn.K + 63) / 64 <= kGramParts;
       }
     }
-    if ((st = launch_update_rows(h, a, ro, R, Rs, flags, Ginv, lo, hi, momentum, s, gram_next)) != NMD_OK)
-      return st;
-    if (gram_next) {
-      h->gpre.active = true;
-      h->gpre.f = fm;
-      h->gpre.q0 = ro.m0 + lo;
-      h->gpre.K = hi - lo;
-      h->gpre.step = h->step_index + 1;
-    }
+    if ((st = launch_update_rows(h, a, ro, R, Rs, flags, Ginv, lo, hi, momentum, s)) != NMD_OK) return st;
     if (lo > 0 || hi < ro.M) {
       CK(h, cudaEventRecord(h->ev_prio, s));
       CK(h, cudaStreamWaitEvent(h->aux, h->ev_prio, 0));
@@ -1152,7 +1133,6 @@ nmd_status nmd_sweep(nmd_handle* h) {
   for (size_t t = 0; t < steps.size() && st == NMD_OK; ++t)
     st = run_step(h, steps[t].side, steps[t].block, steps[t].kind, true,
                   t + 1 < steps.size() ? &steps[t + 1] : nullptr);
-  h->gpre.active = false;
   // `stream` continues after every kernel of the sweep, deferred ones included
   nmd_status st2 = wait_all_pending(h);
   h->cur = h->stream;
@@ -1277,7 +1257,6 @@ nmd_status nmd_embed(nmd_handle* h, float* d_xi, float* d_sigma) {
   if (st != NMD_OK) return st;
   if ((int64_t)h->n * h->rp < 6 * (int64_t)h->r * h->r)   // the r x r work space lives in R
     return fail(h, NMD_ERR_INVALID, "the cell embedding needs at least 6 r cells");
-  h->gpre.active = false;   // the Gram partials are overwritten
   st = launch_embed(h->W, h->B, h->n, h->r, h->rp, h->ws.gram_part, h->ws.G, h->ws.G2, h->ws.R, h->ws.Gx,
                     h->ws.Tm, d_sigma ? d_sigma : h->ws.Ginv2, d_xi, h->num_sms, h->stream, &h->launches);
   if (st != NMD_OK) return fail(h, st, "cudaFuncSetAttribute(embed_rows_kernel)");

@@ -1032,8 +1032,7 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
                                                      const float* __restrict__ Ginv,
                                                      const bf16* __restrict__ gsplit, float eta,
                                                      float gamma, int momentum, int delta_form, int write_lo,
-                                                     int* __restrict__ status, float* __restrict__ gpart,
-                                                     int gram_round) {
+                                                     int* __restrict__ status) {
   using C = UpdCfg<RP, TC>;
   constexpr int NV = C::TR * RP / 4 / 256;   // float4 of a tile per thread
   constexpr int CW = C::CW, TR = C::TR, TX = C::TX, CPT = C::CPT, SR = C::SR;
@@ -1234,22 +1233,10 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
       }
     }
     }
-    // Gram partials of the new rows (r_pad <= 64, one block column): the
-    // tile's R staging buffer receives the new rows once every thread is done
-    // with it (rows past the end read as zero)
-    constexpr bool GRAM_OK = RP <= 64 && CW == RP && TR == 64;
-    const bool gram = GRAM_OK && gpart != nullptr;
-    float* Ms = Rb + buf * TR * SR;
-    if (gram) __syncthreads();
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const int64_t li = base + 4 * ty + i;
-      if (li >= rows) {
-        if (gram)
-#pragma unroll
-          for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * SR + upd_col<CPT, TX>(tx, j)] = 0.f;
-        continue;
-      }
+      if (li >= rows) continue;
       const int64_t g = (m0 + li) * RP + cw0;
       bool finite = true;
       float nv[CPT], ev[CPT];
@@ -1296,47 +1283,6 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
         }
       }
       if (!finite) set_status(status, NMD_ERR_DIVERGED, (int)(m0 + li), 0);
-      if (gram)
-#pragma unroll
-        for (int j = 0; j < CPT; ++j) Ms[(4 * ty + i) * SR + upd_col<CPT, TX>(tx, j)] = nv[j];
-    }
-    if constexpr (GRAM_OK) {
-      if (gram) {
-        // partial t of the Gram matrix of the new rows (gram_round: of their
-        // bf16 rounding, the hi pieces just written): every entry summed over
-        // the tile's 64 rows in ascending order with fmaf, the same operations
-        // as gram_kernel on a part of 64 rows, so that a step gets the same G
-        // whichever kernel formed its partials
-        __syncthreads();
-        constexpr int GA = RP / 16;
-        const int a0 = (threadIdx.x / 16) * GA, b0 = (threadIdx.x % 16) * GA;
-        float g1[GA][GA];
-#pragma unroll
-        for (int u = 0; u < GA; ++u)
-#pragma unroll
-          for (int v = 0; v < GA; ++v) g1[u][v] = 0.f;
-        for (int rr = 0; rr < TR; ++rr) {
-          float av[GA], bv[GA];
-#pragma unroll
-          for (int u = 0; u < GA; ++u) {
-            av[u] = Ms[rr * SR + a0 + u];
-            bv[u] = Ms[rr * SR + b0 + u];
-            if (gram_round) {
-              av[u] = __bfloat162float(__float2bfloat16_rn(av[u]));
-              bv[u] = __bfloat162float(__float2bfloat16_rn(bv[u]));
-            }
-          }
-#pragma unroll
-          for (int u = 0; u < GA; ++u)
-#pragma unroll
-            for (int v = 0; v < GA; ++v) g1[u][v] = fmaf(av[u], bv[v], g1[u][v]);
-        }
-        float* o1 = gpart + (size_t)t * RP * RP;
-#pragma unroll
-        for (int u = 0; u < GA; ++u)
-#pragma unroll
-          for (int v = 0; v < GA; ++v) o1[(a0 + u) * RP + b0 + v] = g1[u][v];
-      }
     }
     __syncthreads();   // the buffer read above is refilled by the next iteration's copy
   }
@@ -1467,14 +1413,12 @@ void launch_unpack(const float* master, bool dst_is_rxN, int64_t N, int r, int r
 
 void launch_gram(const Factor* fq, bool rounded, int64_t q0, int64_t K, int r, int rp, float* parts, int nparts,
                  int64_t chunk, float ridge, float* G, cudaStream_t s) {
-  if (fq) {
-    int nt = (rp + 63) / 64;
-    dim3 grid(nt * (nt + 1) / 2, nparts);
-    if (rounded)
-      gram_kernel<bf16><<<grid, 256, 0, s>>>(fq->hi, q0, K, rp, parts, chunk);
-    else
-      gram_kernel<float><<<grid, 256, 0, s>>>(fq->master, q0, K, rp, parts, chunk);
-  }
+  int nt = (rp + 63) / 64;
+  dim3 grid(nt * (nt + 1) / 2, nparts);
+  if (rounded)
+    gram_kernel<bf16><<<grid, 256, 0, s>>>(fq->hi, q0, K, rp, parts, chunk);
+  else
+    gram_kernel<float><<<grid, 256, 0, s>>>(fq->master, q0, K, rp, parts, chunk);
   gram_reduce_kernel<<<(unsigned)((rp * rp + 255) / 256), 256, 0, s>>>(parts, nparts, r, rp, ridge, G);
 }
 
@@ -1773,8 +1717,7 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
 
 template <int RP, bool TC>
 static void update_rp(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
-                      const bf16* gsplit, float eta, float gamma, bool momentum, int* status, float* gpart, bool gram_round,
-                      cudaStream_t s) {
+                      const bf16* gsplit, float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
   using C = UpdCfg<RP, TC>;
   // the attribute and the occupancy belong to the current device
   static std::atomic<int> cache[kMaxDevices];
@@ -1796,7 +1739,7 @@ static void update_rp(const StepArgs& a, const float* R, const float* Rs, const 
   const Factor& f = *a.fm;
   update_kernel<RP, TC><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, flags, Ginv,
                                                    gsplit, eta, gamma, momentum, a.epilogue == NMD_EPI_DELTA,
-                                                   a.precision == NMD_FP32, status, gpart, gram_round ? 1 : 0);
+                                                   a.precision == NMD_FP32, status);
 }
 
 // X = (R + Rs) G^{-1}: in the bf16 mode on the tensor cores (two bf16 pieces
@@ -1804,18 +1747,17 @@ static void update_rp(const StepArgs& a, const float* R, const float* Rs, const 
 // deferred update shares with the dense kernel have no tensor memory free),
 // in the other modes on the CUDA cores in fp32
 void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
-                   const bf16* gsplit, float eta, float gamma, bool momentum, int* status, float* gpart,
-                   bool gram_round, cudaStream_t s) {
+                   const bf16* gsplit, float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
   const bool tc = a.precision == NMD_BF16 && gsplit != nullptr;
   switch (a.rp) {
-#define NMD_UPD(RPV, GP, GR)                                                                     \
-  (tc ? update_rp<RPV, true>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, GP, GR, s)     \
-      : update_rp<RPV, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, GP, GR, s))
-    case 16: NMD_UPD(16, gpart, gram_round); break;
-    case 32: NMD_UPD(32, gpart, gram_round); break;
-    case 64: NMD_UPD(64, gpart, gram_round); break;
-    case 128: NMD_UPD(128, nullptr, false); break;
-    default: update_rp<256, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, nullptr, false, s); break;
+#define NMD_UPD(RPV)                                                                      \
+  (tc ? update_rp<RPV, true>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, s) \
+      : update_rp<RPV, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, s))
+    case 16: NMD_UPD(16); break;
+    case 32: NMD_UPD(32); break;
+    case 64: NMD_UPD(64); break;
+    case 128: NMD_UPD(128); break;
+    default: update_rp<256, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, s); break;
 #undef NMD_UPD
   }
 }

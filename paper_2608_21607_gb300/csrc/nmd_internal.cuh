@@ -209,13 +209,6 @@ struct nmd_handle {
   const uint8_t* cur_flags = nullptr;   // the support-row flags of the last step
   float* cur_G = nullptr;
   float* cur_Ginv = nullptr;   // the inverse the last step's update applied
-  // Gram partials of the next step's Q-side block, written by this step's
-  // update of exactly those rows (see run_step); valid for step `step` only
-  struct GramPre {
-    bool active = false;
-    int f = -1;
-    int64_t q0 = 0, K = 0, step = -1;
-  } gpre;
   nmd::Workspace ws;
   nmd::Factor W, B;            // A = W (m x r), B = H^T (n x r)
   nmd::PanelSet panels[2][2];  // [side][kind]
@@ -246,8 +239,7 @@ void launch_unpack(const float* master, bool dst_is_rxN, int64_t N, int r, int r
                    cudaStream_t s);
 // G = Q^T Q of the Q-side rows [q0, q0 + K) (+ ridge on the diagonal) via
 // nparts fixed-order partials of `chunk` rows; rounded: of their bf16 pieces
-// (hi) instead of the fp32 masters.  fq == nullptr: the partials are already
-// there (written by launch_update's gpart) and only the reduction runs.
+// (hi) instead of the fp32 masters.
 void launch_gram(const Factor* fq, bool rounded, int64_t q0, int64_t K, int r, int rp, float* parts, int nparts,
                  int64_t chunk, float ridge, float* G, cudaStream_t s);
 // Ginv = G^{-1} through the Cholesky (L D L^T) factorisation; NMD_ERR_NOT_SPD
@@ -267,14 +259,11 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
                    const int32_t* qidx, const float* vals, float* R, float* partials, int64_t seg_first,
                    cudaStream_t s);
 // flags: one byte per row of the step (Rs is read only where it is nonzero)
-// gpart, when not nullptr and r_pad <= 64: also write the Gram partials of the
-// new rows, one per 64-row tile (gram_round: of their bf16 rounding), exactly
-// as launch_gram would with parts of 64 rows
 // gsplit: G^{-1}'s pieces as written by launch_chol_inv (read by the bf16
 // mode's tensor-core product at r_pad <= 128)
 void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags,
                    const float* Ginv, const bf16* gsplit, float eta, float gamma, bool momentum, int* status,
-                   float* gpart, bool gram_round, cudaStream_t s);
+                   cudaStream_t s);
 void launch_combine(float* R, const float* Rs, const uint8_t* flags, int64_t rows, int rp, cudaStream_t s);
 // the bounded pipeline wait, run on a barrier that never completes
 void launch_wait_selftest(int* status, uint64_t limit_ns, cudaStream_t s);
