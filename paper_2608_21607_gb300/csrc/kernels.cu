@@ -1724,6 +1724,10 @@ static void update_rp(const StepArgs& a, const float* R, const float* Rs, const 
   const int per_sm = per_device(cache, [] {
     int n = 0;
     cudaFuncSetAttribute(update_kernel<RP, TC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    // at r_pad <= 64 the largest shared-memory configuration, like the dense
+    // kernel's, so that an SM running update blocks can take a dense CTA and
+    // vice versa
+    if (RP <= 64) cudaFuncSetAttribute(update_kernel<RP, TC>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, update_kernel<RP, TC>, 256, C::SMEM) != cudaSuccess ||
         n < 1)
       n = 1;

@@ -934,11 +934,20 @@ nmd_status run(const Factor& fm, const Factor& fq, const TcParams& p, int grid, 
   // that the rows of a ragged last tile past the block read as zero
   CUtensorMap tw = th;
   if (C::WSMEM && !tensor_map(fm.hi, p.m0 + p.M, RP, C::PANEL_W, BM, &tw)) return NMD_ERR_CUDA;
-  // the shared-memory attribute belongs to the current device
+  // the shared-memory attributes belong to the current device.  At r_pad <=
+  // 64 the carveout asks for the largest shared-memory configuration (228 KB
+  // per SM): with the 166 KB of a CTA an SM would otherwise be set to 196 KB,
+  // leaving no room for an update block (37 KB) beside it, and the deferred
+  // update would run only on the SMs the grid leaves free.  (At r_pad = 256
+  // the same setting slowed the sweep by 15%: there nothing fits beside a
+  // CTA, and the L1 it takes away is lost.)
   static std::atomic<int> attr_set[kMaxDevices];
   if (!per_device(attr_set, [] {
-        return cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, MODE, SKIPM>,
-                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) == cudaSuccess ? 1 : 0;
+        return (cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, MODE, SKIPM>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM) == cudaSuccess &&
+                (RP > 64 || cudaFuncSetAttribute(panel_tc_kernel<RP, EPI, SPLIT, MODE, SKIPM>,
+                                                 cudaFuncAttributePreferredSharedMemoryCarveout,
+                                                 100) == cudaSuccess)) ? 1 : 0;
       }))
     return NMD_ERR_CUDA;
   const unsigned gz = p.ksplit ? (unsigned)((p.K + p.ksplit - 1) / p.ksplit) : 1u;
