@@ -544,9 +544,8 @@ Span panel_span(const Roles& ro) {
 }
 
 nmd_status launch_span(nmd_handle* h, const StepArgs& a, const Roles& ro, const Span& sp, float* Rs, cudaStream_t s) {
-  launch_sparse(a, sp.rows, sp.nrows, sp.whole, sp.nwhole, sp.seg, sp.nseg, sp.multi, sp.nmulti, ro.qidx, ro.vals,
-                Rs, h->ws.seg_partials, sp.seg_first, s);
-  h->launches += (sp.nrows > 0) + (sp.nwhole > 0) + 2 * (sp.nseg > 0);
+  h->launches += launch_sparse(a, sp.rows, sp.nrows, sp.whole, sp.nwhole, sp.seg, sp.nseg, sp.multi, sp.nmulti,
+                               ro.qidx, ro.vals, Rs, h->ws.seg_partials, sp.seg_first, s);
   return NMD_OK;
 }
 

@@ -1023,6 +1023,142 @@ __device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uin
   lo = reinterpret_cast<const uint32_t&>(l);
 }
 
+// ---------------------------------------------------------------------------
+// The support term with the step's whole Q-side block in shared memory (bf16
+// mode, r_pad 16 or 32, the block's bf16 rows within kSparseQBytes: the
+// planted and identity workloads, whose panels are dense enough that the q-row
+// gathers, not the CSR stream, set the pace of the kernels above).  One CTA
+// of 16 warps per SM copies the block's rows into shared memory once; then
+// each warp takes work items -- the short rows, the whole long rows and the
+// segments of split rows, the lists the other kernels take -- and gives each
+// lane one entry at a time: its q row from shared memory, the dot product with
+// m_i (which every lane holds) summed in column order, c = S_ik - min(0,
+// L_ik), and c q_k added to the lane's own partial row.  At the end of the
+// item the 32 partial rows are summed in lane order through shared memory
+// and written once.  An item's indices and values (at most 128 entries: four
+// per lane) are loaded while the previous item is computed.  In shared
+// memory, 16-byte chunk j of row k sits at chunk j ^ ((k >> 1) & (NCH - 1)),
+// so that a quarter warp reading chunk j of random rows spreads over the
+// eight 16-byte bank groups.
+// ---------------------------------------------------------------------------
+constexpr size_t kSparseQBytes = 156 * 1024;   // with 16 warps' reduction buffers, within 227 KB
+
+template <int RP>
+struct SpSmem {
+  static constexpr int NCH = RP * 2 / 16;   // 16-byte chunks per bf16 row
+  static constexpr int WARPS = 16;
+  static constexpr int LDB = RP + 1;        // row stride of a warp's reduction buffer (floats)
+  static constexpr size_t RED_BYTES = (size_t)WARPS * 32 * LDB * sizeof(float);
+};
+
+// 8 floats from 16 bytes of bf16
+__device__ __forceinline__ void unpack8(const uint4& u, float* f) {
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int q = 0; q < 4; ++q) {
+    f[2 * q] = __uint_as_float(w[q] << 16);
+    f[2 * q + 1] = __uint_as_float(w[q] & 0xffff0000u);
+  }
+}
+
+template <int RP>
+__global__ void __launch_bounds__(512, 1) sparse_smem_kernel(
+    const PanelRow* __restrict__ rows, int64_t nrows, const PanelRow* __restrict__ whole, int64_t nwhole,
+    const PanelRow* __restrict__ seg, int64_t nseg, const bf16* __restrict__ Mop, int64_t m0,
+    const bf16* __restrict__ Qop, int64_t q0, int64_t K, const int32_t* __restrict__ qidx,
+    const float* __restrict__ vals, float* __restrict__ R, float* __restrict__ partials) {
+  using C = SpSmem<RP>;
+  constexpr int NCH = C::NCH, LDB = C::LDB;
+  static_assert(RP == 16 || RP == 32, "r_pad 16 or 32");
+  extern __shared__ __align__(16) unsigned char sp_smem[];
+  float* red = reinterpret_cast<float*>(sp_smem);
+  uint4* qs = reinterpret_cast<uint4*>(sp_smem + C::RED_BYTES);
+  const uint4* qsrc = reinterpret_cast<const uint4*>(Qop + q0 * RP);
+  for (int64_t e = threadIdx.x; e < K * NCH; e += blockDim.x) {
+    const int64_t k = e / NCH;
+    const int j = (int)(e % NCH);
+    cp_async16(qs + k * NCH + (j ^ (int)((k >> 1) & (NCH - 1))), qsrc + e);
+  }
+  cp_async_commit();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float* rb = red + warp * 32 * LDB;
+  const int64_t nlong = nrows + nwhole, nitems = nlong + nseg;
+  const int64_t stride = (int64_t)gridDim.x * C::WARPS;
+  int64_t w = (int64_t)blockIdx.x * C::WARPS + warp;
+  // an item's descriptor, and its indices (relative to the block) and values
+  auto fetch = [&](int64_t x, PanelRow& pr, int* k4, float* s4) {
+    pr = x < nrows ? rows[x] : x < nlong ? whole[x - nrows] : seg[x - nlong];
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      const int e = lane + 32 * t;
+      const bool live = e < pr.len;
+      k4[t] = live ? (int)(__ldg(qidx + pr.beg + e) - q0) : 0;
+      s4[t] = live ? __ldg(vals + pr.beg + e) : 0.f;
+    }
+  };
+  PanelRow cur{0, 0, 0};
+  int kk[4] = {0, 0, 0, 0};
+  float ss[4] = {0.f, 0.f, 0.f, 0.f};
+  if (w < nitems) fetch(w, cur, kk, ss);
+  cp_async_wait_0();
+  __syncthreads();
+  for (; w < nitems; w += stride) {
+    PanelRow nxt{0, 0, 0};
+    int kn[4] = {0, 0, 0, 0};
+    float sn[4] = {0.f, 0.f, 0.f, 0.f};
+    if (w + stride < nitems) fetch(w + stride, nxt, kn, sn);
+    float mv[RP], acc[RP];
+    const uint4* mp = reinterpret_cast<const uint4*>(Mop + (int64_t)cur.row * RP);
+#pragma unroll
+    for (int c = 0; c < NCH; ++c) unpack8(__ldg(mp + c), mv + 8 * c);
+#pragma unroll
+    for (int c = 0; c < RP; ++c) acc[c] = 0.f;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      if (32 * t >= cur.len) break;   // warp-uniform
+      if (lane + 32 * t < cur.len) {
+        const int k = kk[t];
+        uint4 qc[NCH];
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) qc[j] = qs[k * NCH + (j ^ ((k >> 1) & (NCH - 1)))];
+        float dot = 0.f;
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+          float f[8];
+          unpack8(qc[j], f);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) dot = fmaf(mv[8 * j + q], f[q], dot);
+        }
+        const float cv = ss[t] - fminf(0.f, dot);
+#pragma unroll
+        for (int j = 0; j < NCH; ++j) {
+          float f[8];
+          unpack8(qc[j], f);
+#pragma unroll
+          for (int q = 0; q < 8; ++q) acc[8 * j + q] = fmaf(cv, f[q], acc[8 * j + q]);
+        }
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < RP; ++c) rb[lane * LDB + c] = acc[c];
+    __syncwarp();
+    float* out = w < nlong ? R + ((int64_t)cur.row - m0) * RP : partials + (w - nlong) * RP;
+    if (lane < RP) {
+      float sum = 0.f;
+#pragma unroll 8
+      for (int l = 0; l < 32; ++l) sum += rb[l * LDB + lane];
+      out[lane] = sum;
+    }
+    __syncwarp();   // the buffer is rewritten by the next item
+    cur = nxt;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+      kk[t] = kn[t];
+      ss[t] = sn[t];
+    }
+  }
+}
+
 template <int RP, bool TC>
 __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
                                                      bf16* __restrict__ Mlo, bf16* __restrict__ Mlo2,
@@ -1674,12 +1810,44 @@ static void launch_reduce(const PanelRow* multi, int64_t nmulti, const float* pa
   }
 }
 
-void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole, int64_t nwhole,
-                   const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
-                   const float* vals, float* R, float* partials, int64_t seg_first, cudaStream_t s) {
+template <int RP>
+static bool launch_sparse_smem(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole,
+                               int64_t nwhole, const PanelRow* seg, int64_t nseg, const int32_t* qidx,
+                               const float* vals, float* R, float* partials, cudaStream_t s) {
+  using C = SpSmem<RP>;
+  static std::atomic<int> attr[kMaxDevices];
+  if (!per_device(attr, [] {
+        return cudaFuncSetAttribute(sparse_smem_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)(C::RED_BYTES + kSparseQBytes)) == cudaSuccess ? 1 : 0;
+      }))
+    return false;
+  const int64_t nitems = nrows + nwhole + nseg;
+  const int64_t grid = std::min<int64_t>(a.num_sms, (nitems + C::WARPS - 1) / C::WARPS);
+  const size_t smem = C::RED_BYTES + (size_t)a.K * RP * sizeof(bf16);
+  sparse_smem_kernel<RP><<<(unsigned)grid, 32 * C::WARPS, smem, s>>>(rows, nrows, whole, nwhole, seg, nseg, a.fm->hi,
+                                                                    a.m0, a.fq->hi, a.q0, a.K, qidx, vals, R,
+                                                                    partials);
+  return true;
+}
+
+int launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole, int64_t nwhole,
+                  const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti, const int32_t* qidx,
+                  const float* vals, float* R, float* partials, int64_t seg_first, cudaStream_t s) {
   // slice w of `seg` is slice seg_first + w of its block, whose partial slot
   // the reduction (multi[].beg, relative to the block) reads
   float* seg_partials = partials + seg_first * a.rp;
+  // the Q-side block in shared memory where its bf16 rows fit
+  if (a.precision == NMD_BF16 && (a.rp == 16 || a.rp == 32) && a.K * a.rp * 2 <= (int64_t)kSparseQBytes &&
+      nrows + nwhole + nseg > 0) {
+    const bool ok = a.rp == 16 ? launch_sparse_smem<16>(a, rows, nrows, whole, nwhole, seg, nseg, qidx, vals, R,
+                                                        seg_partials, s)
+                               : launch_sparse_smem<32>(a, rows, nrows, whole, nwhole, seg, nseg, qidx, vals, R,
+                                                        seg_partials, s);
+    if (ok) {
+      if (nseg > 0) launch_reduce(multi, nmulti, partials, R, a.m0, a.rp, s);
+      return 1 + (nseg > 0);
+    }
+  }
   // The support term reads the same factor values as the rest of the step's
   // least-squares problem: the bf16 pieces in the bf16 mode (whose dense term
   // and Gram matrix are formed from them), the fp32 masters otherwise.
@@ -1713,6 +1881,7 @@ void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const
   }
 #undef NMD_SP2
 #undef NMD_SP
+  return (nrows > 0) + (nwhole > 0) + 2 * (nseg > 0);
 }
 
 template <int RP, bool TC>

@@ -254,7 +254,8 @@ void launch_small_gemm(const float* A, int64_t lda, const float* B, int64_t ldb,
 // rows: short rows; whole: the whole rows of the long-row kernel; seg: the
 // slices of the split rows, summed per row of `multi` into R
 // (bf16 mode: the factors' hi pieces, else the fp32 masters)
-void launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole,
+// returns the number of kernels launched
+int launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const PanelRow* whole,
                    int64_t nwhole, const PanelRow* seg, int64_t nseg, const PanelRow* multi, int64_t nmulti,
                    const int32_t* qidx, const float* vals, float* R, float* partials, int64_t seg_first,
                    cudaStream_t s);

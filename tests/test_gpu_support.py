@@ -5,8 +5,9 @@ M-side row with support in the block's panel,
 L_ik = m_i . q_k, on the step's own operands (the bf16 pieces in the bf16
 mode, the fp32 masters otherwise), and Rs_i = 0 on the other rows.  Covers
 short rows (one warp per row), whole long rows (lanes over the entries) and
-rows split into 128-entry slices with their fixed-order reduction, every
-padded rank, ragged blocks, all four step kinds.  Tolerance 1e-5 relative
+rows split into 128-entry slices with their fixed-order reduction, the
+shared-memory kernel (whole Q-side block staged, bf16 at r_pad 16 and 32),
+every padded rank, ragged blocks, all four step kinds.  Tolerance 1e-5 relative
 (fp32 accumulation against fp64)."""
 import numpy as np
 import pytest
@@ -41,6 +42,10 @@ CASES = [
     ("dense600x700_r32", lambda: _dense_rows(600, 700, 0.6, 9), 32, 400),   # rows of ~240 entries per panel
     ("dense500_r100", lambda: _dense_rows(500, 500, 0.35, 10), 100, 300),
     ("dense700_r256", lambda: _dense_rows(700, 700, 0.3, 11), 256, 600),
+    # whole Q-side blocks in shared memory (bf16, r_pad 32 and 16) at sizes
+    # near the limit: 2048 rows of 64 B, 4800 rows of 32 B
+    ("dense3000x2400_r32", lambda: _dense_rows(3000, 2400, 0.05, 12), 32, 2048),
+    ("dense2000x5000_r12", lambda: _dense_rows(2000, 5000, 0.02, 13), 12, 4800),
 ]
 
 
