@@ -1028,51 +1028,58 @@ __device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uin
 // mode, r_pad 16 or 32, the block's bf16 rows within kSparseQBytes: the
 // planted and identity workloads, whose panels are dense enough that the q-row
 // gathers, not the CSR stream, set the pace of the kernels above).  One CTA
-// of 16 warps per SM copies the block's rows into shared memory once; then
+// of 24 warps per SM copies the block's rows into shared memory once; then
 // each warp takes work items -- the short rows, the whole long rows and the
-// segments of split rows, the lists the other kernels take -- and gives each
-// lane one entry at a time: its q row from shared memory, the dot product with
-// m_i (which every lane holds) summed in column order, c = S_ik - min(0,
-// L_ik), and c q_k added to the lane's own partial row.  At the end of the
-// item the 32 partial rows are summed in lane order through shared memory
-// and written once.  An item's indices and values (at most 128 entries: four
-// per lane) are loaded while the previous item is computed.  In shared
-// memory, 16-byte chunk j of row k sits at chunk j ^ ((k >> 1) & (NCH - 1)),
-// so that a quarter warp reading chunk j of random rows spreads over the
-// eight 16-byte bank groups.
+// segments of split rows, the lists the other kernels take -- and splits each
+// entry's row over NCH lanes, one 16-byte chunk (8 columns) each, so that a
+// warp works on 32 / NCH entries at a time: each lane's partial dot product
+// with m_i (packed fp32 FMAs, the even and odd columns summed apart) is added
+// to the others' by a butterfly, c = S_ik - min(0, L_ik), and every lane adds
+// c times its 8 columns of q_k to its own partial sums.  At the end of
+// the item the partial sums of the entry slots are added by a butterfly over
+// the slots and written once.  Each lane fetches one of every 32 entries'
+// index and value (at most 128 entries per item: four), and they are passed
+// to the lanes of their slot by shuffles; an item's indices, values and m_i
+// are loaded while the previous item is computed, its descriptor two items
+// ahead.  In shared memory, 16-byte chunk j of row k sits at chunk j ^ ((k >>
+// 1) & (NCH - 1)).
 // ---------------------------------------------------------------------------
-constexpr size_t kSparseQBytes = 156 * 1024;   // with 16 warps' reduction buffers, within 227 KB
+constexpr size_t kSparseQBytes = 200 * 1024;
 
 template <int RP>
 struct SpSmem {
-  static constexpr int NCH = RP * 2 / 16;   // 16-byte chunks per bf16 row
-  static constexpr int WARPS = 16;
-  static constexpr int LDB = RP + 1;        // row stride of a warp's reduction buffer (floats)
-  static constexpr size_t RED_BYTES = (size_t)WARPS * 32 * LDB * sizeof(float);
+  static constexpr int NCH = RP * 2 / 16;   // 16-byte chunks per bf16 row = lanes per entry
+  static constexpr int EPW = 32 / NCH;      // entries a warp works on at a time
+  static constexpr int WARPS = 24;
 };
 
-// 8 floats from 16 bytes of bf16
-__device__ __forceinline__ void unpack8(const uint4& u, float* f) {
+// 8 floats from 16 bytes of bf16, as 4 pairs
+__device__ __forceinline__ void unpack8(const uint4& u, float2* f) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-  for (int q = 0; q < 4; ++q) {
-    f[2 * q] = __uint_as_float(w[q] << 16);
-    f[2 * q + 1] = __uint_as_float(w[q] & 0xffff0000u);
-  }
+  for (int q = 0; q < 4; ++q) f[q] = make_float2(__uint_as_float(w[q] << 16), __uint_as_float(w[q] & 0xffff0000u));
+}
+
+// d = a b + c on a pair of floats (one packed fp32 FMA, each half rounded as fmaf)
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{.reg .b64 ra, rb, rc, rd;\n\tmov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
 }
 
 template <int RP>
-__global__ void __launch_bounds__(512, 1) sparse_smem_kernel(
+__global__ void __launch_bounds__(32 * SpSmem<RP>::WARPS, 1) sparse_smem_kernel(
     const PanelRow* __restrict__ rows, int64_t nrows, const PanelRow* __restrict__ whole, int64_t nwhole,
     const PanelRow* __restrict__ seg, int64_t nseg, const bf16* __restrict__ Mop, int64_t m0,
     const bf16* __restrict__ Qop, int64_t q0, int64_t K, const int32_t* __restrict__ qidx,
     const float* __restrict__ vals, float* __restrict__ R, float* __restrict__ partials) {
   using C = SpSmem<RP>;
-  constexpr int NCH = C::NCH, LDB = C::LDB;
+  constexpr int NCH = C::NCH, EPW = C::EPW;
   static_assert(RP == 16 || RP == 32, "r_pad 16 or 32");
-  extern __shared__ __align__(16) unsigned char sp_smem[];
-  float* red = reinterpret_cast<float*>(sp_smem);
-  uint4* qs = reinterpret_cast<uint4*>(sp_smem + C::RED_BYTES);
+  extern __shared__ __align__(16) uint4 qs[];
   const uint4* qsrc = reinterpret_cast<const uint4*>(Qop + q0 * RP);
   for (int64_t e = threadIdx.x; e < K * NCH; e += blockDim.x) {
     const int64_t k = e / NCH;
@@ -1081,13 +1088,15 @@ __global__ void __launch_bounds__(512, 1) sparse_smem_kernel(
   }
   cp_async_commit();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  float* rb = red + warp * 32 * LDB;
+  const int ch = lane % NCH, slot = lane / NCH;
   const int64_t nlong = nrows + nwhole, nitems = nlong + nseg;
   const int64_t stride = (int64_t)gridDim.x * C::WARPS;
-  int64_t w = (int64_t)blockIdx.x * C::WARPS + warp;
-  // an item's descriptor, and its indices (relative to the block) and values
-  auto fetch = [&](int64_t x, PanelRow& pr, int* k4, float* s4) {
-    pr = x < nrows ? rows[x] : x < nlong ? whole[x - nrows] : seg[x - nlong];
+  auto desc = [&](int64_t x) -> PanelRow {
+    if (x >= nitems) return PanelRow{0, 0, 0};
+    return x < nrows ? rows[x] : x < nlong ? whole[x - nrows] : seg[x - nlong];
+  };
+  // an item's indices (relative to the block), values and this lane's chunk of m_i
+  auto fetch = [&](const PanelRow& pr, int* k4, float* s4, uint4& mc) {
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       const int e = lane + 32 * t;
@@ -1095,62 +1104,67 @@ __global__ void __launch_bounds__(512, 1) sparse_smem_kernel(
       k4[t] = live ? (int)(__ldg(qidx + pr.beg + e) - q0) : 0;
       s4[t] = live ? __ldg(vals + pr.beg + e) : 0.f;
     }
+    mc = pr.len > 0 ? __ldg(reinterpret_cast<const uint4*>(Mop + (int64_t)pr.row * RP) + ch) : make_uint4(0, 0, 0, 0);
   };
-  PanelRow cur{0, 0, 0};
-  int kk[4] = {0, 0, 0, 0};
-  float ss[4] = {0.f, 0.f, 0.f, 0.f};
-  if (w < nitems) fetch(w, cur, kk, ss);
+  int64_t w = (int64_t)blockIdx.x * C::WARPS + warp;
+  PanelRow cur = desc(w), nxt = desc(w + stride);
+  int kk[4];
+  float ss[4];
+  uint4 mc;
+  fetch(cur, kk, ss, mc);
   cp_async_wait_0();
   __syncthreads();
   for (; w < nitems; w += stride) {
-    PanelRow nxt{0, 0, 0};
-    int kn[4] = {0, 0, 0, 0};
-    float sn[4] = {0.f, 0.f, 0.f, 0.f};
-    if (w + stride < nitems) fetch(w + stride, nxt, kn, sn);
-    float mv[RP], acc[RP];
-    const uint4* mp = reinterpret_cast<const uint4*>(Mop + (int64_t)cur.row * RP);
+    const PanelRow after = desc(w + 2 * stride);
+    int kn[4];
+    float sn[4];
+    uint4 mn;
+    fetch(nxt, kn, sn, mn);
+    float2 mv[4], acc[4];
+    unpack8(mc, mv);
 #pragma unroll
-    for (int c = 0; c < NCH; ++c) unpack8(__ldg(mp + c), mv + 8 * c);
+    for (int q = 0; q < 4; ++q) acc[q] = make_float2(0.f, 0.f);
 #pragma unroll
-    for (int c = 0; c < RP; ++c) acc[c] = 0.f;
+    for (int it = 0; it < 128 / EPW; ++it) {
+      if (it * EPW >= cur.len) break;   // warp-uniform
+      const int e = it * EPW + slot;
+      constexpr int PER = 32 / EPW;       // iterations per batch of 32 entries
+      const int k = __shfl_sync(0xffffffffu, kk[it / PER], e & 31);
+      const float sv = __shfl_sync(0xffffffffu, ss[it / PER], e & 31);
+      const bool live = e < cur.len;
+      uint4 qc = make_uint4(0, 0, 0, 0);
+      if (live) qc = qs[k * NCH + (ch ^ ((k >> 1) & (NCH - 1)))];
+      float2 f[4];
+      unpack8(qc, f);
+      // the even and the odd columns' products summed separately, then added
+      float2 d2 = make_float2(0.f, 0.f);
 #pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      if (32 * t >= cur.len) break;   // warp-uniform
-      if (lane + 32 * t < cur.len) {
-        const int k = kk[t];
-        uint4 qc[NCH];
+      for (int q = 0; q < 4; ++q) d2 = ffma2(mv[q], f[q], d2);
+      float dot = d2.x + d2.y;
 #pragma unroll
-        for (int j = 0; j < NCH; ++j) qc[j] = qs[k * NCH + (j ^ ((k >> 1) & (NCH - 1)))];
-        float dot = 0.f;
+      for (int o = 1; o < NCH; o <<= 1) dot += __shfl_xor_sync(0xffffffffu, dot, o);
+      if (live) {
+        const float cv = sv - fminf(0.f, dot);
+        const float2 c2 = make_float2(cv, cv);
 #pragma unroll
-        for (int j = 0; j < NCH; ++j) {
-          float f[8];
-          unpack8(qc[j], f);
-#pragma unroll
-          for (int q = 0; q < 8; ++q) dot = fmaf(mv[8 * j + q], f[q], dot);
-        }
-        const float cv = ss[t] - fminf(0.f, dot);
-#pragma unroll
-        for (int j = 0; j < NCH; ++j) {
-          float f[8];
-          unpack8(qc[j], f);
-#pragma unroll
-          for (int q = 0; q < 8; ++q) acc[8 * j + q] = fmaf(cv, f[q], acc[8 * j + q]);
-        }
+        for (int q = 0; q < 4; ++q) acc[q] = ffma2(c2, f[q], acc[q]);
       }
     }
 #pragma unroll
-    for (int c = 0; c < RP; ++c) rb[lane * LDB + c] = acc[c];
-    __syncwarp();
-    float* out = w < nlong ? R + ((int64_t)cur.row - m0) * RP : partials + (w - nlong) * RP;
-    if (lane < RP) {
-      float sum = 0.f;
-#pragma unroll 8
-      for (int l = 0; l < 32; ++l) sum += rb[l * LDB + lane];
-      out[lane] = sum;
+    for (int o = NCH; o < 32; o <<= 1)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        acc[q].x += __shfl_xor_sync(0xffffffffu, acc[q].x, o);
+        acc[q].y += __shfl_xor_sync(0xffffffffu, acc[q].y, o);
+      }
+    if (slot == 0) {
+      float* out = (w < nlong ? R + ((int64_t)cur.row - m0) * RP : partials + (w - nlong) * RP) + 8 * ch;
+      *(float4*)out = make_float4(acc[0].x, acc[0].y, acc[1].x, acc[1].y);
+      *(float4*)(out + 4) = make_float4(acc[2].x, acc[2].y, acc[3].x, acc[3].y);
     }
-    __syncwarp();   // the buffer is rewritten by the next item
     cur = nxt;
+    nxt = after;
+    mc = mn;
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       kk[t] = kn[t];
@@ -1818,12 +1832,12 @@ static bool launch_sparse_smem(const StepArgs& a, const PanelRow* rows, int64_t 
   static std::atomic<int> attr[kMaxDevices];
   if (!per_device(attr, [] {
         return cudaFuncSetAttribute(sparse_smem_kernel<RP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)(C::RED_BYTES + kSparseQBytes)) == cudaSuccess ? 1 : 0;
+                                    (int)kSparseQBytes) == cudaSuccess ? 1 : 0;
       }))
     return false;
   const int64_t nitems = nrows + nwhole + nseg;
   const int64_t grid = std::min<int64_t>(a.num_sms, (nitems + C::WARPS - 1) / C::WARPS);
-  const size_t smem = C::RED_BYTES + (size_t)a.K * RP * sizeof(bf16);
+  const size_t smem = (size_t)a.K * RP * sizeof(bf16);
   sparse_smem_kernel<RP><<<(unsigned)grid, 32 * C::WARPS, smem, s>>>(rows, nrows, whole, nwhole, seg, nseg, a.fm->hi,
                                                                     a.m0, a.fq->hi, a.q0, a.K, qidx, vals, R,
                                                                     partials);
