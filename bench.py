@@ -50,7 +50,7 @@ WORKLOADS = {
 # while the kernel's sources hash to the digest recorded with it (else null)
 DENSE_TRAFFIC = {
     # (workload, precision, epilogue): (bytes per launch, dense_source_digest() of the code measured)
-    ("connectome-139255-r64", "bf16", "z"): (18397952, "fa2f9dd428e48a57"),
+    ("connectome-139255-r64", "bf16", "z"): (18395392, "5094500fd5d511bc"),
 }
 
 
@@ -91,11 +91,15 @@ def dense_source_digest():
 
 
 def support_bytes_per_sweep(wl, elem_bytes):
-    """Algorithmic bytes of the support term over one sweep (each step once):
-    per support entry its index and value (8 B) and the q row (r elements);
-    per M-side row with support in the step's panel its m row (r elements)
-    and its row of Rs (r fp32 values, written).  Every nonzero is in one
-    column step and one row step; the panel rows are counted per step."""
+    """Algorithmic DRAM bytes of the support term over one sweep (each step
+    once), and the q-row gathers on top of them.  DRAM: per support entry its
+    index and value (8 B); per M-side row with support in the step's panel
+    its m row (r elements) and its row of Rs (r fp32 values, written); each
+    step's Q-side block once (r elements per row: over a sweep, both factors
+    once).  Gathers: per support entry its q row (r elements), which the
+    kernels read from L2 or from the block staged in shared memory.  Every
+    nonzero is in one column step and one row step; the panel rows are
+    counted per step."""
     import numpy as np
     S = wl.S
     rows = np.repeat(np.arange(S.m, dtype=np.int64), np.diff(S.row_ptr))
@@ -104,7 +108,8 @@ def support_bytes_per_sweep(wl, elem_bytes):
     col_pairs = np.unique(rows * (-(-S.n // wl.block_cols)) + cols // wl.block_cols).size
     row_pairs = np.unique(cols * (-(-S.m // wl.block_rows)) + rows // wl.block_rows).size
     nnz = int(S.row_ptr[-1])
-    return 2 * nnz * (8 + elem_bytes * wl.r) + (col_pairs + row_pairs) * (elem_bytes * wl.r + 4 * wl.r)
+    dram = 2 * nnz * 8 + (col_pairs + row_pairs) * (elem_bytes * wl.r + 4 * wl.r) + (S.m + S.n) * elem_bytes * wl.r
+    return dram, 2 * nnz * elem_bytes * wl.r
 
 
 def measure_support(sol, wl, N):
@@ -429,10 +434,11 @@ def main():
             pk, pk_kind = peaks()
             hbm = pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
             ms, nst = measure_support(sol, wl, N)
-            by = support_bytes_per_sweep(wl, 2 if prec == N.NMD_BF16 else 4)
-            print(json.dumps({"metric": "support term alone, algorithmic GB/s", "value": by / (ms / 1e3) / 1e9,
+            by, gb = support_bytes_per_sweep(wl, 2 if prec == N.NMD_BF16 else 4)
+            print(json.dumps({"metric": "support term alone, algorithmic DRAM GB/s", "value": by / (ms / 1e3) / 1e9,
                               "unit": "GB/s", "frac": by / (ms / 1e3) / 1e9 / hbm, "ms_per_sweep": ms,
-                              "steps": nst, "bytes_per_sweep": by, "workload": wl.name,
+                              "steps": nst, "bytes_per_sweep": by, "gather_bytes_per_sweep": gb,
+                              "with_gathers_gbs": (by + gb) / (ms / 1e3) / 1e9, "workload": wl.name,
                               "precision": args.precision}))
         rep.close()
         return 0
@@ -544,15 +550,20 @@ def main():
     # support term alone (HBM roofline by algorithmic bytes)
     hbm = pk.get("hbm_gbs", FALLBACK_PEAKS["hbm_gbs"])
     sp_ms, sp_steps = measure_support(sol, wl, N)
-    sp_bytes = support_bytes_per_sweep(wl, 2 if prec == N.NMD_BF16 else 4)
+    sp_bytes, sp_gather = support_bytes_per_sweep(wl, 2 if prec == N.NMD_BF16 else 4)
     sp_gbs = sp_bytes / (sp_ms / 1e3) / 1e9
     roofline_sparse = {"bound": "hbm", "kernel": "support term (sparse_group_kernel, sparse_long_kernel, "
-                                                 "sparse_reduce_kernel), alone",
+                                                 "sparse_reduce_kernel; sparse_smem_kernel where the Q-side "
+                                                 "block fits in shared memory), alone",
                        "achieved": sp_gbs, "peak": hbm, "unit": "GB/s", "frac": sp_gbs / hbm,
                        "traffic": None, "peak_kind": "%s copy bandwidth" % pk_kind,
                        "bytes_per_sweep": sp_bytes, "ms_per_sweep": sp_ms, "steps": sp_steps,
-                       "bytes_rule": "per support entry 8 B + r operand elements; per panel row r operand "
-                                     "elements + 4 r B (Rs); operands bf16 in the bf16 mode"}
+                       "bytes_rule": "DRAM: per support entry 8 B; per panel row r operand elements + 4 r B "
+                                     "(Rs); each step's Q-side block once; operands bf16 in the bf16 mode",
+                       "gather_bytes_per_sweep": sp_gather,
+                       "with_gathers_gbs": (sp_bytes + sp_gather) / (sp_ms / 1e3) / 1e9,
+                       "gather_rule": "per support entry the r operand elements of its q row (from L2 or "
+                                      "shared memory)"}
 
     # the fp32-accurate mode on the same workload and start, same run
     modes = None
