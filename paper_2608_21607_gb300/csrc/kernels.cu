@@ -968,10 +968,12 @@ __global__ void __launch_bounds__(256) sparse_reduce_kernel(const PanelRow* __re
 // columns 4 tx + 4 TX g (g < CPT / 4), so that a quarter warp reads 128
 // contiguous bytes of G^{-1} and a half warp writes whole 256-byte rows.
 // ---------------------------------------------------------------------------
-template <int RP, bool TC = false>
+template <int RP, bool TC = false, int TRT = 64>
 struct UpdCfg {
   static constexpr int CW = RP <= 128 ? RP : 128;   // output columns per block
-  static constexpr int TR = RP <= 128 ? 64 : 32;    // rows per tile
+  // rows per tile: on the tensor cores 64, or 32 for launches with fewer
+  // 64-row tiles than SMs (the rows the next step reads: more blocks at once)
+  static constexpr int TR = TC ? TRT : (RP <= 128 ? 64 : 32);
   static constexpr int TY = TR / 4;                  // row groups of four
   static constexpr int TX = 256 / TY;                // column groups
   static constexpr int CPT = CW / TX;                // columns per thread (1, 2, 4 or 8)
@@ -984,7 +986,10 @@ struct UpdCfg {
   static constexpr size_t SMEM = TC ? (size_t)TR * SR * sizeof(float) + 2 * (size_t)RP * SB * sizeof(bf16)
                                     : ((size_t)RP * CW + 2 * (size_t)TR * RP) * sizeof(float);
   static_assert(CPT >= 1 && (CPT < 4 || CPT % 4 == 0), "column split");
-  static_assert(!TC || (CW == RP && TR == 64), "tensor-core product: one block column, tiles of 64 rows");
+  // tensor-core product: TR / 16 row groups of warps, each warp RP / (8 /
+  // (TR / 16)) columns (at least one 8-column tile)
+  static constexpr int RG = TR / 16, WC = TC ? RP / (8 / RG) : 8;
+  static_assert(!TC || (CW == RP && (TR == 64 || TR == 32) && WC >= 8), "tensor-core product tiling");
 };
 
 template <int CPT, int TX>
@@ -1173,7 +1178,7 @@ __global__ void __launch_bounds__(32 * SpSmem<RP>::WARPS, 1) sparse_smem_kernel(
   }
 }
 
-template <int RP, bool TC>
+template <int RP, bool TC, int TRT>
 __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* __restrict__ M, bf16* __restrict__ Mhi,
                                                      bf16* __restrict__ Mlo, bf16* __restrict__ Mlo2,
                                                      float* __restrict__ E, int64_t m0, int64_t rows,
@@ -1183,7 +1188,7 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
                                                      const bf16* __restrict__ gsplit, float eta,
                                                      float gamma, int momentum, int delta_form, int write_lo,
                                                      int* __restrict__ status) {
-  using C = UpdCfg<RP, TC>;
+  using C = UpdCfg<RP, TC, TRT>;
   constexpr int NV = C::TR * RP / 4 / 256;   // float4 of a tile per thread
   constexpr int CW = C::CW, TR = C::TR, TX = C::TX, CPT = C::CPT, SR = C::SR;
   extern __shared__ __align__(16) float sm[];
@@ -1294,12 +1299,12 @@ __global__ void __launch_bounds__(256, (RP <= 64 ? 3 : 1)) update_kernel(float* 
     if constexpr (TC) {
       // X = (R + Rs) G^{-1} on the tensor cores: both factors as hi + lo
       // bf16 pieces, three products (lo hi, hi lo, hi hi; lo lo dropped), fp32
-      // accumulation.  Warp w takes rows 16 (w % 4) .. + 15 and columns
-      // (w / 4) RP / 2 .. + RP / 2 - 1 of the tile's product.
-      constexpr int NT = RP / 16;   // 8-column tiles per warp (and 16-wide k steps)
+      // accumulation.  Warp w takes rows 16 (w % RG) .. + 15 and columns
+      // (w / RG) WC .. + WC - 1 of the tile's product.
+      constexpr int RG = C::RG, WC = C::WC, NT = WC / 8;   // NT: 8-column tiles per warp
       float* Rt = Rb;
       const int lane = threadIdx.x % 32, warp = threadIdx.x / 32, g = lane / 4, c2 = 2 * (lane % 4);
-      const int r0 = 16 * (warp % 4), n0 = (warp / 4) * (RP / 2);
+      const int r0 = 16 * (warp % RG), n0 = (warp / RG) * WC;
       float acc[NT][4];
 #pragma unroll
       for (int n = 0; n < NT; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
@@ -1898,20 +1903,20 @@ int launch_sparse(const StepArgs& a, const PanelRow* rows, int64_t nrows, const 
   return (nrows > 0) + (nwhole > 0) + 2 * (nseg > 0);
 }
 
-template <int RP, bool TC>
+template <int RP, bool TC, int TRT = 64>
 static void update_rp(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
                       const bf16* gsplit, float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
-  using C = UpdCfg<RP, TC>;
+  using C = UpdCfg<RP, TC, TRT>;
   // the attribute and the occupancy belong to the current device
   static std::atomic<int> cache[kMaxDevices];
   const int per_sm = per_device(cache, [] {
     int n = 0;
-    cudaFuncSetAttribute(update_kernel<RP, TC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
+    cudaFuncSetAttribute(update_kernel<RP, TC, TRT>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)C::SMEM);
     // at r_pad <= 64 the largest shared-memory configuration, like the dense
     // kernel's, so that an SM running update blocks can take a dense CTA and
     // vice versa
-    if (RP <= 64) cudaFuncSetAttribute(update_kernel<RP, TC>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, update_kernel<RP, TC>, 256, C::SMEM) != cudaSuccess ||
+    if (RP <= 64) cudaFuncSetAttribute(update_kernel<RP, TC, TRT>, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, update_kernel<RP, TC, TRT>, 256, C::SMEM) != cudaSuccess ||
         n < 1)
       n = 1;
     return n;
@@ -1924,7 +1929,7 @@ static void update_rp(const StepArgs& a, const float* R, const float* Rs, const 
   const int64_t tiles = (a.M + C::TR - 1) / C::TR;
   dim3 grid((unsigned)std::min<int64_t>(tiles, (int64_t)a.num_sms * per_sm * 65535), RP / C::CW);
   const Factor& f = *a.fm;
-  update_kernel<RP, TC><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, flags, Ginv,
+  update_kernel<RP, TC, TRT><<<grid, 256, C::SMEM, s>>>(f.master, f.hi, f.lo, f.lo2, f.E, a.m0, a.M, R, Rs, flags, Ginv,
                                                    gsplit, eta, gamma, momentum, a.epilogue == NMD_EPI_DELTA,
                                                    a.precision == NMD_FP32, status);
 }
@@ -1936,10 +1941,14 @@ static void update_rp(const StepArgs& a, const float* R, const float* Rs, const 
 void launch_update(const StepArgs& a, const float* R, const float* Rs, const uint8_t* flags, const float* Ginv,
                    const bf16* gsplit, float eta, float gamma, bool momentum, int* status, cudaStream_t s) {
   const bool tc = a.precision == NMD_BF16 && gsplit != nullptr;
+  // 32-row tiles where the rows fill fewer 64-row tiles than there are SMs
+  const bool small = a.M < (int64_t)a.num_sms * 64;
   switch (a.rp) {
-#define NMD_UPD(RPV)                                                                      \
-  (tc ? update_rp<RPV, true>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, s) \
-      : update_rp<RPV, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, s))
+#define NMD_UPD(RPV)                                                                                          \
+  (!tc ? update_rp<RPV, false>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, s)                 \
+       : (small && RPV >= 32) ? update_rp<RPV, true, (RPV >= 32 ? 32 : 64)>(a, R, Rs, flags, Ginv, gsplit, eta, \
+                                                                            gamma, momentum, status, s)        \
+                              : update_rp<RPV, true>(a, R, Rs, flags, Ginv, gsplit, eta, gamma, momentum, status, s))
     case 16: NMD_UPD(16); break;
     case 32: NMD_UPD(32); break;
     case 64: NMD_UPD(64); break;
