@@ -68,15 +68,17 @@ typedef enum { NMD_ALTERNATE = 0, NMD_PHASED = 1 } nmd_order;
  *               (L = M_hi Q_hi^T and R = P Q_hi on the tcgen05 tensor cores,
  *               fp32 accumulation), the support term (on the hi pieces) and
  *               the Gram matrix G = Q_hi^T Q_hi all use them, so the rounding
- *               is not a coherent error between R and G; the update itself is
- *               applied to the fp32 masters;
+ *               is not a coherent error between R and G; the solve X = (R +
+ *               Rs) G^{-1} runs on the tensor cores with R + Rs and G^{-1} as
+ *               hi + lo bf16 pieces (three products, fp32 accumulation), and
+ *               the update is applied to the fp32 masters;
  *   NMD_FP32 -- fp32-accurate: L = M_hi Q_hi^T + M_hi Q_lo^T + M_lo Q_hi^T,
  *               P = P_hi + P_lo (two bf16 pieces), R = P_hi (Q_hi + Q_lo +
  *               Q_lo2) + P_lo Q_hi on the tensor cores; the support term and
  *               G from the fp32 masters;
  *   NMD_SIMT -- plain fp32 FMA on the CUDA cores (slow; reference path).
  * Gram matrices are formed in fp32, factored in fp32 (L D L^T Cholesky form),
- * updates are fp32; loss reductions are fp64. */
+ * updates are fp32 (the NMD_BF16 solve as above); loss reductions are fp64. */
 typedef enum { NMD_BF16 = 0, NMD_FP32 = 1, NMD_SIMT = 2 } nmd_precision;
 
 /* Form of the dense contraction (both give the same update, Sec. 3.2):
