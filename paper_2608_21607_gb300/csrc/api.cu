@@ -1039,6 +1039,34 @@ nmd_status nmd_create(int64_t m, int64_t n, int32_t r, const int64_t* row_ptr,
   return NMD_OK;
 }
 
+// A copy of `bytes` in four pieces on the handle's four streams, so that
+// several copy engines move it at once (a host <-> device copy on one
+// engine stays well below what the link carries); ordered after the earlier
+// work of `s`, which continues after all four pieces.  Used outside sweeps
+// only (it borrows the sweep's streams and events).
+nmd_status copy_split(nmd_handle* h, void* dst, const void* src, size_t bytes, cudaMemcpyKind kind, cudaStream_t s) {
+  constexpr int kPieces = 4;
+  if (bytes < ((size_t)8 << 20)) {
+    CK(h, cudaMemcpyAsync(dst, src, bytes, kind, s));
+    return NMD_OK;
+  }
+  cudaStream_t t[kPieces] = {s, h->side, h->side2, h->aux};
+  cudaEvent_t done[kPieces] = {nullptr, h->ev_join, h->ev_join2, h->ev_prio};
+  const size_t piece = (bytes / kPieces + 255) & ~(size_t)255;
+  CK(h, cudaEventRecord(h->ev_fork, s));
+  for (int q = 0; q < kPieces; ++q) {
+    const size_t off = (size_t)q * piece;
+    if (off >= bytes) break;
+    if (q > 0) CK(h, cudaStreamWaitEvent(t[q], h->ev_fork, 0));
+    CK(h, cudaMemcpyAsync((char*)dst + off, (const char*)src + off, std::min(piece, bytes - off), kind, t[q]));
+    if (q > 0) {
+      CK(h, cudaEventRecord(done[q], t[q]));
+      CK(h, cudaStreamWaitEvent(s, done[q], 0));
+    }
+  }
+  return NMD_OK;
+}
+
 nmd_status nmd_set_factors(nmd_handle* h, const float* W, const float* H, int on_device) {
   if (!h || !W || !H) return fail(h, NMD_ERR_INVALID, "NULL argument to nmd_set_factors");
   DeviceScope dg(h);
@@ -1047,11 +1075,13 @@ nmd_status nmd_set_factors(nmd_handle* h, const float* W, const float* H, int on
   cudaStream_t s = h->stream;
   cudaMemcpyKind kind = on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
   // stage through R (max(m, n) x rp floats >= m x r and r x n)
-  CK(h, cudaMemcpyAsync(h->ws.R, W, (size_t)h->m * h->r * 4, kind, s));
+  nmd_status cs = copy_split(h, h->ws.R, W, (size_t)h->m * h->r * 4, kind, s);
+  if (cs != NMD_OK) return cs;
   launch_pack(h->ws.R, false, h->m, h->r, h->rp, h->W, s);
   h->launches++;
-  CK(h, cudaMemcpyAsync(h->ws.R, H, (size_t)h->n * h->r * 4, kind, s));
-  launch_pack(h->ws.R, true, h->n, h->r, h->rp, h->B, s);
+  // H goes to the second copy of R, so that its copy overlaps W's packing
+  if ((cs = copy_split(h, h->ws.R2, H, (size_t)h->n * h->r * 4, kind, s)) != NMD_OK) return cs;
+  launch_pack(h->ws.R2, true, h->n, h->r, h->rp, h->B, s);
   h->launches++;
   CK(h, cudaMemsetAsync(h->W.E, 0, (size_t)h->m * h->rp * 4, s));
   CK(h, cudaMemsetAsync(h->B.E, 0, (size_t)h->n * h->rp * 4, s));
@@ -1070,12 +1100,14 @@ nmd_status nmd_get_factors(nmd_handle* h, float* W, float* H, int on_device) {
   if (W) {
     launch_unpack(h->W.master, false, h->m, h->r, h->rp, h->ws.R, s);
     h->launches++;
-    CK(h, cudaMemcpyAsync(W, h->ws.R, (size_t)h->m * h->r * 4, kind, s));
+    nmd_status cs = copy_split(h, W, h->ws.R, (size_t)h->m * h->r * 4, kind, s);
+    if (cs != NMD_OK) return cs;
   }
   if (H) {
-    launch_unpack(h->B.master, true, h->n, h->r, h->rp, h->ws.R, s);
+    launch_unpack(h->B.master, true, h->n, h->r, h->rp, h->ws.R2, s);
     h->launches++;
-    CK(h, cudaMemcpyAsync(H, h->ws.R, (size_t)h->n * h->r * 4, kind, s));
+    nmd_status cs = copy_split(h, H, h->ws.R2, (size_t)h->n * h->r * 4, kind, s);
+    if (cs != NMD_OK) return cs;
   }
   CK(h, cudaStreamSynchronize(s));
   return st;
