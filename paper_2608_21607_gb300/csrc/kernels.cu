@@ -1047,7 +1047,9 @@ __device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uin
 // to the lanes of their slot by shuffles; an item's indices, values and m_i
 // are loaded while the previous item is computed, its descriptor two items
 // ahead.  In shared memory, 16-byte chunk j of row k sits at chunk j ^ ((k >>
-// 1) & (NCH - 1)).
+// 1) & (NCH - 1)).  Every index lies in [q0, q0 + K): the panel lists are
+// built at create from the CSR cut to the block's columns (rows, for row
+// steps), as for the kernels above.
 // ---------------------------------------------------------------------------
 constexpr size_t kSparseQBytes = 200 * 1024;
 
